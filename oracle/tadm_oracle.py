@@ -1,0 +1,460 @@
+"""Plain fp64 CPU oracle of TADM's anchor-cache reverse-diffusion sampling loop.
+
+TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and the
+CPU-baseline leg of ``bench.py`` import this module.  The CUDA library never
+calls it and shares no code with it; both only consume the same seeded inputs
+(``workloads``).
+
+What it computes (paper section / equation it follows):
+
+* Model decomposition ``c = S(z)``, ``h = A(c)``, ``x = D(Phi(c, h))``: §3.1.
+* Stale-anchor fusion, general form ``h~ = h' + g * Delta``: §3.2,
+  Eq. (stale-anchor-fusion).  Two instances:
+    - gated residual MLP (TADM:Pretraining): App. C.2;
+    - paired attention with cached shallow state (TADM:Post-train): App. C.1,
+      Eqs. (paired-attention-difference) and (stale-anchor-fusion-app).
+* Anchor-cache inference loop: Alg. 1 (Anchor-Cache Inference), §3.3;
+  transformer-layer cost: Eq. (anchor-cache-compute).
+* Masked-diffusion reverse step with zero-masking and carry-over unmasking:
+  App. B.1.1, Eq. (mdlm-posterior-unk).
+* Block diffusion with a KV cache over committed blocks (the encoder prefills
+  the context causally, the decoder denoises the active block
+  bidirectionally): App. C.1, "Architecture Details".
+* Backbone layer: pre-norm transformer (RMSNorm, RoPE, multi-head attention
+  with grouped KV heads, SwiGLU / GeGLU FFN), the layer type the workloads
+  name; the paper treats it as a black box.
+
+Readings where the paper is silent (each one is listed in the design doc):
+* sampler P: confidence top-k within the active block; conf = max softmax
+  probability over the vocabulary without MASK, k_n = floor((n+1)G/T) -
+  floor(nG/T), ties broken toward the lower position;
+* refresh at n = T - i with n mod K == 0, counter restarting per block;
+* A3 LayerNorms are LayerNorm(eps 1e-6) with affine terms, GELU is the erf
+  form; GeGLU uses the tanh-approximate GELU;
+* A4: J = [Z, U] and F = [U; Z0; Z - Z0; M] concatenate features; the gate
+  MLP hidden width is r; the mixer attention has no positional encoding;
+* h_cache is the raw residual stream leaving A (no final norm);
+* commit / prefill passes run S, A, Phi(c, A(c)), D fresh, with causal
+  attention inside the block being committed.
+
+All arithmetic is float64.  Weights arrive as float32 arrays or raw bf16 bit
+arrays and are widened exactly.
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, field
+from typing import Dict, List, Optional
+
+import numpy as np
+
+NEG_INF = -np.inf
+
+
+# ---------------------------------------------------------------------------
+# elementary ops (textbook definitions)
+# ---------------------------------------------------------------------------
+def widen(w: np.ndarray) -> np.ndarray:
+    """Exact float64 values of a float32 or raw-bf16-bits array."""
+    if w.dtype == np.uint16:
+        return (w.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    return w.astype(np.float64)
+
+
+def rms_norm(x: np.ndarray, gain: np.ndarray, eps: float) -> np.ndarray:
+    """x / sqrt(mean(x^2) + eps) * gain, over the last axis."""
+    return x / np.sqrt(np.mean(x * x, axis=-1, keepdims=True) + eps) * gain
+
+
+def layer_norm(x: np.ndarray, w: np.ndarray, b: np.ndarray, eps: float) -> np.ndarray:
+    """(x - mean) / sqrt(var + eps) * w + b, over the last axis (biased variance)."""
+    mu = np.mean(x, axis=-1, keepdims=True)
+    var = np.mean((x - mu) ** 2, axis=-1, keepdims=True)
+    return (x - mu) / np.sqrt(var + eps) * w + b
+
+
+def sigmoid(x: np.ndarray) -> np.ndarray:
+    return 1.0 / (1.0 + np.exp(-x))
+
+
+def silu(x: np.ndarray) -> np.ndarray:
+    return x * sigmoid(x)
+
+
+try:  # library erf when available, else the scalar one from the C library
+    from scipy.special import erf as _erf
+except ImportError:  # pragma: no cover
+    def _erf(x: np.ndarray) -> np.ndarray:
+        return np.vectorize(math.erf, otypes=[np.float64])(x)
+
+
+def gelu_erf(x: np.ndarray) -> np.ndarray:
+    """GELU, exact form x * Phi(x) (Hendrycks & Gimpel 2016)."""
+    return 0.5 * x * (1.0 + _erf(x / math.sqrt(2.0)))
+
+
+def gelu_tanh(x: np.ndarray) -> np.ndarray:
+    """GELU, tanh approximation (Hendrycks & Gimpel 2016)."""
+    return 0.5 * x * (1.0 + np.tanh(math.sqrt(2.0 / math.pi) * (x + 0.044715 * x ** 3)))
+
+
+def linear(x: np.ndarray, w: np.ndarray, b: Optional[np.ndarray] = None) -> np.ndarray:
+    """y = x W^T (+ b); W is [out, in]."""
+    y = x @ w.T
+    return y if b is None else y + b
+
+
+def rope(x: np.ndarray, pos: np.ndarray, theta: float) -> np.ndarray:
+    """Rotary position embedding, rotate-half pairing (j, j + hd/2).
+
+    x: [H, L, hd]; pos: [L] absolute positions.
+    """
+    hd = x.shape[-1]
+    half = hd // 2
+    j = np.arange(half, dtype=np.float64)
+    inv_freq = theta ** (-2.0 * j / hd)
+    ang = pos.astype(np.float64)[:, None] * inv_freq[None, :]
+    c, s = np.cos(ang), np.sin(ang)
+    x1, x2 = x[..., :half], x[..., half:]
+    return np.concatenate([x1 * c - x2 * s, x2 * c + x1 * s], axis=-1)
+
+
+def attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, q_pos: np.ndarray, k_pos: np.ndarray,
+              causal: bool) -> np.ndarray:
+    """softmax(q k^T / sqrt(hd)) v with grouped KV heads.
+
+    q: [Hq, Lq, hd]; k, v: [Hkv, Lk, hd]; query head h reads KV head
+    h // (Hq / Hkv).  causal: key allowed iff k_pos <= q_pos.
+    Returns [Hq, Lq, hd].
+    """
+    Hq, Lq, hd = q.shape
+    Hkv = k.shape[0]
+    group = Hq // Hkv
+    out = np.empty_like(q)
+    for h in range(Hq):
+        kh, vh = k[h // group], v[h // group]
+        s = q[h] @ kh.T / math.sqrt(hd)
+        if causal:
+            s = np.where(k_pos[None, :] <= q_pos[:, None], s, NEG_INF)
+        s = s - np.max(s, axis=-1, keepdims=True)
+        p = np.exp(s)
+        p = p / np.sum(p, axis=-1, keepdims=True)
+        out[h] = p @ vh
+    return out
+
+
+# ---------------------------------------------------------------------------
+# the sampler P (confidence top-k in the active block)
+# ---------------------------------------------------------------------------
+def confidence(logits: np.ndarray, mask_id: int):
+    """Per row: tok = argmax over v != MASK (lowest id on ties), conf = p(tok).
+
+    Zero-masking (App. B.1.1): the MASK logit is excluded, so the model never
+    predicts MASK.  conf = 1 / sum_v exp(l_v - l_max), in float64.
+    """
+    l = np.array(logits, dtype=np.float64, copy=True)
+    l[..., mask_id] = NEG_INF
+    tok = np.argmax(l, axis=-1)
+    m = np.take_along_axis(l, tok[..., None], axis=-1)
+    conf = 1.0 / np.sum(np.exp(l - m), axis=-1)
+    return conf, tok.astype(np.int64)
+
+
+def unmask_count(n: int, T: int, G: int) -> int:
+    """k_n = floor((n+1) G / T) - floor(n G / T): G masked positions spread
+    evenly over T steps, all of them committed by the last step."""
+    return (n + 1) * G // T - n * G // T
+
+
+def select_topk(z: np.ndarray, conf: np.ndarray, k: int, mask_id: int) -> np.ndarray:
+    """Positions to unmask in one sequence: the k masked positions of largest
+    conf, ties toward the lower position.  Carry-over (App. B.1.1): positions
+    already holding a token are never candidates."""
+    cand = np.nonzero(z == mask_id)[0]
+    if k <= 0 or cand.size == 0:
+        return np.zeros(0, dtype=np.int64)
+    order = np.lexsort((cand, -conf[cand]))  # primary: conf desc, secondary: position asc
+    return cand[order[:k]]
+
+
+def layer_cost(L_S: int, L_A: int, L_D: int, T: int, K: int):
+    """Eq. (anchor-cache-compute): (C_full, C_cache) transformer-layer calls."""
+    c_full = T * (L_S + L_A + L_D)
+    c_cache = T * (L_S + L_D) + (-(-T // K)) * L_A
+    return c_full, c_cache
+
+
+# ---------------------------------------------------------------------------
+# the model
+# ---------------------------------------------------------------------------
+@dataclass
+class _Seq:
+    """Per-sequence KV context (block mode): one (K, V) pair per layer."""
+    ctx_len: int = 0
+    kv: Dict[str, List[np.ndarray]] = field(default_factory=dict)
+
+
+class Oracle:
+    """fp64 reference of the TADM networks and the Alg. 1 loop.
+
+    ``model`` is any object with the attributes vocab, d_model, n_heads,
+    n_kv_heads, head_dim, ffn, glu, n_shared, n_anchor, n_denoise, fusion,
+    fusion_rank, fusion_heads, tied_lm_head, norm_eps, rope_theta.
+    ``weights`` maps tensor names to arrays (float32 or raw bf16 bits).
+    """
+
+    def __init__(self, model, weights: Dict[str, np.ndarray], cache_f64_limit: int = 2 << 30):
+        self.m = model
+        self.mask_id = model.vocab - 1
+        self._raw = weights
+        total = sum(w.size for w in weights.values())
+        self._keep = total * 8 <= cache_f64_limit
+        self._w64: Dict[str, np.ndarray] = {}
+        self.counters = {"shared": 0, "anchor": 0, "denoise": 0, "anchor_calls": 0, "steps": 0}
+        self.refresh_log: List[tuple] = []
+
+    def W(self, name: str) -> np.ndarray:
+        if name in self._w64:
+            return self._w64[name]
+        w = widen(self._raw[name])
+        if self._keep:
+            self._w64[name] = w
+        return w
+
+    # -- backbone layer (pre-norm) ------------------------------------------
+    def layer(self, name: str, x: np.ndarray, pos: np.ndarray, seq: Optional[_Seq], causal: bool,
+              keep_kv: bool) -> np.ndarray:
+        """x <- x + Wo Attn(RoPE(Q), RoPE(K), V) from RMSNorm(x); then
+        x <- x + Wdown (act(Wg n) * (Wu n)) with n = RMSNorm(x).
+
+        Keys are the context cached in ``seq`` (committed positions) followed
+        by the rows of x.  With ``keep_kv`` the rows' K, V are appended to the
+        context (commit / prefill pass).
+        """
+        m = self.m
+        hd, Hq, Hkv, F = m.head_dim, m.n_heads, m.n_kv_heads, m.ffn
+        L = x.shape[0]
+        n = rms_norm(x, self.W(name + "attn_norm"), m.norm_eps)
+        qkv = linear(n, self.W(name + "wqkv"))
+        q = qkv[:, : Hq * hd].reshape(L, Hq, hd).transpose(1, 0, 2)
+        k = qkv[:, Hq * hd: (Hq + Hkv) * hd].reshape(L, Hkv, hd).transpose(1, 0, 2)
+        v = qkv[:, (Hq + Hkv) * hd:].reshape(L, Hkv, hd).transpose(1, 0, 2)
+        q = rope(q, pos, m.rope_theta)
+        k = rope(k, pos, m.rope_theta)
+        if seq is not None and name in seq.kv:
+            kc, vc = seq.kv[name]
+            k_all = np.concatenate([kc, k], axis=1)
+            v_all = np.concatenate([vc, v], axis=1)
+            k_pos = np.concatenate([np.arange(kc.shape[1]), pos])
+        else:
+            k_all, v_all, k_pos = k, v, pos
+        o = attention(q, k_all, v_all, pos, k_pos, causal)
+        x = x + linear(o.transpose(1, 0, 2).reshape(L, Hq * hd), self.W(name + "wo"))
+        n = rms_norm(x, self.W(name + "ffn_norm"), m.norm_eps)
+        gu = linear(n, self.W(name + "wgu"))
+        g, u = gu[:, :F], gu[:, F:]
+        act = silu(g) if m.glu == "swiglu" else gelu_tanh(g)
+        x = x + linear(act * u, self.W(name + "wdown"))
+        if keep_kv and seq is not None:
+            if name in seq.kv:
+                kc, vc = seq.kv[name]
+                seq.kv[name] = [np.concatenate([kc, k], axis=1), np.concatenate([vc, v], axis=1)]
+            else:
+                seq.kv[name] = [k, v]
+        return x
+
+    def stack(self, net: str, n_layers: int, x, pos, seq, causal, keep_kv, count=True):
+        for i in range(n_layers):
+            x = self.layer(f"{net}.{i}.", x, pos, seq, causal, keep_kv)
+        if count:
+            self.counters[net] += n_layers
+        return x
+
+    # -- S, A, D (§3.1) -----------------------------------------------------
+    def S(self, z: np.ndarray, pos, seq, causal=False, keep_kv=False, count=True) -> np.ndarray:
+        """Shared network: token embedding, then L_S backbone layers."""
+        c = self.W("embed")[z.astype(np.int64)]
+        return self.stack("shared", self.m.n_shared, c, pos, seq, causal, keep_kv, count)
+
+    def A(self, c, pos, seq, causal=False, keep_kv=False, count=True) -> np.ndarray:
+        """Anchor network: L_A backbone layers; the raw residual stream is h."""
+        return self.stack("anchor", self.m.n_anchor, c, pos, seq, causal, keep_kv, count)
+
+    def D_hidden(self, h, pos, seq, causal=False, keep_kv=False, count=True) -> np.ndarray:
+        return self.stack("denoise", self.m.n_denoise, h, pos, seq, causal, keep_kv, count)
+
+    def lm_head(self, y: np.ndarray) -> np.ndarray:
+        """Final RMSNorm then the output projection (tied to the embedding when
+        ``tied_lm_head``)."""
+        n = rms_norm(y, self.W("final_norm"), self.m.norm_eps)
+        w = self.W("embed") if self.m.tied_lm_head else self.W("lm_head")
+        return linear(n, w)
+
+    # -- fusion Phi (§3.2) ----------------------------------------------------
+    def fusion_gated_mlp(self, c: np.ndarray, h: np.ndarray) -> np.ndarray:
+        """App. C.2: u = [LN(c); LN(h)], g = sigmoid(W_g u + b_g),
+        Delta = W_2 GELU(W_1 u + b_1) + b_2, h~ = LN(h + g * Delta)."""
+        m, d, eps = self.m, self.m.d_model, self.m.norm_eps
+        s = layer_norm(c, self.W("fusion.ln_c.w"), self.W("fusion.ln_c.b"), eps)
+        a = layer_norm(h, self.W("fusion.ln_h.w"), self.W("fusion.ln_h.b"), eps)
+        u = np.concatenate([s, a], axis=-1)
+        wg1, bg1 = self.W("fusion.w_g1"), self.W("fusion.b_g1")
+        g = sigmoid(linear(u, wg1[:d], bg1[:d]))
+        delta = linear(gelu_erf(linear(u, wg1[d:], bg1[d:])), self.W("fusion.w2"), self.W("fusion.b2"))
+        return layer_norm(h + g * delta, self.W("fusion.ln_out.w"), self.W("fusion.ln_out.b"), eps)
+
+    def _rms_scale(self, x: np.ndarray) -> np.ndarray:
+        """s_i = sqrt(mean_j x_ij^2 + eps), eps = 1e-6 (App. C.1)."""
+        return np.sqrt(np.mean(x * x, axis=-1, keepdims=True) + 1e-6)
+
+    def mixer(self, Z: np.ndarray, U: np.ndarray) -> np.ndarray:
+        """Shared mixer phi (App. C.1): J = [Z, U]; Q, K, V = J W_{Q,K,V};
+        R = Z + MHA(Q, K, V) W_O; phi = R + SiLU(R W_1) W_2.  Attention is
+        bidirectional over the rows of the current canvas."""
+        r, H = self.m.fusion_rank, self.m.fusion_heads
+        L = Z.shape[0]
+        J = np.concatenate([Z, U], axis=-1)
+        wqkv = self.W("fusion.wqkv")
+        q = linear(J, wqkv[:r]).reshape(L, H, r // H).transpose(1, 0, 2)
+        k = linear(J, wqkv[r:2 * r]).reshape(L, H, r // H).transpose(1, 0, 2)
+        v = linear(J, wqkv[2 * r:]).reshape(L, H, r // H).transpose(1, 0, 2)
+        pos = np.arange(L)
+        o = attention(q, k, v, pos, pos, causal=False).transpose(1, 0, 2).reshape(L, r)
+        R = Z + linear(o, self.W("fusion.wo"))
+        return R + linear(silu(linear(R, self.W("fusion.w1"))), self.W("fusion.w2"))
+
+    def paired_refresh(self, C0: np.ndarray, H0: np.ndarray) -> dict:
+        """Quantities of App. C.1 that depend only on the refresh step:
+        s_C, s_H, Z0 = (C0/s_C) W_C, U = (H0/s_H) W_H and phi(Z0, U)."""
+        sC, sH = self._rms_scale(C0), self._rms_scale(H0)
+        Z0 = linear(C0 / sC, self.W("fusion.wc"))
+        U = linear(H0 / sH, self.W("fusion.wh"))
+        return {"H0": H0, "C0": C0, "sC": sC, "sH": sH, "Z0": Z0, "U": U, "phi0": self.mixer(Z0, U)}
+
+    def fusion_paired_attn(self, C: np.ndarray, st: dict) -> np.ndarray:
+        """App. C.1: M = phi(Z, U) - phi(Z0, U)  (Eq. paired-attention-difference);
+        F = [U; Z0; Z - Z0; M]; g = sigmoid(SiLU(F W_g1) W_g2 + b_g);
+        H~ = H0 + g * s_H * (M W_up)  (Eq. stale-anchor-fusion-app)."""
+        Z = linear(C / st["sC"], self.W("fusion.wc"))
+        M = self.mixer(Z, st["U"]) - st["phi0"]
+        F = np.concatenate([st["U"], st["Z0"], Z - st["Z0"], M], axis=-1)
+        g = sigmoid(linear(silu(linear(F, self.W("fusion.wg1"))), self.W("fusion.wg2"), self.W("fusion.bg")))
+        return st["H0"] + g * st["sH"] * linear(M, self.W("fusion.wup"))
+
+    def make_cache(self, c: np.ndarray, h: np.ndarray):
+        """What the anchor cache holds for one sequence."""
+        if self.m.fusion == "paired_attn":
+            return self.paired_refresh(c, h)
+        return {"h": h}
+
+    def fuse(self, c: np.ndarray, cache) -> np.ndarray:
+        if self.m.fusion == "paired_attn":
+            return self.fusion_paired_attn(c, cache)
+        return self.fusion_gated_mlp(c, cache["h"])
+
+    # -- sessions (block mode context) ----------------------------------------
+    def new_session(self, batch: int) -> List[_Seq]:
+        return [_Seq() for _ in range(batch)]
+
+    def _fresh_pass(self, seq: _Seq, z_rows: np.ndarray):
+        """Causal fresh pass S -> A -> Phi(c, A(c)) -> D over rows appended to
+        the context; every layer's K, V for these rows join the context."""
+        L = z_rows.shape[0]
+        pos = seq.ctx_len + np.arange(L)
+        c = self.S(z_rows, pos, seq, causal=True, keep_kv=True, count=False)
+        h = self.A(c, pos, seq, causal=True, keep_kv=True, count=False)
+        ht = self.fuse(c, self.make_cache(c, h))
+        self.D_hidden(ht, pos, seq, causal=True, keep_kv=True, count=False)
+        seq.ctx_len += L
+
+    def prefill(self, sess: List[_Seq], prompts: np.ndarray):
+        """Encoder prefill of the prompt (block mode, App. C.1)."""
+        for b, seq in enumerate(sess):
+            self._fresh_pass(seq, prompts[b])
+
+    def commit_block(self, sess: List[_Seq], z_block: np.ndarray):
+        """Append a finalized block to the context (block mode, App. C.1)."""
+        for b, seq in enumerate(sess):
+            self._fresh_pass(seq, z_block[b])
+
+    # -- one refresh / one denoising step of Alg. 1 -----------------------------
+    def anchor_forward(self, sess: List[_Seq], z_rows: np.ndarray) -> list:
+        """Refresh branch of Alg. 1: h_cache <- A(S(z)) for every sequence."""
+        out = []
+        for b, seq in enumerate(sess):
+            pos = seq.ctx_len + np.arange(z_rows.shape[1])
+            c = self.S(z_rows[b], pos, seq, count=False)
+            h = self.A(c, pos, seq, count=(b == 0))
+            out.append(self.make_cache(c, h))
+        self.counters["anchor_calls"] += 1
+        return out
+
+    def denoise_logits(self, sess: List[_Seq], z_rows: np.ndarray, cache: list) -> np.ndarray:
+        """c = S(z); h~ = Phi(c, h_cache); logits = head(D(h~)).  [B, R, V]."""
+        B, R = z_rows.shape
+        out = np.empty((B, R, self.m.vocab), dtype=np.float64)
+        for b, seq in enumerate(sess):
+            pos = seq.ctx_len + np.arange(R)
+            c = self.S(z_rows[b], pos, seq, count=(b == 0))
+            ht = self.fuse(c, cache[b])
+            out[b] = self.lm_head(self.D_hidden(ht, pos, seq, count=(b == 0)))
+        return out
+
+    def sample(self, z_rows: np.ndarray, conf: np.ndarray, tok: np.ndarray, n: int, T: int, G: int):
+        """Sampler P: unmask k_n positions per sequence.  Returns the new canvas
+        and the selected positions ([B, k_n], -1 padded)."""
+        k = unmask_count(n, T, G)
+        z_new = z_rows.copy()
+        sel = np.full((z_rows.shape[0], max(k, 0)), -1, dtype=np.int64)
+        for b in range(z_rows.shape[0]):
+            p = select_topk(z_rows[b], conf[b], k, self.mask_id)
+            z_new[b, p] = tok[b, p]
+            sel[b, : p.size] = p
+        return z_new, sel
+
+    def denoise_step(self, sess, z_rows, cache, n: int, T: int, G: int):
+        """One reverse step after the (optional) refresh: logits, conf, tok and
+        the sampler update.  Returns a dict."""
+        logits = self.denoise_logits(sess, z_rows, cache)
+        conf, tok = confidence(logits, self.mask_id)
+        z_new, sel = self.sample(z_rows, conf, tok, n, T, G)
+        self.counters["steps"] += 1
+        return {"logits": logits, "conf": conf, "tok": tok, "z": z_new, "selected": sel}
+
+    # -- Alg. 1 over every block -----------------------------------------------
+    def generate(self, prompts: np.ndarray, gen_len: int, steps_per_block: int, K: int,
+                 block_len: int = 0, step_hook=None) -> np.ndarray:
+        """Alg. 1 per block.  block_len == 0: a single block over the whole
+        canvas (prompt + gen_len masks, bidirectional, no KV context).
+        Otherwise the prompt is prefilled, then blocks of ``block_len`` masks
+        are denoised and committed one after the other."""
+        B, P = prompts.shape
+        mask = self.mask_id
+        T = steps_per_block
+        if block_len == 0:
+            z = np.concatenate([prompts.astype(np.int32), np.full((B, gen_len), mask, np.int32)], axis=1)
+            sess = self.new_session(B)
+            z = self._run_block(sess, z, T, K, gen_len, 0, step_hook)
+            return z
+        assert gen_len % block_len == 0
+        sess = self.new_session(B)
+        self.prefill(sess, prompts.astype(np.int32))
+        blocks = []
+        for bi in range(gen_len // block_len):
+            zb = np.full((B, block_len), mask, np.int32)
+            zb = self._run_block(sess, zb, T, K, block_len, bi, step_hook)
+            self.commit_block(sess, zb)
+            blocks.append(zb)
+        return np.concatenate([prompts.astype(np.int32)] + blocks, axis=1)
+
+    def _run_block(self, sess, z, T, K, G, block_idx, step_hook):
+        cache = None
+        for n in range(T):           # n = T - i, i = T .. 1
+            if n % K == 0:           # Alg. 1 refresh test (T - i) mod K = 0
+                cache = self.anchor_forward(sess, z)
+                self.refresh_log.append((block_idx, n))
+            r = self.denoise_step(sess, z, cache, n, T, G)
+            if step_hook is not None:
+                step_hook(block_idx, n, z, r)
+            z = r["z"]
+        return z

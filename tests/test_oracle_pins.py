@@ -1,0 +1,447 @@
+"""Pins of the CPU oracle against things the paper and mathematics fix.
+
+No GPU.  Each test pins one part of ``oracle/`` against a closed form, a
+library routine, a value printed in the paper (``tests/golden``), an
+invariant of the method, or brute force on a tiny input.
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+import torch.nn.functional as Fn
+
+import workloads as wl
+from oracle import tadm_oracle as O
+
+GOLD = os.path.join(os.path.dirname(__file__), "golden")
+rng = np.random.default_rng(1234)
+
+
+def tiny_model(**kw):
+    base = dict(vocab=64, d_model=32, n_heads=4, n_kv_heads=2, head_dim=8, ffn=48, n_shared=0,
+                n_anchor=2, n_denoise=1, dtype="f32", fusion="gated_mlp", fusion_rank=16, fusion_heads=4)
+    base.update(kw)
+    return wl.ModelConfig(**base)
+
+
+def tiny_oracle(seed=3, affine_std=0.1, std=0.2, **kw):
+    m = tiny_model(**kw)
+    return O.Oracle(m, wl.make_weights(m, seed=seed, std=std, affine_std=affine_std))
+
+
+# --------------------------------------------------------------------------- generator
+def test_philox_known_answers():
+    kat = json.load(open(os.path.join(GOLD, "philox_kat.json")))
+    for v in kat["vectors"]:
+        ctr = [int(x, 16) for x in v["ctr"]]
+        key = [int(x, 16) for x in v["key"]]
+        assert wl.philox4x32_10(ctr, key) == tuple(int(x, 16) for x in v["out"])
+
+
+def test_generator_moments_and_bf16_rounding():
+    x = wl.normal(7, 11, 1 << 20, 0.0, 0.02, "f32").astype(np.float64)
+    assert abs(x.mean()) < 1e-4 and abs(x.std() - 0.02) < 1e-4
+    b = wl.normal(7, 11, 4096, 0.0, 0.02, "bf16")
+    f = wl.normal(7, 11, 4096, 0.0, 0.02, "f32")
+    # bf16 is the round-to-nearest-even of the float32 draw
+    wide = wl.bf16_bits_to_f32(b).astype(np.float64)
+    assert np.all(np.abs(wide - f) <= np.abs(wide) * 2.0 ** -8)   # within half a bf16 ulp
+    ref = torch.from_numpy(f).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    assert np.array_equal(ref, b)                                  # torch's conversion is also RNE
+
+
+# --------------------------------------------------------------------------- elementary ops
+def test_norms_against_torch_and_closed_form():
+    x = rng.standard_normal((5, 12))
+    g, b = rng.standard_normal(12), rng.standard_normal(12)
+    ref = Fn.layer_norm(torch.from_numpy(x), (12,), torch.from_numpy(g), torch.from_numpy(b), 1e-6)
+    np.testing.assert_allclose(O.layer_norm(x, g, b, 1e-6), ref.numpy(), rtol=1e-12, atol=1e-12)
+    ref = Fn.rms_norm(torch.from_numpy(x), (12,), torch.from_numpy(g), 1e-6)
+    np.testing.assert_allclose(O.rms_norm(x, g, 1e-6), ref.numpy(), rtol=1e-12, atol=1e-12)
+    # constant row c: RMSNorm -> sign(c) * gain * |c|/sqrt(c^2 + eps)
+    c = -3.0
+    out = O.rms_norm(np.full((1, 4), c), np.array([1.0, 2.0, 3.0, 4.0]), 1e-6)
+    np.testing.assert_allclose(out[0], -np.array([1, 2, 3, 4]) * 3.0 / math.sqrt(9 + 1e-6), rtol=1e-14)
+    # hand example: LayerNorm of [1, 2, 3, 4]: mean 2.5, var 1.25
+    ln = O.layer_norm(np.array([[1.0, 2.0, 3.0, 4.0]]), np.ones(4), np.zeros(4), 0.0)
+    np.testing.assert_allclose(ln[0], np.array([-1.5, -0.5, 0.5, 1.5]) / math.sqrt(1.25), rtol=1e-14)
+
+
+def test_activations_against_torch():
+    x = np.linspace(-6, 6, 101)
+    t = torch.from_numpy(x)
+    np.testing.assert_allclose(O.gelu_erf(x), Fn.gelu(t).numpy(), rtol=1e-12, atol=1e-14)
+    np.testing.assert_allclose(O.gelu_tanh(x), Fn.gelu(t, approximate="tanh").numpy(), rtol=1e-12, atol=1e-14)
+    np.testing.assert_allclose(O.silu(x), Fn.silu(t).numpy(), rtol=1e-12, atol=1e-14)
+    np.testing.assert_allclose(O.sigmoid(x), torch.sigmoid(t).numpy(), rtol=1e-12, atol=1e-14)
+
+
+def test_rope_complex_form_and_relative_property():
+    hd, L = 16, 7
+    x = rng.standard_normal((3, L, hd))
+    pos = np.array([0, 1, 5, 9, 100, 1000, 4095])
+    out = O.rope(x, pos, 10000.0)
+    # complex form: (x_j + i x_{j+hd/2}) * exp(i * pos * theta^(-2j/hd))
+    z = x[..., : hd // 2] + 1j * x[..., hd // 2:]
+    freq = 10000.0 ** (-np.arange(hd // 2) * 2.0 / hd)
+    zr = z * np.exp(1j * pos[:, None] * freq[None, :])
+    np.testing.assert_allclose(out, np.concatenate([zr.real, zr.imag], -1), rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(O.rope(x, np.zeros(L, int), 1e4), x)   # position 0 is the identity
+    # dot products depend only on the position difference
+    q, k = rng.standard_normal((1, 1, hd)), rng.standard_normal((1, 1, hd))
+    d1 = (O.rope(q, np.array([7]), 1e4) * O.rope(k, np.array([3]), 1e4)).sum()
+    d2 = (O.rope(q, np.array([104]), 1e4) * O.rope(k, np.array([100]), 1e4)).sum()
+    assert abs(d1 - d2) < 1e-12
+
+
+@pytest.mark.parametrize("causal", [False, True])
+def test_attention_against_sdpa(causal):
+    Hq, Hkv, L, hd = 4, 2, 9, 8
+    q = rng.standard_normal((Hq, L, hd))
+    k = rng.standard_normal((Hkv, L, hd))
+    v = rng.standard_normal((Hkv, L, hd))
+    pos = np.arange(L)
+    out = O.attention(q, k, v, pos, pos, causal)
+    kk = torch.from_numpy(k).repeat_interleave(Hq // Hkv, 0)
+    vv = torch.from_numpy(v).repeat_interleave(Hq // Hkv, 0)
+    ref = Fn.scaled_dot_product_attention(torch.from_numpy(q), kk, vv, is_causal=causal)
+    np.testing.assert_allclose(out, ref.numpy(), rtol=1e-12, atol=1e-12)
+
+
+def test_attention_brute_force_scalar_loops():
+    Hq, Hkv, Lq, Lk, hd = 2, 1, 3, 5, 4
+    q = rng.standard_normal((Hq, Lq, hd))
+    k = rng.standard_normal((Hkv, Lk, hd))
+    v = rng.standard_normal((Hkv, Lk, hd))
+    qp, kp = np.array([2, 3, 4]), np.arange(Lk)
+    out = O.attention(q, k, v, qp, kp, causal=True)
+    for h in range(Hq):
+        for i in range(Lq):
+            w = [math.exp(sum(q[h, i, t] * k[0, j, t] for t in range(hd)) / 2.0) if j <= qp[i] else 0.0
+                 for j in range(Lk)]
+            s = sum(w)
+            for t in range(hd):
+                assert abs(out[h, i, t] - sum(w[j] * v[0, j, t] for j in range(Lk)) / s) < 1e-12
+
+
+# --------------------------------------------------------------------------- backbone layer
+def _layer_parts(o, name):
+    m = o.m
+    hd, Hq, Hkv = m.head_dim, m.n_heads, m.n_kv_heads
+    W = o.W
+    return (W(name + "wqkv")[: Hq * hd], W(name + "wqkv")[Hq * hd:(Hq + Hkv) * hd],
+            W(name + "wqkv")[(Hq + Hkv) * hd:])
+
+
+def test_layer_single_token_closed_form():
+    """One token at position 0: RoPE is the identity and attention returns V,
+    so the layer is x + Wo expand(Wv n1) + Wdown(act(Wg n2) * Wu n2)."""
+    for glu in ("swiglu", "geglu"):
+        o = tiny_oracle(glu=glu)
+        m = o.m
+        x = rng.standard_normal((1, m.d_model))
+        out = o.layer("anchor.0.", x, np.array([0]), None, causal=False, keep_kv=False)
+        _, _, wv = _layer_parts(o, "anchor.0.")
+        n1 = O.rms_norm(x, o.W("anchor.0.attn_norm"), m.norm_eps)
+        v = (n1 @ wv.T).reshape(m.n_kv_heads, m.head_dim)
+        attn = np.repeat(v, m.n_heads // m.n_kv_heads, axis=0).reshape(1, -1)   # head h reads KV h // group
+        x1 = x + attn @ o.W("anchor.0.wo").T
+        n2 = O.rms_norm(x1, o.W("anchor.0.ffn_norm"), m.norm_eps)
+        wgu = o.W("anchor.0.wgu")
+        gate, up = n2 @ wgu[: m.ffn].T, n2 @ wgu[m.ffn:].T
+        act = O.silu(gate) if glu == "swiglu" else O.gelu_tanh(gate)
+        np.testing.assert_allclose(out, x1 + (act * up) @ o.W("anchor.0.wdown").T, rtol=1e-12, atol=1e-12)
+
+
+def test_layer_shift_invariance_and_causal_prefix():
+    o = tiny_oracle()
+    x = rng.standard_normal((6, o.m.d_model))
+    a = o.layer("anchor.1.", x, np.arange(6), None, False, False)
+    b = o.layer("anchor.1.", x, np.arange(6) + 37, None, False, False)
+    np.testing.assert_allclose(a, b, rtol=1e-10, atol=1e-10)        # RoPE is relative
+    c1 = o.layer("anchor.1.", x, np.arange(6), None, True, False)
+    c2 = o.layer("anchor.1.", x[:4], np.arange(4), None, True, False)
+    np.testing.assert_allclose(c1[:4], c2, rtol=1e-12, atol=1e-12)  # causal rows ignore later rows
+    assert not np.allclose(a[:4], c1[:4])
+
+
+def test_gqa_equals_mha_with_repeated_kv_heads():
+    og = tiny_oracle(n_heads=4, n_kv_heads=2)
+    mm = tiny_model(n_heads=4, n_kv_heads=4)
+    w = dict(og._raw)
+    hd, d = 8, 32
+    wqkv = og.W("anchor.0.wqkv")
+    q, k, v = wqkv[:32], wqkv[32:48], wqkv[48:64]
+    rep = lambda t: np.repeat(t.reshape(2, hd, d), 2, axis=0).reshape(4 * hd, d)
+    w["anchor.0.wqkv"] = np.concatenate([q, rep(k), rep(v)]).astype(np.float32)
+    om = O.Oracle(mm, w)
+    x = rng.standard_normal((5, d))
+    np.testing.assert_allclose(og.layer("anchor.0.", x, np.arange(5), None, False, False),
+                               om.layer("anchor.0.", x, np.arange(5), None, False, False), rtol=1e-12, atol=1e-12)
+
+
+def test_kv_context_equals_one_causal_pass():
+    """Prefill + commit through the KV cache equals one causal fresh pass over
+    the concatenated rows (block-mode encoder, App. C.1)."""
+    o = tiny_oracle(n_shared=1)
+    z = rng.integers(0, 63, size=11).astype(np.int32)
+    s1 = o.new_session(1)[0]
+    o._fresh_pass(s1, z[:7])
+    o._fresh_pass(s1, z[7:])
+    s2 = o.new_session(1)[0]
+    o._fresh_pass(s2, z)
+    for name in s1.kv:
+        np.testing.assert_allclose(s1.kv[name][0], s2.kv[name][0], rtol=1e-10, atol=1e-12)
+        np.testing.assert_allclose(s1.kv[name][1], s2.kv[name][1], rtol=1e-10, atol=1e-12)
+
+
+# --------------------------------------------------------------------------- fusion (App. C.2)
+def test_gated_mlp_zero_weights_closed_form():
+    """W = 0, b_g = beta_g, b_2 = beta: g = sigmoid(beta_g), Delta = beta,
+    h~ = LN(h + sigmoid(beta_g) * beta)."""
+    o = tiny_oracle(affine_std=0.0)
+    d = o.m.d_model
+    w = dict(o._raw)
+    w["fusion.w_g1"] = np.zeros_like(w["fusion.w_g1"])
+    w["fusion.w2"] = np.zeros_like(w["fusion.w2"])
+    bg = rng.standard_normal(5 * d).astype(np.float32)
+    b2 = rng.standard_normal(d).astype(np.float32)
+    w["fusion.b_g1"], w["fusion.b2"] = bg, b2
+    o2 = O.Oracle(o.m, w)
+    c, h = rng.standard_normal((3, d)), rng.standard_normal((3, d))
+    exp = O.layer_norm(h + O.sigmoid(bg[:d].astype(np.float64)) * b2, np.ones(d), np.zeros(d), 1e-6)
+    np.testing.assert_allclose(o2.fusion_gated_mlp(c, h), exp, rtol=1e-12, atol=1e-12)
+
+
+def test_gated_mlp_gate_and_hidden_rows():
+    """With W2 = I-like selection the output isolates g * GELU(W1 u + b1):
+    checks which rows are the gate and which the hidden projection."""
+    o = tiny_oracle(affine_std=0.0)
+    d = o.m.d_model
+    w = dict(o._raw)
+    w2 = np.zeros((d, 4 * d), np.float32)
+    w2[np.arange(d), np.arange(d)] = 1.0            # Delta_j = GELU(hidden_j)
+    w["fusion.w2"] = w2
+    w["fusion.b2"] = np.zeros(d, np.float32)
+    o2 = O.Oracle(o.m, w)
+    c, h = rng.standard_normal((2, d)), rng.standard_normal((2, d))
+    u = np.concatenate([O.layer_norm(c, 1, 0, 1e-6), O.layer_norm(h, 1, 0, 1e-6)], -1)
+    wg1, bg1 = o2.W("fusion.w_g1"), o2.W("fusion.b_g1")
+    g = O.sigmoid(u @ wg1[:d].T + bg1[:d])
+    hid = O.gelu_erf(u @ wg1[d:2 * d].T + bg1[d:2 * d])
+    np.testing.assert_allclose(o2.fusion_gated_mlp(c, h), O.layer_norm(h + g * hid, 1, 0, 1e-6), rtol=1e-11, atol=1e-12)
+
+
+# --------------------------------------------------------------------------- fusion (App. C.1)
+def paired_oracle(**kw):
+    return tiny_oracle(fusion="paired_attn", n_shared=1, tied_lm_head=True, **kw)
+
+
+def test_paired_attention_identity_at_fresh_anchor():
+    """C = C0 implies M = 0 and H~ = H0 exactly (App. C.1)."""
+    o = paired_oracle()
+    C0, H0 = rng.standard_normal((6, 32)), rng.standard_normal((6, 32))
+    st = o.paired_refresh(C0, H0)
+    out = o.fusion_paired_attn(C0.copy(), st)
+    assert np.array_equal(out, H0)
+    C = C0 + 0.3 * rng.standard_normal((6, 32))
+    assert not np.allclose(o.fusion_paired_attn(C, st), H0)
+
+
+def test_paired_attention_zero_up_projection():
+    o = paired_oracle()
+    w = dict(o._raw)
+    w["fusion.wup"] = np.zeros_like(w["fusion.wup"])
+    o2 = O.Oracle(o.m, w)
+    C0, H0 = rng.standard_normal((5, 32)), rng.standard_normal((5, 32))
+    st = o2.paired_refresh(C0, H0)
+    np.testing.assert_array_equal(o2.fusion_paired_attn(rng.standard_normal((5, 32)), st), H0)
+
+
+def test_paired_attention_uniform_mixer_closed_form():
+    """W_Q = W_K = 0 makes every attention row uniform, so MHA returns the
+    column mean of V = J W_V; with W_1 = 0 the FFN vanishes, hence
+    phi(Z, U) = Z + mean_rows(J W_V) W_O, and with W_g1 = 0 the gate is
+    sigmoid(b_g).  Then H~ = H0 + sigmoid(b_g) s_H (M W_up) in closed form."""
+    o = paired_oracle()
+    r = o.m.fusion_rank
+    w = dict(o._raw)
+    wqkv = w["fusion.wqkv"].copy()
+    wqkv[: 2 * r] = 0.0
+    w["fusion.wqkv"] = wqkv
+    w["fusion.w1"] = np.zeros_like(w["fusion.w1"])
+    w["fusion.wg1"] = np.zeros_like(w["fusion.wg1"])
+    w["fusion.bg"] = np.array([0.7], np.float32)
+    o2 = O.Oracle(o.m, w)
+    W = o2.W
+    L = 5
+    C0, H0, C = (rng.standard_normal((L, 32)) for _ in range(3))
+    sC = np.sqrt((C0 ** 2).mean(-1, keepdims=True) + 1e-6)
+    sH = np.sqrt((H0 ** 2).mean(-1, keepdims=True) + 1e-6)
+    Z0, Z, U = (C0 / sC) @ W("fusion.wc").T, (C / sC) @ W("fusion.wc").T, (H0 / sH) @ W("fusion.wh").T
+    wv = W("fusion.wqkv")[2 * r:]
+
+    def phi(Zx):
+        V = np.concatenate([Zx, U], -1) @ wv.T
+        return Zx + np.repeat(V.mean(0, keepdims=True), L, 0) @ W("fusion.wo").T
+
+    M = phi(Z) - phi(Z0)
+    exp = H0 + O.sigmoid(float(np.float32(0.7))) * sH * (M @ W("fusion.wup").T)
+    st = o2.paired_refresh(C0, H0)
+    np.testing.assert_allclose(o2.fusion_paired_attn(C, st), exp, rtol=1e-10, atol=1e-12)
+
+
+# --------------------------------------------------------------------------- sampler P
+def test_confidence_hand_values():
+    V = 6
+    l = np.log(np.array([[1.0, 2.0, 2.0, 1.0, 1.0, 50.0]]))   # MASK (id 5) would win: excluded
+    conf, tok = O.confidence(l, mask_id=V - 1)
+    assert tok[0] == 1                                          # tie between ids 1, 2 -> lower id
+    assert abs(conf[0] - 2.0 / 7.0) < 1e-15
+    conf, tok = O.confidence(np.zeros((2, V)), V - 1)
+    np.testing.assert_allclose(conf, 1.0 / (V - 1))
+    assert np.all(tok == 0)
+
+
+def test_topk_brute_force_and_carry_over():
+    mask = 9
+    for trial in range(200):
+        L = int(rng.integers(1, 20))
+        z = np.where(rng.random(L) < 0.6, mask, rng.integers(0, 9, L))
+        conf = rng.choice([0.1, 0.2, 0.3, 0.5], size=L)             # many ties
+        k = int(rng.integers(0, L + 2))
+        got = O.select_topk(z, conf, k, mask)
+        cand = [p for p in range(L) if z[p] == mask]
+        want = sorted(cand, key=lambda p: (-conf[p], p))[:k]
+        assert list(got) == want
+        assert all(z[p] == mask for p in got)
+
+
+def test_unmask_schedule():
+    for G, T, k in ((96, 32, 3), (768, 128, 6), (32, 16, 2), (32, 32, 1), (7, 3, None), (5, 8, None)):
+        ks = [O.unmask_count(n, T, G) for n in range(T)]
+        assert sum(ks) == G and min(ks) >= 0
+        if k is not None:
+            assert ks == [k] * T
+
+
+def test_layer_cost_against_tables_1_and_2():
+    g = json.load(open(os.path.join(GOLD, "layer_cost.json")))
+    for row in g["table1_ratio"]:
+        full, cache = O.layer_cost(row["L_S"], row["L_A"], row["L_D"], row["T"], row["K"])
+        assert round(cache / full, 2) == row["ratio_2dp"]
+    for row in g["table2_calls"]:
+        _, tadm = O.layer_cost(0, 12, 6, row["T"], row["K"])
+        mdlm, _ = O.layer_cost(0, 0, 12, row["T"], 1)
+        assert tadm == row["tadm"] and mdlm == row["mdlm"]
+        assert round(tadm / mdlm, 2) == row["ratio_2dp"]
+
+
+# --------------------------------------------------------------------------- Alg. 1 loop
+def _gen(o, K, block_len=0, P=5, G=12, T=4, hook=None):
+    prompts = rng.integers(0, o.m.vocab - 1, size=(2, P)).astype(np.int32)
+    return prompts, o.generate(prompts, G, T, K, block_len, step_hook=hook)
+
+
+def test_refresh_schedule_and_count():
+    for K in (1, 2, 3, 4, 5):
+        o = tiny_oracle()
+        T, nblk = 6, 2
+        _gen(o, K, block_len=4, G=8, T=T)
+        assert o.refresh_log == [(b, n) for b in range(nblk) for n in range(T) if n % K == 0]
+        assert o.counters["anchor_calls"] == nblk * (-(-T // K))
+        assert o.counters["anchor"] == nblk * (-(-T // K)) * o.m.n_anchor
+        assert o.counters["denoise"] == nblk * T * o.m.n_denoise
+
+
+def test_k1_is_single_stage_dlm():
+    """K = 1 refreshes at every step, so each step is one fresh pass
+    D(Phi(c, A(c))): rebuild that loop directly and compare trajectories."""
+    o = tiny_oracle()
+    prompts, z1 = _gen(o, K=1, G=9, T=3)
+    z = np.concatenate([prompts, np.full((2, 9), o.mask_id, np.int32)], 1)
+    for n in range(3):
+        logits = np.stack([o.lm_head(o.D_hidden(o.fusion_gated_mlp(c, o.A(c, np.arange(14), None)),
+                                                np.arange(14), None))
+                           for c in (o.S(z[b], np.arange(14), None) for b in range(2))])
+        conf, tok = O.confidence(logits, o.mask_id)
+        for b in range(2):
+            p = O.select_topk(z[b], conf[b], O.unmask_count(n, 3, 9), o.mask_id)
+            z[b, p] = tok[b, p]
+    np.testing.assert_array_equal(z, z1)
+
+
+@pytest.mark.parametrize("fusion,block_len", [("gated_mlp", 0), ("gated_mlp", 4), ("paired_attn", 4)])
+def test_carry_over_zero_masking_and_stale_cache(fusion, block_len):
+    o = tiny_oracle(fusion=fusion, n_shared=1 if fusion == "paired_attn" else 0,
+                    tied_lm_head=fusion == "paired_attn")
+    seen = []
+
+    def hook(b, n, z, r):
+        assert np.all(r["tok"] != o.mask_id)                       # zero-masking
+        fixed = z != o.mask_id
+        assert np.array_equal(r["z"][fixed], z[fixed])             # carry-over
+        assert np.sum((z == o.mask_id) & (r["z"] != o.mask_id)) == 2 * O.unmask_count(n, 4, 4 if block_len else 12)
+        seen.append((b, n))
+
+    prompts, z = _gen(o, K=3, block_len=block_len, hook=hook)
+    assert np.all(z != o.mask_id)
+    np.testing.assert_array_equal(z[:, :5], prompts)
+    assert len(seen) == (3 if block_len else 1) * 4
+
+
+def test_stale_anchor_is_reused_between_refreshes():
+    """Between refreshes the fusion reads the cached h of the refresh step
+    (Alg. 1): the step-1 logits of K=2 equal D(Phi(S(z_1), A(S(z_0))))."""
+    o = tiny_oracle()
+    logs = {}
+    prompts, _ = _gen(o, K=2, G=8, T=4, hook=lambda b, n, z, r: logs.setdefault(n, (z.copy(), r["logits"])))
+    z0, _ = logs[0]
+    z1, l1 = logs[1]
+    L = z0.shape[1]
+    pos = np.arange(L)
+    for b in range(2):
+        h0 = o.A(o.S(z0[b], pos, None), pos, None)
+        want = o.lm_head(o.D_hidden(o.fusion_gated_mlp(o.S(z1[b], pos, None), h0), pos, None))
+        np.testing.assert_allclose(l1[b], want, rtol=1e-12, atol=1e-12)
+
+
+def test_paired_attention_gate_features():
+    """A gate MLP that reads one feature of the Z - Z0 block of F:
+    W_g1 row 0 selects column 2r (first feature of Z - Z0), W_g2 = [alpha, 0..],
+    so g = sigmoid(alpha * SiLU((Z - Z0)_0) + b_g) per row, recovered from
+    (H~ - H0) / (s_H * (M W_up))."""
+    o = paired_oracle()
+    r = o.m.fusion_rank
+    w = dict(o._raw)
+    wg1 = np.zeros((r, 4 * r), np.float32)
+    wg1[0, 2 * r] = 1.0
+    wg2 = np.zeros((1, r), np.float32)
+    wg2[0, 0] = 1.5
+    w["fusion.wg1"], w["fusion.wg2"], w["fusion.bg"] = wg1, wg2, np.array([-0.25], np.float32)
+    o2 = O.Oracle(o.m, w)
+    L = 6
+    C0, H0 = rng.standard_normal((L, 32)), rng.standard_normal((L, 32))
+    C = C0 + rng.standard_normal((L, 32))
+    st = o2.paired_refresh(C0, H0)
+    out = o2.fusion_paired_attn(C, st)
+    sC = np.sqrt((C0 ** 2).mean(-1, keepdims=True) + 1e-6)
+    dz0 = ((C - C0) / sC) @ o2.W("fusion.wc")[0]
+    g = 1.0 / (1.0 + np.exp(-(1.5 * dz0 / (1.0 + np.exp(-dz0)) - 0.25)))
+    Z = (C / sC) @ o2.W("fusion.wc").T
+    MW = (o2.mixer(Z, st["U"]) - st["phi0"]) @ o2.W("fusion.wup").T
+    np.testing.assert_allclose((out - H0) / (st["sH"] * MW), np.repeat(g[:, None], 32, 1), rtol=1e-8)
+
+
+def test_tied_head_reads_the_embedding():
+    """Tied output head: logits = RMSNorm(y) E^T, so for y = E[t] the
+    self inner product wins and the argmax is t."""
+    m = tiny_model(fusion="paired_attn", n_shared=1, tied_lm_head=True, d_model=64, vocab=128)
+    o = O.Oracle(m, wl.make_weights(m, seed=5, std=0.2))
+    assert "lm_head" not in o._raw
+    E = o.W("embed")
+    logits = o.lm_head(E[:127])
+    assert np.array_equal(np.argmax(logits, -1), np.arange(127))
