@@ -1,0 +1,261 @@
+/*
+ * tadm.h - C ABI of the GB300 (sm_103a) implementation of TADM's
+ * anchor-cache reverse-diffusion sampling loop (Time-Anchored Diffusion
+ * Language Models).
+ *
+ * The method (paper §3): a denoising network is split into a shared network
+ * S, an expensive anchor network A, a small fusion module Phi and a light
+ * denoiser D.  The anchor latent h = A(S(z)) is refreshed once every K
+ * reverse steps and cached in HBM; every step encodes the current canvas
+ * c = S(z), fuses it with the stale cache, h~ = Phi(c, h_cache)
+ * (Eq. stale-anchor-fusion), and denoises, x = D(h~) (Alg. 1).  The sampler
+ * unmasks the most confident masked positions of the active block.
+ *
+ * Conventions for every call:
+ *  - Pointers named "device" are CUDA device pointers; the caller owns and
+ *    frees all of them (the library allocates no device memory).  "host"
+ *    pointers are plain host memory.
+ *  - Token ids are int32.  MASK is vocab - 1.  Every id the caller passes
+ *    must lie in [0, vocab - 1].
+ *  - Matrices are row-major.  A projection from n_in to n_out features is a
+ *    weight [n_out, n_in] (y = x W^T).
+ *  - Calls that take a stream only enqueue work on it and return at once;
+ *    kernels that give up a bounded wait set a device status word that
+ *    tadm_sync_status() turns into TADM_ERR_TIMEOUT.  Argument errors are
+ *    detected on the host, before anything is enqueued.
+ *  - No call throws, aborts or exits.  On error the returned status is
+ *    non-zero and tadm_last_error() describes it.
+ *  - A handle must not be used by two host threads at once.
+ */
+#ifndef TADM_H
+#define TADM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define TADM_API __attribute__((visibility("default")))
+#else
+#define TADM_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* cudaStream_t; NULL means the legacy default stream. */
+typedef struct CUstream_st* tadm_stream;
+
+typedef enum {
+  TADM_OK = 0,
+  TADM_ERR_INVALID_ARG = 1, /* bad shape, size, pointer or alignment */
+  TADM_ERR_UNSUPPORTED = 2, /* valid model, but a shape this build does not run */
+  TADM_ERR_CUDA = 3,        /* a CUDA runtime call failed */
+  TADM_ERR_OOM = 4,         /* the bound workspace is smaller than required */
+  TADM_ERR_TIMEOUT = 5,     /* a kernel gave up a bounded wait */
+  TADM_ERR_STATE = 6        /* call out of order (no workspace, context full, ...) */
+} tadm_status;
+
+/*
+ * Model description (paper §3.1, App. C.1, App. C.2).
+ *  glu:     0 = SwiGLU (SiLU gate), 1 = GeGLU (tanh-approximate GELU gate).
+ *  n_shared, n_anchor, n_denoise: L_S, L_A, L_D of Eq. (anchor-cache-compute);
+ *           S is the token embedding followed by n_shared layers.
+ *  fusion:  0 = gated residual MLP (App. C.2):
+ *              u = [LN(c); LN(h)], g = sigmoid(W_g u + b_g),
+ *              Delta = W_2 GELU(W_1 u + b_1) + b_2, h~ = LN(h + g * Delta);
+ *           1 = paired attention with cached shallow state (App. C.1,
+ *              Eqs. paired-attention-difference, stale-anchor-fusion-app).
+ *  fusion_rank, fusion_heads: r and the mixer heads of fusion 1.
+ *  dtype:   0 = fp32 weights and activations, 1 = bf16 weights and GEMM
+ *           operands (fp32 accumulation, fp32 residual stream).
+ *  tied_lm_head: 1 = the output head reuses the embedding matrix.
+ */
+typedef struct {
+  int32_t vocab, d_model, n_heads, n_kv_heads, head_dim, ffn;
+  int32_t glu;
+  int32_t n_shared, n_anchor, n_denoise;
+  int32_t fusion;
+  int32_t fusion_rank, fusion_heads;
+  int32_t dtype;
+  int32_t tied_lm_head;
+  float norm_eps, rope_theta;
+} tadm_config;
+
+typedef struct tadm_handle tadm_handle;
+
+/* ---------------------------------------------------------------- weights --
+ * The model's parameters are passed as an array of device pointers in the
+ * order this inventory lists them.  Element type: fp32 when dtype = 0, bf16
+ * when dtype = 1.  Each tensor is contiguous, row-major [rows, cols] (vectors
+ * have cols = 1... rows = length) and 16-byte aligned.
+ *
+ * Inventory: "embed" [V, d]; then for net in (shared, anchor, denoise) and
+ * each layer i: "<net>.<i>.attn_norm" [d], ".wqkv" [(Hq + 2 Hkv) hd, d]
+ * (rows: Q heads, K heads, V heads), ".wo" [d, Hq hd], ".ffn_norm" [d],
+ * ".wgu" [2F, d] (rows: gate, then up), ".wdown" [d, F]; then the fusion
+ * parameters; "final_norm" [d]; "lm_head" [V, d] unless tied.
+ */
+/* Number of weight tensors of cfg, or -1 if cfg is invalid. */
+TADM_API int tadm_weight_count(const tadm_config* cfg);
+/* Name (NUL-terminated, truncated to name_cap) and shape of tensor `index`.
+ * Vectors report cols = 1.  INVALID_ARG for a bad index or config. */
+TADM_API tadm_status tadm_weight_info(const tadm_config* cfg, int index, char* name, int name_cap,
+                             int64_t* rows, int64_t* cols);
+
+/* ----------------------------------------------------------------- handle --
+ * tadm_create validates cfg and copies the weight pointers (the weights must
+ * stay valid for the handle's life).  Sizes fix the workspace:
+ *   max_batch: sequences per call;
+ *   max_rows:  canvas rows per sequence in one step (block_len in block mode,
+ *              prompt + generation length in single-block mode);
+ *   max_ctx:   block mode: positions per sequence that hold K/V (the prompt,
+ *              every committed block and the active block, i.e. at least
+ *              prompt + generation length); 0 when only the single-block
+ *              mode is used.
+ */
+TADM_API tadm_status tadm_create(const tadm_config* cfg, const void* const* weights, int n_weights,
+                        int max_batch, int max_rows, int max_ctx, tadm_handle** out);
+TADM_API void tadm_destroy(tadm_handle* h);
+TADM_API const char* tadm_last_error(const tadm_handle* h);
+TADM_API const char* tadm_status_string(tadm_status s);
+
+/* Device workspace: activations, KV caches, the internal anchor cache of
+ * tadm_generate and the status word.  Caller allocates >= *bytes, 256-byte
+ * aligned, and binds it before any compute call.  Binding synchronises the
+ * device once (it fills the RoPE table). */
+TADM_API tadm_status tadm_workspace_size(const tadm_handle* h, size_t* bytes);
+TADM_API tadm_status tadm_bind_workspace(tadm_handle* h, void* dev_ptr, size_t bytes);
+
+/* Bytes of one anchor cache for `batch` sequences of `rows` canvas rows
+ * (fusion 0: h, fp32 [batch*rows, d]; fusion 1: H0, s_C, s_H, Z0, U and
+ * phi(Z0, U)).  Caller-allocated, device, 256-byte aligned. */
+TADM_API tadm_status tadm_cache_size(const tadm_handle* h, int batch, int rows, size_t* bytes);
+
+/* ------------------------------------------------------ one step of Alg. 1 --
+ * Block mode: tadm_reset, tadm_prefill(prompt), then per block the steps on
+ * the block's canvas rows, then tadm_commit_block.  Single-block mode:
+ * tadm_reset then steps on the whole canvas (context stays empty).
+ * x_t: device int32 [batch, rows] canvas of the active rows, positions
+ * ctx .. ctx + rows - 1 where ctx is the committed context length.
+ */
+TADM_API tadm_status tadm_reset(tadm_handle* h, int batch);
+
+/* Causal fresh pass S -> A -> Phi(c, A(c)) -> D over the prompt; every
+ * layer's K, V join the context (App. C.1, encoder prefill).
+ * prompt: device int32 [batch, prompt_len]. */
+TADM_API tadm_status tadm_prefill(tadm_handle* h, const int32_t* prompt, int batch, int prompt_len,
+                         tadm_stream stream);
+
+/* Refresh branch of Alg. 1: h_cache <- A(S(x_t)).  `t` is the step index i of
+ * Alg. 1 (informational; time conditioning is off).  h_cache: device, at
+ * least tadm_cache_size(batch, rows) bytes. */
+TADM_API tadm_status tadm_anchor_forward(tadm_handle* h, const int32_t* x_t, int batch, int rows, int t,
+                                void* h_cache, tadm_stream stream);
+
+/* Optional outputs of a denoising step (device pointers, each may be NULL):
+ *  logits:   fp32 [batch*rows, vocab] (written only if non-NULL; the fast
+ *            path never materialises them);
+ *  conf:     fp32 [batch*rows] max softmax probability over ids != MASK;
+ *  tok:      int32 [batch*rows] its argmax (lowest id on ties);
+ *  selected: int32 [batch, k_n] positions unmasked this step, ascending rank,
+ *            -1 padded;
+ *  fused:    fp32 [batch*rows, d] the fused latent h~ = Phi(c, h_cache) that
+ *            enters D. */
+typedef struct {
+  float* logits;
+  float* conf;
+  int32_t* tok;
+  int32_t* selected;
+  float* fused;
+} tadm_step_outputs;
+
+/* One reverse step: c = S(x_t), h~ = Phi(c, h_cache), logits = head(D(h~)),
+ * then the sampler unmasks k_n = floor((n+1) G / T) - floor(n G / T)
+ * positions per sequence (n = T - t, G = n_masked_at_start): the masked
+ * positions of largest confidence, ties toward the lower position.  Tokens
+ * already unmasked are never changed (carry-over), MASK is never predicted
+ * (zero-masking).  x_t is updated in place.  `out` may be NULL. */
+TADM_API tadm_status tadm_denoise_step(tadm_handle* h, int32_t* x_t, int batch, int rows, int t, int T,
+                              int n_masked_at_start, const void* h_cache,
+                              const tadm_step_outputs* out, tadm_stream stream);
+
+/* Causal fresh pass over a finalised block; its K, V join the context. */
+TADM_API tadm_status tadm_commit_block(tadm_handle* h, const int32_t* x_block, int batch, int rows,
+                              tadm_stream stream);
+
+/* Whole generation (Alg. 1 per block).  prompt: device int32 [batch,
+ * prompt_len]; out: device int32 [batch, prompt_len + gen_len], the final
+ * canvas.  block_len = 0: one block over the whole canvas (bidirectional,
+ * no KV context); else gen_len % block_len == 0 and the prompt is prefilled.
+ * The anchor refreshes at n = 0, K, 2K, ... of every block. */
+TADM_API tadm_status tadm_generate(tadm_handle* h, const int32_t* prompt, int batch, int prompt_len,
+                          int32_t* out, int gen_len, int steps_per_block, int K, int block_len,
+                          tadm_stream stream);
+
+/* Waits for the last stream used by h, then reports TADM_ERR_TIMEOUT if a
+ * kernel gave up a bounded wait since the last reset of the status word
+ * (tadm_generate and tadm_reset clear it), TADM_ERR_CUDA on a CUDA error. */
+TADM_API tadm_status tadm_sync_status(tadm_handle* h);
+
+/* ------------------------------------------------------------- accounting --
+ * Layer evaluations and anchor calls issued by reverse steps since the last
+ * tadm_reset / tadm_generate (prefill and commit passes are counted apart),
+ * the quantities of Eq. (anchor-cache-compute). */
+typedef struct {
+  int64_t shared_layers, anchor_layers, denoise_layers;
+  int64_t anchor_calls, denoise_steps;
+  int64_t commit_passes;
+} tadm_counters;
+TADM_API tadm_status tadm_get_counters(const tadm_handle* h, tadm_counters* out);
+
+/* Plan of tadm_generate (host only, no GPU): the ordered phases it issues.
+ * kind: 0 prefill, 1 anchor refresh, 2 denoise step, 3 commit.  For kinds 1
+ * and 2, n is the step within the block and k the positions unmasked
+ * (kind 2).  Writes at most `cap` events; *n_events gets the full count. */
+typedef struct {
+  int32_t kind, block, n, k;
+} tadm_plan_event;
+TADM_API tadm_status tadm_plan(int prompt_len, int gen_len, int steps_per_block, int K, int block_len,
+                      tadm_plan_event* events, int cap, int* n_events);
+
+/* Eq. (anchor-cache-compute): C_full = T (L_S + L_A + L_D) and
+ * C_cache = T (L_S + L_D) + ceil(T / K) L_A. */
+TADM_API tadm_status tadm_layer_cost(int L_S, int L_A, int L_D, int T, int K, int64_t* c_full,
+                            int64_t* c_cache);
+
+/* --------------------------------------------------------- building blocks --
+ * The kernels of the path, exposed for unit parity tests and benchmarks.
+ * They use no handle and need no workspace; all pointers are device pointers.
+ */
+/* C[M, N] = A[M, K] B[N, K]^T.  dtype 1: A, B bf16 (tcgen05 tensor cores,
+ * fp32 accumulate); dtype 0: fp32 (CUDA cores).  c_dtype: 0 fp32, 1 bf16.
+ * Row strides lda, ldb, ldc in elements; rows 16-byte aligned. */
+TADM_API tadm_status tadm_gemm(const void* A, const void* B, void* C, int M, int N, int K, int lda, int ldb,
+                      int ldc, int dtype, int c_dtype, tadm_stream stream);
+
+/* Per row of fp32 logits [rows, vocab]: tok = argmax over ids != mask_id
+ * (lowest id on ties), conf = 1 / sum_v exp(l_v - l_tok). */
+TADM_API tadm_status tadm_confidence(const float* logits, int rows, int vocab, int mask_id, float* conf,
+                            int32_t* tok, tadm_stream stream);
+
+/* Sampler update of z [batch, rows] (row stride ldz) from per-position conf
+ * and tok ([batch, rows], dense): unmask the k masked positions of largest
+ * conf in each sequence (ties -> lower position); selected [batch, k] or
+ * NULL. */
+TADM_API tadm_status tadm_topk_unmask(int32_t* z, int ldz, const float* conf, const int32_t* tok, int batch,
+                             int rows, int k, int mask_id, int32_t* selected, tadm_stream stream);
+
+/* softmax(Q K^T / sqrt(hd)) V for queries at positions ctx .. ctx+rows-1 over
+ * keys 0 .. ctx+rows-1 (keys < ctx always visible; the rest bidirectional,
+ * or causal if `causal`).  dtype 1: bf16, 0: fp32.
+ * q: [batch, n_heads, rows, hd]; k, v: [batch, n_kv_heads, kv_stride, hd];
+ * o: [batch*rows, n_heads*hd]. */
+TADM_API tadm_status tadm_attention(const void* q, const void* k, const void* v, void* o, int batch,
+                           int n_heads, int n_kv_heads, int head_dim, int rows, int ctx,
+                           int kv_stride, int causal, int dtype, tadm_stream stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* TADM_H */

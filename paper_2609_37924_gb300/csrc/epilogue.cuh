@@ -1,0 +1,315 @@
+// GEMM epilogues.  Every GEMM of the path computes acc = A B^T for one output
+// row at a time and hands the accumulator row, in chunks of 32 fp32 columns,
+// to one of these functions.  They fuse what follows each projection: the
+// residual add, RoPE and the K/V cache write, the GLU activation, the two
+// fusion-module epilogues (gate / hidden activations; h + g * Delta), and the
+// per-row partial max / argmax / sum-exp of the output head.
+#pragma once
+#include "common.cuh"
+
+namespace tadm {
+
+enum EpiKind : int {
+  EPI_STORE = 0,     // out = acc
+  EPI_RESID = 1,     // resid += acc (+ bias)
+  EPI_QKV = 2,       // split into Q / K / V heads, optional RoPE, K/V into the cache
+  EPI_GLU = 3,       // out = act(gate) * up (gate and up are the two halves of the tile)
+  EPI_FUSION1 = 4,   // [g | hidden] = [sigmoid(acc + b) | GELU(acc + b)]
+  EPI_FUSION2 = 5,   // out = h + g * (acc + b)
+  EPI_LMHEAD = 6,    // per-row (max, sum exp, argmax) partial of this column tile
+  EPI_PA_UP = 7,     // out = H0 + g[row] * sH[row] * acc
+  EPI_SILU = 8,      // out = SiLU(acc)
+  EPI_ADD = 9,       // out = base + acc (+ act copy in out2)
+  EPI_PA_GATE = 10,  // g[row] = sigmoid(sum_j SiLU(acc_j) w_j + b), single column tile
+};
+
+struct EpiParams {
+  int M, N;                 // output rows / columns (EPI_GLU: the F output columns)
+  void* out;
+  int ldo, out_bf16;        // out element type: bf16 (1) or fp32 (0)
+  float* resid;
+  int ldr;
+  const float* base;        // EPI_ADD base, EPI_FUSION2 h, EPI_PA_UP H0
+  int ldb;
+  const void* bias;         // [N] weights dtype
+  int bias_bf16;
+  // EPI_QKV
+  void *q, *k, *v;
+  int R, ctx, kv_stride, n_heads, n_kv_heads, head_dim, rope;
+  const float2* rope_tab;   // [position][head_dim / 2] = (cos, sin)
+  // EPI_GLU
+  int glu;                  // 0 SiLU, 1 tanh-GELU
+  // EPI_FUSION1 / EPI_ADD
+  int d_split;
+  void* out2;
+  int ldo2;
+  // EPI_FUSION2 (act type [M, N]) / EPI_PA_UP (fp32 [M])
+  const void* gate;
+  int ldg;
+  const float* rowscale;
+  // EPI_LMHEAD
+  float* part;              // [M][n_tiles][3] = (max, sum, argmax bits)
+  int n_tiles, mask_id;
+  float* logits;            // optional fp32 [M, ld_logits]
+  int ld_logits;
+  // EPI_PA_GATE: vec = W_g2 [N] (weights dtype), bias = b_g [1]
+  const void* vec;
+};
+
+__device__ __forceinline__ float ld_param(const void* p, int bf, int i) {
+  return bf ? __bfloat162float(static_cast<const bf16*>(p)[i]) : static_cast<const float*>(p)[i];
+}
+
+__device__ __forceinline__ float silu_f(float x) { return x / (1.0f + expf(-x)); }
+__device__ __forceinline__ float sigmoid_f(float x) { return 1.0f / (1.0f + expf(-x)); }
+__device__ __forceinline__ float gelu_erf_f(float x) { return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f)); }
+__device__ __forceinline__ float gelu_tanh_f(float x) {
+  return 0.5f * x * (1.0f + tanhf(0.79788456080286536f * (x + 0.044715f * x * x * x)));
+}
+
+// Stores 32 consecutive values (n0 .. n0+31) of one row; `n_valid` of them.
+__device__ __forceinline__ void store32(void* base, int bf, size_t off, const float (&v)[32], int n_valid) {
+  if (bf) {
+    bf16* p = static_cast<bf16*>(base) + off;
+    if (n_valid >= 32 && (off & 7) == 0) {
+      uint4* p4 = reinterpret_cast<uint4*>(p);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        __nv_bfloat162 t0 = __floats2bfloat162_rn(v[8 * i + 0], v[8 * i + 1]);
+        __nv_bfloat162 t1 = __floats2bfloat162_rn(v[8 * i + 2], v[8 * i + 3]);
+        __nv_bfloat162 t2 = __floats2bfloat162_rn(v[8 * i + 4], v[8 * i + 5]);
+        __nv_bfloat162 t3 = __floats2bfloat162_rn(v[8 * i + 6], v[8 * i + 7]);
+        uint4 u;
+        u.x = *reinterpret_cast<uint32_t*>(&t0);
+        u.y = *reinterpret_cast<uint32_t*>(&t1);
+        u.z = *reinterpret_cast<uint32_t*>(&t2);
+        u.w = *reinterpret_cast<uint32_t*>(&t3);
+        p4[i] = u;
+      }
+    } else {
+      for (int i = 0; i < n_valid; ++i) p[i] = __float2bfloat16_rn(v[i]);
+    }
+  } else {
+    float* p = static_cast<float*>(base) + off;
+    if (n_valid >= 32 && (off & 3) == 0) {
+      float4* p4 = reinterpret_cast<float4*>(p);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) p4[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+    } else {
+      for (int i = 0; i < n_valid; ++i) p[i] = v[i];
+    }
+  }
+}
+
+__device__ __forceinline__ void load32f(const float* p, int n_valid, float (&v)[32]) {
+  if (n_valid >= 32 && (reinterpret_cast<uintptr_t>(p) & 15) == 0) {
+    const float4* p4 = reinterpret_cast<const float4*>(p);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      float4 t = p4[i];
+      v[4 * i] = t.x; v[4 * i + 1] = t.y; v[4 * i + 2] = t.z; v[4 * i + 3] = t.w;
+    }
+  } else {
+    for (int i = 0; i < 32; ++i) v[i] = i < n_valid ? p[i] : 0.0f;
+  }
+}
+
+__device__ __forceinline__ void load32a(const void* p, int bf, size_t off, int n_valid, float (&v)[32]) {
+  if (bf) {
+    const bf16* q = static_cast<const bf16*>(p) + off;
+    for (int i = 0; i < 32; ++i) v[i] = i < n_valid ? __bfloat162float(q[i]) : 0.0f;
+  } else {
+    load32f(static_cast<const float*>(p) + off, n_valid, v);
+  }
+}
+
+// One output row of one column tile.  `ncols` accumulator columns (a multiple
+// of 64) are available from src.load(chunk, v); the tile's first output column
+// is n_blk * ncols (n_blk * ncols / 2 for EPI_GLU).  Control flow is uniform
+// across a warp except for the stores (src.load may be warp-collective).
+template <int EPI, class Src>
+__device__ __forceinline__ void epilogue_row(const EpiParams& p, int m, int n_blk, int ncols, Src& src) {
+  const bool row_ok = m < p.M;
+  const int nch = ncols / 32;
+  float v[32];
+  if constexpr (EPI == EPI_STORE || EPI == EPI_RESID || EPI == EPI_SILU || EPI == EPI_ADD ||
+                EPI == EPI_FUSION1 || EPI == EPI_FUSION2 || EPI == EPI_PA_UP) {
+    for (int c = 0; c < nch; ++c) {
+      src.load(c, v);
+      const int n0 = n_blk * ncols + 32 * c;
+      const int nv = min(32, p.N - n0);
+      if (!row_ok || nv <= 0) continue;
+      const size_t mrow = static_cast<size_t>(m);
+      if constexpr (EPI == EPI_STORE) {
+        store32(p.out, p.out_bf16, mrow * p.ldo + n0, v, nv);
+      } else if constexpr (EPI == EPI_SILU) {
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = silu_f(v[i]);
+        store32(p.out, p.out_bf16, mrow * p.ldo + n0, v, nv);
+      } else if constexpr (EPI == EPI_RESID) {
+        float r[32];
+        float* rp = p.resid + mrow * p.ldr + n0;
+        load32f(rp, nv, r);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          float b = (p.bias && i < nv) ? ld_param(p.bias, p.bias_bf16, n0 + i) : 0.0f;
+          r[i] += v[i] + b;
+        }
+        store32(p.resid, 0, mrow * p.ldr + n0, r, nv);
+      } else if constexpr (EPI == EPI_ADD) {
+        float r[32];
+        load32f(p.base + mrow * p.ldb + n0, nv, r);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) r[i] += v[i];
+        store32(p.out, 0, mrow * p.ldo + n0, r, nv);
+        if (p.out2) store32(p.out2, p.out_bf16, mrow * p.ldo2 + n0, r, nv);
+      } else if constexpr (EPI == EPI_FUSION1) {
+        float g[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const int n = n0 + i;
+          const float b = (i < nv) ? ld_param(p.bias, p.bias_bf16, n) : 0.0f;
+          g[i] = (n < p.d_split) ? sigmoid_f(v[i] + b) : gelu_erf_f(v[i] + b);
+        }
+        // d_split is a multiple of 32: a chunk is all gate or all hidden
+        if (n0 < p.d_split)
+          store32(p.out, p.out_bf16, mrow * p.ldo + n0, g, min(nv, p.d_split - n0));
+        else
+          store32(p.out2, p.out_bf16, mrow * p.ldo2 + (n0 - p.d_split), g, nv);
+      } else if constexpr (EPI == EPI_FUSION2) {
+        float h[32], g[32];
+        load32f(p.base + mrow * p.ldb + n0, nv, h);
+        load32a(p.gate, p.out_bf16, mrow * p.ldg + n0, nv, g);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const float b = (p.bias && i < nv) ? ld_param(p.bias, p.bias_bf16, n0 + i) : 0.0f;
+          h[i] = h[i] + g[i] * (v[i] + b);
+        }
+        store32(p.out, 0, mrow * p.ldo + n0, h, nv);
+      } else if constexpr (EPI == EPI_PA_UP) {
+        float h[32];
+        load32f(p.base + mrow * p.ldb + n0, nv, h);
+        const float gs = static_cast<const float*>(p.gate)[m] * p.rowscale[m];
+#pragma unroll
+        for (int i = 0; i < 32; ++i) h[i] = h[i] + gs * v[i];
+        store32(p.out, 0, mrow * p.ldo + n0, h, nv);
+      }
+    }
+  } else if constexpr (EPI == EPI_GLU) {
+    const int half = ncols / 2;
+    for (int c = 0; c < half / 32; ++c) {
+      float u[32];
+      src.load(c, v);
+      src.load(c + half / 32, u);
+      const int n0 = n_blk * half + 32 * c;
+      const int nv = min(32, p.N - n0);
+      if (!row_ok || nv <= 0) continue;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) v[i] = (p.glu ? gelu_tanh_f(v[i]) : silu_f(v[i])) * u[i];
+      store32(p.out, p.out_bf16, static_cast<size_t>(m) * p.ldo + n0, v, nv);
+    }
+  } else if constexpr (EPI == EPI_QKV) {
+    const int hd = p.head_dim;
+    const int hpt = ncols / hd;       // heads per tile
+    const int b = m / p.R, r = m - (m / p.R) * p.R;
+    const int pos = p.ctx + r;
+    for (int hh = 0; hh < hpt; ++hh) {
+      const int nb = n_blk * ncols + hh * hd;
+      const int gh = nb / hd;
+      int region = 2, head = gh - p.n_heads - p.n_kv_heads;
+      if (gh < p.n_heads) { region = 0; head = gh; }
+      else if (gh < p.n_heads + p.n_kv_heads) { region = 1; head = gh - p.n_heads; }
+      void* dst;
+      size_t off;
+      if (region == 0) {
+        dst = p.q;
+        off = ((static_cast<size_t>(b) * p.n_heads + head) * p.R + r) * hd;
+      } else {
+        dst = region == 1 ? p.k : p.v;
+        off = ((static_cast<size_t>(b) * p.n_kv_heads + head) * p.kv_stride + pos) * hd;
+      }
+      const bool ok = row_ok && nb < p.N;
+      if (hd == 32) {  // rotate-half pairs (i, i + 16) inside one chunk
+        src.load(hh, v);
+        if (!ok) continue;
+        if (p.rope && region < 2) {
+          const float2* tab = p.rope_tab + static_cast<size_t>(pos) * 16;
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const float2 cs = tab[i];
+            const float a = v[i], c2 = v[i + 16];
+            v[i] = a * cs.x - c2 * cs.y;
+            v[i + 16] = c2 * cs.x + a * cs.y;
+          }
+        }
+        store32(dst, p.out_bf16, off, v, 32);
+        continue;
+      }
+      for (int j2 = 0; j2 < hd / 64; ++j2) {
+        float w[32];
+        const int ca = (hh * hd) / 32 + j2, cb = ca + hd / 64;
+        src.load(ca, v);
+        src.load(cb, w);
+        if (!ok) continue;
+        if (p.rope && region < 2) {
+          const float2* tab = p.rope_tab + static_cast<size_t>(pos) * (hd / 2) + 32 * j2;
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float2 cs = tab[i];
+            const float a = v[i], c2 = w[i];
+            v[i] = a * cs.x - c2 * cs.y;
+            w[i] = c2 * cs.x + a * cs.y;
+          }
+        }
+        store32(dst, p.out_bf16, off + 32 * j2, v, 32);
+        store32(dst, p.out_bf16, off + hd / 2 + 32 * j2, w, 32);
+      }
+    }
+  } else if constexpr (EPI == EPI_LMHEAD) {
+    float mx = -INFINITY, sum = 0.0f;
+    int arg = -1;
+    for (int c = 0; c < nch; ++c) {
+      src.load(c, v);
+      const int n0 = n_blk * ncols + 32 * c;
+      const int nv = min(32, p.N - n0);
+      if (!row_ok || nv <= 0) continue;
+      if (p.logits) store32(p.logits, 0, static_cast<size_t>(m) * p.ld_logits + n0, v, nv);
+      float cmx = -INFINITY;
+      int carg = -1;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        const int n = n0 + i;
+        if (i < nv && n != p.mask_id && v[i] > cmx) { cmx = v[i]; carg = n; }
+      }
+      if (carg < 0) continue;
+      const float nm = fmaxf(mx, cmx);
+      float s = (mx == -INFINITY) ? 0.0f : sum * expf(mx - nm);
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        const int n = n0 + i;
+        if (i < nv && n != p.mask_id) s += expf(v[i] - nm);
+      }
+      if (cmx > mx) arg = carg;
+      mx = nm;
+      sum = s;
+    }
+    if (row_ok) {
+      float* o = p.part + (static_cast<size_t>(m) * p.n_tiles + n_blk) * 3;
+      o[0] = mx;
+      o[1] = sum;
+      o[2] = __int_as_float(arg);
+    }
+  } else if constexpr (EPI == EPI_PA_GATE) {
+    float s = 0.0f;
+    for (int c = 0; c < nch; ++c) {
+      src.load(c, v);
+      const int n0 = 32 * c;
+      const int nv = min(32, p.N - n0);
+      if (!row_ok || nv <= 0) continue;
+      for (int i = 0; i < nv; ++i) s += silu_f(v[i]) * ld_param(p.vec, p.bias_bf16, n0 + i);
+    }
+    if (row_ok) static_cast<float*>(p.out)[m] = sigmoid_f(s + ld_param(p.bias, p.bias_bf16, 0));
+  }
+}
+
+}  // namespace tadm

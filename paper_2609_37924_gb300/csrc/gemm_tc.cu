@@ -1,0 +1,283 @@
+// bf16 GEMM on the 5th-generation tensor cores (tcgen05) for sm_103a.
+//
+//   acc[M, N] = A[M, K] * B[N, K]^T     (A, B bf16, K-major; fp32 accumulate)
+//
+// Persistent kernel, one CTA per SM, warp-specialised:
+//   warp 0      one thread issues TMA loads of A / B tiles into a 4-stage
+//               shared-memory ring (128-byte swizzle);
+//   warp 1      allocates 512 TMEM columns (two 128 x 256 fp32 accumulators)
+//               and one thread issues tcgen05.mma (M=128, N=256, K=16);
+//   warps 2..5  epilogue: tcgen05.ld the accumulator rows (one TMEM lane per
+//               thread) and run the fused epilogue of epilogue.cuh, while the
+//               MMA warp fills the other accumulator.
+// Every mbarrier wait is bounded (mbar_wait_bounded): a role that gives up
+// raises a shared abort flag and the device status word, and the CTA drains
+// its in-flight copies and MMAs, frees TMEM and exits.
+#include <cudaTypedefs.h>
+#include <mutex>
+
+#include "epilogue.cuh"
+#include "kernels.h"
+
+namespace tadm {
+
+namespace {
+constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
+constexpr int A_BYTES = BM * BK * 2;   // 16 KB
+constexpr int B_BYTES = BN * BK * 2;   // 32 KB
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int TMEM_COLS = 512;
+constexpr int NUM_THREADS = 192;
+constexpr size_t SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;
+
+struct TmemSrc {
+  uint32_t taddr;
+  __device__ __forceinline__ void load(int chunk, float (&v)[32]) {
+    __syncwarp();  // tcgen05.ld is warp-collective: reconverge after divergent stores
+    tmem_ld32(taddr + 32 * chunk, v);
+  }
+};
+
+struct TcArgs {
+  int M, N_acc, K;         // N_acc: accumulator columns in total (2F for GLU)
+  int b_split;             // >0: B tile = 128 rows at n*128 and 128 rows at b_split + n*128
+  int n_tiles_n;
+  int* status;
+  EpiParams ep;
+};
+
+template <int EPI>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const TcArgs args) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + STAGES * A_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint64_t* empty = full + STAGES;
+  uint64_t* tfull = empty + STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* drain = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], 128);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int num_m = (args.M + BM - 1) / BM;
+  const int tiles = num_m * args.n_tiles_n;
+  const int kblocks = (args.K + BK - 1) / BK;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------------------------------------------------------- producer
+      int stage = 0;
+      uint32_t phase = 0;
+      int issued[STAGES];
+      for (int s = 0; s < STAGES; ++s) issued[s] = 0;
+      for (int tile = blockIdx.x; tile < tiles && !*abort_flag; tile += gridDim.x) {
+        const int mb = tile % num_m, nb = tile / num_m;
+        bool ok = true;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait_bounded(&empty[stage], phase ^ 1, abort_flag, args.status)) { ok = false; break; }
+          mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
+          tma_load_2d(sA + stage * A_BYTES, &tmA, &full[stage], kb * BK, mb * BM);
+          if (args.b_split > 0) {
+            tma_load_2d(sB + stage * B_BYTES, &tmB, &full[stage], kb * BK, nb * (BN / 2));
+            tma_load_2d(sB + stage * B_BYTES + B_BYTES / 2, &tmB, &full[stage], kb * BK,
+                        args.b_split + nb * (BN / 2));
+          } else {
+            tma_load_2d(sB + stage * B_BYTES, &tmB, &full[stage], kb * BK, nb * BN);
+          }
+          ++issued[stage];
+          if (++stage == STAGES) { stage = 0; phase ^= 1; }
+        }
+        if (!ok) break;
+      }
+      // every copy this thread started has landed before the CTA may exit
+      for (int s = 0; s < STAGES; ++s)
+        if (issued[s] > 0) {
+          volatile int never = 0;
+          mbar_wait_bounded(&full[s], (issued[s] - 1) & 1, &never, args.status);
+        }
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------------------------------------------------------- MMA issuer
+      constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      for (int tile = blockIdx.x; tile < tiles && !*abort_flag; tile += gridDim.x) {
+        if (!mbar_wait_bounded(&tempty[acc], acc_phase ^ 1, abort_flag, args.status)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * BN;
+        bool ok = true;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait_bounded(&full[stage], phase, abort_flag, args.status)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(sA + stage * A_BYTES);
+          const uint32_t b0 = smem_u32(sB + stage * B_BYTES);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k) {
+            umma_bf16(d_tmem, sdesc_kmajor_sw128(a0 + 32 * k), sdesc_kmajor_sw128(b0 + 32 * k), idesc,
+                      (kb | k) != 0);
+          }
+          umma_commit(&empty[stage]);
+          if (++stage == STAGES) { stage = 0; phase ^= 1; }
+        }
+        if (!ok) break;
+        umma_commit(&tfull[acc]);
+        if (++acc == 2) { acc = 0; acc_phase ^= 1; }
+      }
+      // all MMAs issued by this thread are complete before TMEM is freed
+      umma_commit(drain);
+      volatile int never = 0;
+      mbar_wait_bounded(drain, 0, &never, args.status);
+    }
+  } else {
+    // ------------------------------------------------------------------ epilogue
+    const int quad = warp & 3;   // TMEM lanes 32*quad .. 32*quad+31
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
+      if (!mbar_wait_bounded(&tfull[acc], acc_phase, abort_flag, args.status)) break;
+      tc_fence_after();
+      const int mb = tile % num_m, nb = tile / num_m;
+      TmemSrc src{tmem_base + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(quad * 32) << 16)};
+      epilogue_row<EPI>(args.ep, mb * BM + quad * 32 + lane, nb, BN, src);
+      tc_fence_before();
+      mbar_arrive(&tempty[acc]);
+      if (++acc == 2) { acc = 0; acc_phase ^= 1; }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem_base, TMEM_COLS);
+  }
+}
+
+// --------------------------------------------------------------------- host
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::once_flag g_encode_once;
+int g_num_sms = 0;
+
+bool get_encoder() {
+  std::call_once(g_encode_once, [] {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
+  });
+  return g_encode != nullptr;
+}
+
+// 2-D bf16 tensor map over rows x cols (row stride ld elements), box of
+// box_rows x 64 elements, 128-byte swizzle, zero fill out of bounds.
+bool make_map(CUtensorMap* m, const void* ptr, int64_t rows, int64_t cols, int64_t ld, int box_rows) {
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld * 2)};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+template <int EPI>
+cudaError_t launch_epi(const CUtensorMap& ta, const CUtensorMap& tb, const TcArgs& a, int grid, cudaStream_t s) {
+  static bool attr_set = false;
+  if (!attr_set) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(SMEM_BYTES));
+    if (e != cudaSuccess) return e;
+    attr_set = true;
+  }
+  gemm_tc_kernel<EPI><<<grid, NUM_THREADS, SMEM_BYTES, s>>>(ta, tb, a);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
+  if (!get_encoder()) return "cuTensorMapEncodeTiled is unavailable";
+  if (g.M <= 0 || g.N <= 0 || g.K <= 0) return nullptr;
+  if (g.K % 8 || g.lda % 8 || g.ldb % 8) return "bf16 GEMM needs K, lda, ldb multiples of 8";
+  if ((reinterpret_cast<uintptr_t>(g.A) | reinterpret_cast<uintptr_t>(g.B)) & 15)
+    return "bf16 GEMM operands must be 16-byte aligned";
+  const bool glu = g.epi == EPI_GLU;
+  CUtensorMap ta, tb;
+  if (!make_map(&ta, g.A, g.A_rows > 0 ? g.A_rows : g.M, g.K, g.lda, BM)) return "tensor map (A) encode failed";
+  const int64_t b_rows = glu ? 2LL * g.N : g.N;
+  if (!make_map(&tb, g.B, b_rows, g.K, g.ldb, glu ? BN / 2 : BN)) return "tensor map (B) encode failed";
+  TcArgs a;
+  a.M = g.M;
+  a.K = g.K;
+  a.N_acc = glu ? 2 * g.N : g.N;
+  a.b_split = glu ? g.N : 0;
+  a.n_tiles_n = glu ? (g.N + BN / 2 - 1) / (BN / 2) : (g.N + BN - 1) / BN;
+  if (glu && g.N % (BN / 2)) return "GLU GEMM needs the FFN width to be a multiple of 128";
+  if (g.epi == EPI_QKV && BN % g.ep.head_dim) return "head_dim must divide 256";
+  if (g.epi == EPI_PA_GATE && g.N > BN) return "gate GEMM needs N <= 256";
+  a.status = g.status;
+  a.ep = g.ep;
+  a.ep.M = g.M;
+  a.ep.N = g.N;
+  a.ep.n_tiles = a.n_tiles_n;
+  const int tiles = ((g.M + BM - 1) / BM) * a.n_tiles_n;
+  const int grid = tiles < g_num_sms ? tiles : g_num_sms;
+  cudaError_t e;
+  switch (g.epi) {
+    case EPI_STORE: e = launch_epi<EPI_STORE>(ta, tb, a, grid, s); break;
+    case EPI_RESID: e = launch_epi<EPI_RESID>(ta, tb, a, grid, s); break;
+    case EPI_QKV: e = launch_epi<EPI_QKV>(ta, tb, a, grid, s); break;
+    case EPI_GLU: e = launch_epi<EPI_GLU>(ta, tb, a, grid, s); break;
+    case EPI_FUSION1: e = launch_epi<EPI_FUSION1>(ta, tb, a, grid, s); break;
+    case EPI_FUSION2: e = launch_epi<EPI_FUSION2>(ta, tb, a, grid, s); break;
+    case EPI_LMHEAD: e = launch_epi<EPI_LMHEAD>(ta, tb, a, grid, s); break;
+    case EPI_PA_UP: e = launch_epi<EPI_PA_UP>(ta, tb, a, grid, s); break;
+    case EPI_SILU: e = launch_epi<EPI_SILU>(ta, tb, a, grid, s); break;
+    case EPI_ADD: e = launch_epi<EPI_ADD>(ta, tb, a, grid, s); break;
+    case EPI_PA_GATE: e = launch_epi<EPI_PA_GATE>(ta, tb, a, grid, s); break;
+    default: return "unknown epilogue";
+  }
+  return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
+}
+
+int gemm_tc_tiles_n(int N, int epi) { return epi == EPI_GLU ? (N + 127) / 128 : (N + 255) / 256; }
+
+}  // namespace tadm

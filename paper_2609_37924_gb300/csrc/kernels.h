@@ -1,0 +1,65 @@
+// Host-side launchers of the sm_103a kernels (internal to libtadm).  Each
+// returns nullptr on success or a static error string.
+#pragma once
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "epilogue.cuh"
+
+namespace tadm {
+
+struct GemmCall {
+  const void* A;   // [M, K] (A_rows rows visible to the tensor map when > 0)
+  const void* B;   // [N, K]  (EPI_GLU: [2N, K], gate rows then up rows)
+  int M, N, K, lda, ldb;
+  int64_t A_rows;
+  int epi;
+  EpiParams ep;
+  int* status;
+};
+
+// tcgen05 path (bf16 operands)
+const char* gemm_tc(const GemmCall& g, cudaStream_t s);
+int gemm_tc_tiles_n(int N, int epi);
+// CUDA-core path (fp32 operands)
+const char* gemm_simt(const GemmCall& g, cudaStream_t s);
+int gemm_simt_tiles_n(int N, int epi);
+
+struct AttnCall {
+  const void *q, *k, *v;
+  void* o;
+  int batch, n_heads, n_kv_heads, head_dim, rows, ctx, kv_stride, causal;
+  int bf16;
+};
+const char* attention(const AttnCall& a, cudaStream_t s);
+
+// row kernels (act = bf16 when act_bf16 else fp32)
+const char* embed_rows(const int32_t* z, int ldz, int batch, int rows, const void* E, int e_bf16, int d,
+                       int vocab, float* out, float* out2, cudaStream_t s);
+const char* rmsnorm_rows(const float* x, int M, int d, const void* gain, int w_bf16, float eps, void* out,
+                         int ldo, int act_bf16, cudaStream_t s);
+const char* ln_pair_rows(const float* c, const float* h, int M, int d, const void* wc, const void* bc,
+                         const void* wh, const void* bh, int w_bf16, float eps, void* u, int act_bf16,
+                         cudaStream_t s);
+const char* layernorm_rows(const float* x, int M, int d, const void* w, const void* b, int w_bf16, float eps,
+                           float* out, cudaStream_t s);
+const char* rms_scale_rows(const float* x, int M, int d, float eps, float* s_out, cudaStream_t st);
+const char* scale_rows(const float* x, const float* sc, int M, int d, void* out, int act_bf16, cudaStream_t s);
+const char* concat_rows(const float* const* parts, const int* widths, int n_parts, int M, void* out,
+                        int act_bf16, cudaStream_t s);
+const char* sub_rows(const float* a, const float* b, int M, int d, float* out, cudaStream_t s);
+const char* rope_table(float2* tab, int n_pos, int head_dim, float theta, cudaStream_t s);
+const char* fill_canvas(int32_t* z, int ldz, const int32_t* prompt, int batch, int prompt_len, int total,
+                        int mask_id, cudaStream_t s);
+const char* copy_rows_i32(const int32_t* src, int lds, int32_t* dst, int ldd, int batch, int cols,
+                          cudaStream_t s);
+
+// sampler
+const char* confidence_rows(const float* logits, int rows, int vocab, int ld, int mask_id, float* conf,
+                            int32_t* tok, cudaStream_t s);
+const char* combine_partials(const float* part, int rows, int n_tiles, float* conf, int32_t* tok,
+                             cudaStream_t s);
+const char* topk_unmask(int32_t* z, int ldz, const float* conf, const int32_t* tok, int batch, int rows, int k,
+                        int mask_id, int32_t* selected, cudaStream_t s);
+
+}  // namespace tadm

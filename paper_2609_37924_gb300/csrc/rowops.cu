@@ -1,0 +1,301 @@
+// Row-wise kernels of the path (HBM-bound, one warp per row, float4 I/O):
+// token-embedding gather (S), RMSNorm ahead of each projection, the two
+// LayerNorms that build the fusion input u = [LN(c); LN(h)] and the output
+// LayerNorm of the gated-MLP fusion (App. C.2), the RMS scales and feature
+// concatenations of the paired-attention fusion (App. C.1), the RoPE table,
+// and canvas set-up.
+#include "kernels.h"
+
+namespace tadm {
+namespace {
+
+constexpr int WPB = 8;  // warps (rows) per block
+
+template <class T>
+__device__ __forceinline__ void store_act(void* out, size_t i, float v);
+template <>
+__device__ __forceinline__ void store_act<float>(void* out, size_t i, float v) { static_cast<float*>(out)[i] = v; }
+template <>
+__device__ __forceinline__ void store_act<bf16>(void* out, size_t i, float v) {
+  static_cast<bf16*>(out)[i] = __float2bfloat16_rn(v);
+}
+
+__device__ __forceinline__ float ldw(const void* w, int bf, int i) {
+  return bf ? __bfloat162float(static_cast<const bf16*>(w)[i]) : static_cast<const float*>(w)[i];
+}
+
+__global__ void embed_kernel(const int32_t* __restrict__ z, int ldz, int rows, int M, const void* __restrict__ E,
+                             int e_bf16, int d, int vocab, float* __restrict__ out, float* __restrict__ out2) {
+  const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (m >= M) return;
+  const int b = m / rows, r = m - b * rows;
+  int tok = z[static_cast<size_t>(b) * ldz + r];
+  tok = tok < 0 ? 0 : (tok >= vocab ? vocab - 1 : tok);  // ids are validated by the caller; never read outside E
+  float* o = out + static_cast<size_t>(m) * d;
+  float* o2 = out2 ? out2 + static_cast<size_t>(m) * d : nullptr;
+  if (e_bf16) {
+    const bf16* e = static_cast<const bf16*>(E) + static_cast<size_t>(tok) * d;
+    for (int j = lane * 2; j < d; j += 64) {
+      const float2 v = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(e + j));
+      *reinterpret_cast<float2*>(o + j) = v;
+      if (o2) *reinterpret_cast<float2*>(o2 + j) = v;
+    }
+  } else {
+    const float* e = static_cast<const float*>(E) + static_cast<size_t>(tok) * d;
+    for (int j = lane * 4; j < d; j += 128) {
+      const float4 v = *reinterpret_cast<const float4*>(e + j);
+      *reinterpret_cast<float4*>(o + j) = v;
+      if (o2) *reinterpret_cast<float4*>(o2 + j) = v;
+    }
+  }
+}
+
+// out = x / sqrt(mean(x^2) + eps) * gain
+template <class T>
+__global__ void rmsnorm_kernel(const float* __restrict__ x, int M, int d, const void* __restrict__ gain, int w_bf16,
+                               float eps, void* __restrict__ out, int ldo) {
+  const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (m >= M) return;
+  const float* xr = x + static_cast<size_t>(m) * d;
+  float ss = 0.0f;
+  for (int j = lane * 4; j < d; j += 128) {
+    const float4 v = *reinterpret_cast<const float4*>(xr + j);
+    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+  }
+  ss = warp_sum(ss);
+  const float inv = rsqrtf(ss / static_cast<float>(d) + eps);
+  for (int j = lane * 4; j < d; j += 128) {
+    const float4 v = *reinterpret_cast<const float4*>(xr + j);
+    const size_t o = static_cast<size_t>(m) * ldo + j;
+    store_act<T>(out, o + 0, v.x * inv * ldw(gain, w_bf16, j + 0));
+    store_act<T>(out, o + 1, v.y * inv * ldw(gain, w_bf16, j + 1));
+    store_act<T>(out, o + 2, v.z * inv * ldw(gain, w_bf16, j + 2));
+    store_act<T>(out, o + 3, v.w * inv * ldw(gain, w_bf16, j + 3));
+  }
+}
+
+__device__ __forceinline__ void row_mean_var(const float* xr, int d, int lane, float& mean, float& rstd, float eps) {
+  float s = 0.0f;
+  for (int j = lane * 4; j < d; j += 128) {
+    const float4 v = *reinterpret_cast<const float4*>(xr + j);
+    s += v.x + v.y + v.z + v.w;
+  }
+  mean = warp_sum(s) / static_cast<float>(d);
+  float q = 0.0f;
+  for (int j = lane * 4; j < d; j += 128) {
+    const float4 v = *reinterpret_cast<const float4*>(xr + j);
+    const float a = v.x - mean, b = v.y - mean, c = v.z - mean, e = v.w - mean;
+    q += a * a + b * b + c * c + e * e;
+  }
+  rstd = rsqrtf(warp_sum(q) / static_cast<float>(d) + eps);
+}
+
+// u[m] = [LN(c[m]) * wc + bc ; LN(h[m]) * wh + bh]   (act, [M, 2d])
+template <class T>
+__global__ void ln_pair_kernel(const float* __restrict__ c, const float* __restrict__ h, int M, int d,
+                               const void* wc, const void* bc, const void* wh, const void* bh, int w_bf16, float eps,
+                               void* __restrict__ u) {
+  const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (m >= M) return;
+  for (int part = 0; part < 2; ++part) {
+    const float* xr = (part ? h : c) + static_cast<size_t>(m) * d;
+    const void* w = part ? wh : wc;
+    const void* b = part ? bh : bc;
+    float mean, rstd;
+    row_mean_var(xr, d, lane, mean, rstd, eps);
+    for (int j = lane; j < d; j += 32)
+      store_act<T>(u, static_cast<size_t>(m) * 2 * d + part * d + j,
+                   (xr[j] - mean) * rstd * ldw(w, w_bf16, j) + ldw(b, w_bf16, j));
+  }
+}
+
+__global__ void layernorm_kernel(const float* __restrict__ x, int M, int d, const void* w, const void* b, int w_bf16,
+                                 float eps, float* __restrict__ out) {
+  const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (m >= M) return;
+  const float* xr = x + static_cast<size_t>(m) * d;
+  float mean, rstd;
+  row_mean_var(xr, d, lane, mean, rstd, eps);
+  for (int j = lane; j < d; j += 32)
+    out[static_cast<size_t>(m) * d + j] = (xr[j] - mean) * rstd * ldw(w, w_bf16, j) + ldw(b, w_bf16, j);
+}
+
+__global__ void rms_scale_kernel(const float* __restrict__ x, int M, int d, float eps, float* __restrict__ s) {
+  const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (m >= M) return;
+  const float* xr = x + static_cast<size_t>(m) * d;
+  float ss = 0.0f;
+  for (int j = lane; j < d; j += 32) ss += xr[j] * xr[j];
+  ss = warp_sum(ss);
+  if (lane == 0) s[m] = sqrtf(ss / static_cast<float>(d) + eps);
+}
+
+template <class T>
+__global__ void scale_rows_kernel(const float* __restrict__ x, const float* __restrict__ sc, int M, int d,
+                                  void* __restrict__ out) {
+  const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (m >= M) return;
+  const float s = sc[m];
+  for (int j = lane; j < d; j += 32)
+    store_act<T>(out, static_cast<size_t>(m) * d + j, x[static_cast<size_t>(m) * d + j] / s);
+}
+
+struct Parts {
+  const float* p[4];
+  int w[4];
+  int n;
+};
+
+template <class T>
+__global__ void concat_kernel(Parts parts, int M, int width, void* __restrict__ out) {
+  const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (m >= M) return;
+  int col = 0;
+  for (int i = 0; i < parts.n; ++i) {
+    const float* src = parts.p[i] + static_cast<size_t>(m) * parts.w[i];
+    for (int j = lane; j < parts.w[i]; j += 32) store_act<T>(out, static_cast<size_t>(m) * width + col + j, src[j]);
+    col += parts.w[i];
+  }
+}
+
+__global__ void sub_kernel(const float* __restrict__ a, const float* __restrict__ b, size_t n, float* __restrict__ o) {
+  for (size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; i < n;
+       i += static_cast<size_t>(gridDim.x) * blockDim.x)
+    o[i] = a[i] - b[i];
+}
+
+// tab[pos][j] = (cos, sin)(pos * theta^(-2j/hd)), angles evaluated in double
+__global__ void rope_table_kernel(float2* tab, int n_pos, int half, int hd, double theta) {
+  const size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x;
+  if (i >= static_cast<size_t>(n_pos) * half) return;
+  const int pos = static_cast<int>(i / half), j = static_cast<int>(i % half);
+  const double inv = pow(theta, -2.0 * j / hd);
+  const double ang = static_cast<double>(pos) * inv;
+  tab[i] = make_float2(static_cast<float>(cos(ang)), static_cast<float>(sin(ang)));
+}
+
+__global__ void fill_canvas_kernel(int32_t* z, int ldz, const int32_t* prompt, int batch, int P, int total,
+                                   int mask_id) {
+  const size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x;
+  if (i >= static_cast<size_t>(batch) * total) return;
+  const int b = static_cast<int>(i / total), p = static_cast<int>(i % total);
+  z[static_cast<size_t>(b) * ldz + p] = p < P ? prompt[static_cast<size_t>(b) * P + p] : mask_id;
+}
+
+__global__ void copy_i32_kernel(const int32_t* src, int lds, int32_t* dst, int ldd, int batch, int cols) {
+  const size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x;
+  if (i >= static_cast<size_t>(batch) * cols) return;
+  const int b = static_cast<int>(i / cols), c = static_cast<int>(i % cols);
+  dst[static_cast<size_t>(b) * ldd + c] = src[static_cast<size_t>(b) * lds + c];
+}
+
+inline dim3 rows_grid(int M) { return dim3((M + WPB - 1) / WPB); }
+inline const char* err() {
+  cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
+}
+}  // namespace
+
+const char* embed_rows(const int32_t* z, int ldz, int batch, int rows, const void* E, int e_bf16, int d, int vocab,
+                       float* out, float* out2, cudaStream_t s) {
+  const int M = batch * rows;
+  if (M <= 0) return nullptr;
+  if (d % 4) return "d_model must be a multiple of 4";
+  embed_kernel<<<rows_grid(M), WPB * 32, 0, s>>>(z, ldz, rows, M, E, e_bf16, d, vocab, out, out2);
+  return err();
+}
+
+const char* rmsnorm_rows(const float* x, int M, int d, const void* gain, int w_bf16, float eps, void* out, int ldo,
+                         int act_bf16, cudaStream_t s) {
+  if (M <= 0) return nullptr;
+  if (act_bf16)
+    rmsnorm_kernel<bf16><<<rows_grid(M), WPB * 32, 0, s>>>(x, M, d, gain, w_bf16, eps, out, ldo);
+  else
+    rmsnorm_kernel<float><<<rows_grid(M), WPB * 32, 0, s>>>(x, M, d, gain, w_bf16, eps, out, ldo);
+  return err();
+}
+
+const char* ln_pair_rows(const float* c, const float* h, int M, int d, const void* wc, const void* bc, const void* wh,
+                         const void* bh, int w_bf16, float eps, void* u, int act_bf16, cudaStream_t s) {
+  if (M <= 0) return nullptr;
+  if (act_bf16)
+    ln_pair_kernel<bf16><<<rows_grid(M), WPB * 32, 0, s>>>(c, h, M, d, wc, bc, wh, bh, w_bf16, eps, u);
+  else
+    ln_pair_kernel<float><<<rows_grid(M), WPB * 32, 0, s>>>(c, h, M, d, wc, bc, wh, bh, w_bf16, eps, u);
+  return err();
+}
+
+const char* layernorm_rows(const float* x, int M, int d, const void* w, const void* b, int w_bf16, float eps,
+                           float* out, cudaStream_t s) {
+  if (M <= 0) return nullptr;
+  layernorm_kernel<<<rows_grid(M), WPB * 32, 0, s>>>(x, M, d, w, b, w_bf16, eps, out);
+  return err();
+}
+
+const char* rms_scale_rows(const float* x, int M, int d, float eps, float* s_out, cudaStream_t st) {
+  if (M <= 0) return nullptr;
+  rms_scale_kernel<<<rows_grid(M), WPB * 32, 0, st>>>(x, M, d, eps, s_out);
+  return err();
+}
+
+const char* scale_rows(const float* x, const float* sc, int M, int d, void* out, int act_bf16, cudaStream_t s) {
+  if (M <= 0) return nullptr;
+  if (act_bf16)
+    scale_rows_kernel<bf16><<<rows_grid(M), WPB * 32, 0, s>>>(x, sc, M, d, out);
+  else
+    scale_rows_kernel<float><<<rows_grid(M), WPB * 32, 0, s>>>(x, sc, M, d, out);
+  return err();
+}
+
+const char* concat_rows(const float* const* parts, const int* widths, int n_parts, int M, void* out, int act_bf16,
+                        cudaStream_t s) {
+  if (M <= 0) return nullptr;
+  if (n_parts < 1 || n_parts > 4) return "concat of 1..4 parts";
+  Parts p{};
+  int width = 0;
+  for (int i = 0; i < n_parts; ++i) {
+    p.p[i] = parts[i];
+    p.w[i] = widths[i];
+    width += widths[i];
+  }
+  p.n = n_parts;
+  if (act_bf16)
+    concat_kernel<bf16><<<rows_grid(M), WPB * 32, 0, s>>>(p, M, width, out);
+  else
+    concat_kernel<float><<<rows_grid(M), WPB * 32, 0, s>>>(p, M, width, out);
+  return err();
+}
+
+const char* sub_rows(const float* a, const float* b, int M, int d, float* out, cudaStream_t s) {
+  const size_t n = static_cast<size_t>(M) * d;
+  if (n == 0) return nullptr;
+  const int blocks = static_cast<int>((n + 255) / 256 < 65535 ? (n + 255) / 256 : 65535);
+  sub_kernel<<<blocks, 256, 0, s>>>(a, b, n, out);
+  return err();
+}
+
+const char* rope_table(float2* tab, int n_pos, int head_dim, float theta, cudaStream_t s) {
+  const size_t n = static_cast<size_t>(n_pos) * (head_dim / 2);
+  if (n == 0) return nullptr;
+  rope_table_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, s>>>(tab, n_pos, head_dim / 2, head_dim,
+                                                                            static_cast<double>(theta));
+  return err();
+}
+
+const char* fill_canvas(int32_t* z, int ldz, const int32_t* prompt, int batch, int prompt_len, int total,
+                        int mask_id, cudaStream_t s) {
+  const size_t n = static_cast<size_t>(batch) * total;
+  if (n == 0) return nullptr;
+  fill_canvas_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, s>>>(z, ldz, prompt, batch, prompt_len,
+                                                                             total, mask_id);
+  return err();
+}
+
+const char* copy_rows_i32(const int32_t* src, int lds, int32_t* dst, int ldd, int batch, int cols, cudaStream_t s) {
+  const size_t n = static_cast<size_t>(batch) * cols;
+  if (n == 0) return nullptr;
+  copy_i32_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, s>>>(src, lds, dst, ldd, batch, cols);
+  return err();
+}
+
+}  // namespace tadm

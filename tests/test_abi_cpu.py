@@ -1,0 +1,105 @@
+"""The C ABI without a GPU: the library loads, exports every declared entry
+point, and its host-only logic (schedule plan, layer-cost formula, weight
+inventory, argument validation) is right."""
+import ctypes
+import json
+import os
+import re
+
+import pytest
+
+import workloads as wl
+from oracle import tadm_oracle as O
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    import __graft_entry__ as g
+    g.build()
+    from paper_2609_37924_gb300 import tadm
+    return tadm
+
+
+def declared_functions():
+    names = set()
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            src = open(os.path.join(ROOT, "include", fn)).read()
+            names |= set(re.findall(r"^TADM_API\s+[\w\s\*]+?\b(tadm_\w+)\s*\(", src, flags=re.M))
+    return names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    so = lib.load_library()
+    names = declared_functions()
+    assert len(names) >= 20
+    for n in sorted(names):
+        assert hasattr(so, n), n
+    assert set(lib.ABI_FUNCTIONS) == names
+
+
+def test_plan_refresh_schedule(lib):
+    for (P, G, T, K, bl) in [(32, 96, 32, 4, 0), (256, 768, 128, 1, 0), (512, 128, 16, 4, 32), (8, 64, 16, 3, 32)]:
+        ev = lib.tadm_plan(P, G, T, K, bl)
+        nblk = G // bl if bl else 1
+        Gb = bl if bl else G
+        refresh = [(b, n) for (kind, b, n, k) in ev if kind == 1]
+        assert refresh == [(b, n) for b in range(nblk) for n in range(T) if n % K == 0]
+        steps = [(b, n, k) for (kind, b, n, k) in ev if kind == 2]
+        assert [(b, n) for b, n, _ in steps] == [(b, n) for b in range(nblk) for n in range(T)]
+        for b in range(nblk):
+            ks = [k for (bb, n, k) in steps if bb == b]
+            assert ks == [O.unmask_count(n, T, Gb) for n in range(T)] and sum(ks) == Gb
+        assert sum(1 for e in ev if e[0] == 0) == (1 if bl else 0)
+        assert sum(1 for e in ev if e[0] == 3) == (nblk if bl else 0)
+        # every refresh is immediately followed by the step it serves
+        for i, e in enumerate(ev):
+            if e[0] == 1:
+                assert ev[i + 1][0] == 2 and ev[i + 1][1:3] == e[1:3]
+
+
+def test_plan_rejects_bad_arguments(lib):
+    for args in [(8, 60, 16, 4, 32), (8, 64, 0, 4, 0), (8, 64, 16, 0, 0), (8, 0, 16, 1, 0)]:
+        with pytest.raises(lib.TadmError):
+            lib.tadm_plan(*args)
+
+
+def test_layer_cost_matches_paper_tables(lib):
+    g = json.load(open(os.path.join(ROOT, "tests", "golden", "layer_cost.json")))
+    for row in g["table1_ratio"]:
+        full, cache = lib.tadm_layer_cost(row["L_S"], row["L_A"], row["L_D"], row["T"], row["K"])
+        assert round(cache / full, 2) == row["ratio_2dp"]
+    for row in g["table2_calls"]:
+        assert lib.tadm_layer_cost(0, 12, 6, row["T"], row["K"])[1] == row["tadm"]
+    for T in (1, 7, 48, 100):
+        for K in (1, 2, 3, 5, 8):
+            assert lib.tadm_layer_cost(2, 20, 8, T, K) == O.layer_cost(2, 20, 8, T, K)
+
+
+@pytest.mark.parametrize("name", list(wl.WORKLOADS))
+def test_weight_inventory_matches_the_generator(lib, name):
+    m = wl.WORKLOADS[name].model
+    inv = lib.tadm_weight_inventory(lib.make_config(m))
+    specs = wl.weight_specs(m)
+    assert [n for n, _ in inv] == [s.name for s in specs]
+    assert [tuple(s) for _, s in inv] == [s.shape for s in specs]
+
+
+def test_invalid_configs_are_rejected(lib):
+    so = lib.load_library()
+    base = wl.WORKLOADS["small"].model
+    for over in [dict(n_kv_heads=5), dict(vocab=1), dict(head_dim=0), dict(glu="x")]:
+        try:
+            m = wl.ModelConfig(**{**base.__dict__, **over})
+            cfg = lib.make_config(m)
+        except Exception:
+            continue
+        if over.get("glu"):
+            cfg.glu = 7
+        assert so.tadm_weight_count(ctypes.byref(cfg)) == -1
+    h = ctypes.c_void_p()
+    cfg = lib.make_config(base)
+    assert so.tadm_create(ctypes.byref(cfg), None, 0, 1, 1, 0, ctypes.byref(h)) == 1   # no weights
+    assert not h.value

@@ -1,0 +1,138 @@
+"""Kernel-level parity on the GPU, through the C ABI building blocks, against
+the oracle (or its plain definitions) on the same seeded inputs."""
+import numpy as np
+import pytest
+
+import workloads as wl
+from oracle import tadm_oracle as O
+
+pytestmark = pytest.mark.gpu
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def T():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__ as g
+    g.build()
+    from paper_2609_37924_gb300 import tadm
+    return tadm
+
+
+def bf16_tensor(shape, seed, std=1.0):
+    bits = wl.normal(seed, 99, int(np.prod(shape)), 0.0, std, "bf16").reshape(shape)
+    return torch.from_numpy(bits.view(np.int16)).view(torch.bfloat16).cuda(), O.widen(bits)
+
+
+def f32_tensor(shape, seed, std=1.0):
+    x = wl.normal(seed, 98, int(np.prod(shape)), 0.0, std, "f32").reshape(shape)
+    return torch.from_numpy(x).cuda(), x.astype(np.float64)
+
+
+# ------------------------------------------------------------------------------- GEMM
+@pytest.mark.parametrize("M,N,K", [(128, 256, 64), (300, 520, 200), (1024, 768, 768), (77, 2304, 3072),
+                                   (2048, 4096, 2048), (1, 256, 512)])
+def test_gemm_bf16_tcgen05(T, M, N, K):
+    A, a = bf16_tensor((M, K), 1)
+    B, b = bf16_tensor((N, K), 2)
+    C = torch.full((M, N), float("nan"), dtype=torch.float32, device="cuda")
+    T.tadm_gemm(A, B, C, dtype=1)
+    torch.cuda.synchronize()
+    ref = a @ b.T
+    got = C.cpu().numpy().astype(np.float64)
+    # fp32 accumulation of K exact bf16 products: error << 1e-5 of the row scale
+    err = np.abs(got - ref).max() / (np.abs(a).max() * np.abs(b).max() * np.sqrt(K))
+    assert np.isfinite(got).all() and err < 1e-5, err
+    Cb = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+    T.tadm_gemm(A, B, Cb, dtype=1)
+    gb = Cb.float().cpu().numpy().astype(np.float64)
+    assert np.all(np.abs(gb - ref) <= np.abs(ref) * 2.0 ** -8 + 1e-5 * np.sqrt(K))
+
+
+@pytest.mark.parametrize("M,N,K", [(64, 64, 16), (100, 130, 70), (257, 1024, 256)])
+def test_gemm_f32_cuda_cores(T, M, N, K):
+    A, a = f32_tensor((M, K), 3)
+    B, b = f32_tensor((N, K), 4)
+    C = torch.empty((M, N), dtype=torch.float32, device="cuda")
+    T.tadm_gemm(A, B, C, dtype=0)
+    torch.cuda.synchronize()
+    ref = a @ b.T
+    err = np.abs(C.cpu().numpy() - ref).max() / np.sqrt(K)
+    assert err < 1e-5, err
+
+
+# -------------------------------------------------------------------------- attention
+@pytest.mark.parametrize("hd,Hq,Hkv,rows,ctx,causal", [
+    (64, 4, 4, 70, 0, False), (64, 4, 2, 64, 0, True), (128, 4, 2, 32, 37, False), (128, 2, 1, 100, 130, True),
+    (64, 12, 12, 1024, 0, False)])
+def test_attention_bf16(T, hd, Hq, Hkv, rows, ctx, causal):
+    B, stride = 2, ctx + rows + 5
+    q, qd = bf16_tensor((B, Hq, rows, hd), 5)
+    k, kd = bf16_tensor((B, Hkv, stride, hd), 6)
+    v, vd = bf16_tensor((B, Hkv, stride, hd), 7)
+    o = torch.empty((B * rows, Hq * hd), dtype=torch.bfloat16, device="cuda")
+    T.tadm_attention(q, k, v, o, Hq, Hkv, rows, ctx, causal, dtype=1)
+    torch.cuda.synchronize()
+    got = o.float().cpu().numpy().astype(np.float64).reshape(B, rows, Hq, hd)
+    L = ctx + rows
+    for b in range(B):
+        pos = ctx + np.arange(rows)
+        kpos = np.arange(L)
+        # keys < ctx are context: always visible; the causal test covers the rest
+        ref = O.attention(qd[b], kd[b, :, :L], vd[b, :, :L], pos, kpos, causal).transpose(1, 0, 2)
+        rel = np.linalg.norm(got[b] - ref) / np.linalg.norm(ref)
+        assert rel < 1e-2, rel      # P is rounded to bf16 before P V
+
+
+@pytest.mark.parametrize("hd,causal", [(64, False), (64, True), (32, False)])
+def test_attention_f32(T, hd, causal):
+    B, Hq, Hkv, rows, ctx = 1, 4, 2, 45, 9
+    stride = ctx + rows
+    q, qd = f32_tensor((B, Hq, rows, hd), 8)
+    k, kd = f32_tensor((B, Hkv, stride, hd), 9)
+    v, vd = f32_tensor((B, Hkv, stride, hd), 10)
+    o = torch.empty((B * rows, Hq * hd), dtype=torch.float32, device="cuda")
+    T.tadm_attention(q, k, v, o, Hq, Hkv, rows, ctx, causal, dtype=0)
+    torch.cuda.synchronize()
+    ref = O.attention(qd[0], kd[0], vd[0], ctx + np.arange(rows), np.arange(stride), causal).transpose(1, 0, 2)
+    np.testing.assert_allclose(o.cpu().numpy().reshape(rows, Hq, hd), ref, rtol=1e-4, atol=1e-5)
+
+
+# ------------------------------------------------------------------ confidence + top-k
+def test_confidence_bit_exact_argmax(T):
+    rows, V = 333, 32768
+    lg, l64 = f32_tensor((rows, V), 11, std=2.0)
+    host = lg.cpu().numpy()
+    host[5, 100] = host[5, 200] = host[5].max() + 1.0        # tie -> lower id
+    host[7, V - 1] = host[7].max() + 5.0                     # MASK largest -> excluded
+    lg = torch.from_numpy(host).cuda()
+    conf = torch.empty(rows, dtype=torch.float32, device="cuda")
+    tok = torch.empty(rows, dtype=torch.int32, device="cuda")
+    T.tadm_confidence(lg, V - 1, conf, tok)
+    torch.cuda.synchronize()
+    rc, rt = O.confidence(host.astype(np.float64), V - 1)
+    assert np.array_equal(tok.cpu().numpy(), rt)
+    assert tok.cpu().numpy()[5] == 100 and tok.cpu().numpy()[7] != V - 1
+    # fp32 sum of V terms vs the fp64 sum: relative error bound ~ log2(V) * 2^-24 per term, use 4e-6
+    assert np.max(np.abs(conf.cpu().numpy() - rc) / rc) < 4e-6
+
+
+def test_topk_unmask_bit_exact_from_same_keys(T):
+    B, R, mask = 6, 300, 999
+    rng = np.random.default_rng(5)
+    for k in (1, 3, 6, 40, 400):
+        z = np.where(rng.random((B, R)) < 0.7, mask, rng.integers(0, 999, (B, R))).astype(np.int32)
+        conf = rng.choice(np.float32([0.1, 0.25, 0.5, 0.75]), size=(B, R)).astype(np.float32)  # many ties
+        tok = rng.integers(0, 999, (B, R)).astype(np.int32)
+        zt = torch.from_numpy(z).cuda()
+        sel = torch.empty((B, k), dtype=torch.int32, device="cuda")
+        T.tadm_topk_unmask(zt, torch.from_numpy(conf).cuda(), torch.from_numpy(tok).cuda(), k, mask, sel)
+        torch.cuda.synchronize()
+        zg, sg = zt.cpu().numpy(), sel.cpu().numpy()
+        for b in range(B):
+            p = O.select_topk(z[b], conf[b].astype(np.float64), k, mask)
+            zr = z[b].copy()
+            zr[p] = tok[b, p]
+            assert np.array_equal(zg[b], zr)
+            assert list(sg[b, : p.size]) == list(p) and np.all(sg[b, p.size:] == -1)
