@@ -1,0 +1,378 @@
+"""Throughput of TADM's anchor-cache sampling loop on GB300.
+
+One step = one whole generation (Alg. 1 over every block) of the workload's
+batch, i.e. batch * gen_len generated tokens.  Default workload: "small"
+(batch 16, 256 Zipf prompt tokens + 768 masked, 128 reverse steps, K = 4,
+d_model 768, 8 anchor + 4 denoiser layers, vocab 32768, bf16).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload small] [--K 4]
+    python bench.py --impl reference ...      # the CPU oracle on a bounded sample
+
+Under torchrun (N > 1) every rank runs an independent replica on its own
+GPU with its own prompts (sequences are independent: no collective on the
+data path); value = all ranks' tokens / max-over-ranks time.
+Prints one JSON line on rank 0.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "generated tokens/s"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="tadm", choices=["tadm", "reference"])
+    ap.add_argument("--workload", default="small")
+    ap.add_argument("--K", type=int, default=None, help="anchor refresh interval (default: the workload's)")
+    ap.add_argument("--sweep", default="1", help="extra K values timed for the K-sweep (comma list, '' for none)")
+    ap.add_argument("--batch", type=int, default=None)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-sample-seconds", type=float, default=20.0)
+    ap.add_argument("--kernel-bench", default=None,
+                    help="time one building block alone instead, e.g. gemm:16384,32768,768")
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def load_peaks():
+    try:
+        return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except Exception:
+        return None
+
+
+# ----------------------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.path = tempfile.mktemp(prefix="clocks", suffix=".csv")
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(gpu_index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            p = [x.strip() for x in line.split(",")]
+            if len(p) < 9:
+                continue
+            try:
+                sm.append(float(p[1]))
+                mx = float(p[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, p[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        loaded = [x for x in sm if mx and x > 0.5 * mx] or sm
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------- CPU oracle
+def cpu_oracle_sample(workload: str, K: int, budget_s: float, threads: int) -> dict:
+    """Time the CPU oracle (as it stands) on one refresh + K denoising steps of
+    the workload at batch 1 and extrapolate to a whole generation.  Runs in a
+    spawned subprocess so that BLAS threads are set before numpy loads."""
+    code = f"""
+import json, time, sys
+sys.path.insert(0, {ROOT!r})
+import numpy as np
+import workloads as wl
+from oracle import tadm_oracle as O
+w = wl.get_workload({workload!r})
+m = w.model
+host = wl.make_weights(m, seed=w.seed)
+o = O.Oracle(m, host)
+prompts = wl.make_prompts(w, batch=1)
+T, K = w.steps_per_block, {K}
+budget = {budget_s}
+t_start = time.perf_counter()
+sess = o.new_session(1)
+R = w.block_len if w.block_len else w.total_len
+if w.block_len:
+    t0 = time.perf_counter(); o.prefill(sess, prompts); t_prefill = time.perf_counter() - t0
+    z = np.full((1, R), m.vocab - 1, np.int32)
+else:
+    t_prefill = 0.0
+    z = wl.initial_canvas(w, prompts)
+t0 = time.perf_counter(); cache = o.anchor_forward(sess, z); t_anchor = time.perf_counter() - t0
+steps = []
+for n in range(K):
+    t0 = time.perf_counter()
+    r = o.denoise_step(sess, z, cache, n, T, w.block_len or w.gen_len)
+    steps.append(time.perf_counter() - t0)
+    z = r["z"]
+    if time.perf_counter() - t_start > budget and len(steps) >= 1:
+        break
+t_step = sum(steps) / len(steps)
+nb = w.n_blocks
+refresh = nb * (-(-T // K))
+gen_time = refresh * t_anchor + nb * T * t_step + (t_prefill * (1 + nb) if w.block_len else 0.0)
+print(json.dumps(dict(t_anchor=t_anchor, t_step=t_step, steps=len(steps), t_prefill=t_prefill,
+                      gen_time=gen_time, tokens=w.gen_len, wall=time.perf_counter() - t_start)))
+"""
+    env = dict(os.environ, OMP_NUM_THREADS=str(threads), OPENBLAS_NUM_THREADS=str(threads),
+               MKL_NUM_THREADS=str(threads), CUDA_VISIBLE_DEVICES="")
+    r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, timeout=1800)
+    if r.returncode != 0:
+        raise RuntimeError(r.stderr[-2000:])
+    return json.loads(r.stdout.strip().splitlines()[-1])
+
+
+def reference_arm(args):
+    """--impl reference: the CPU oracle timed on the host cores."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    import workloads as wl
+    w = wl.get_workload(args.workload)
+    K = args.K or w.K
+    threads = os.cpu_count() or 1
+    times = []
+    samp = None
+    for i in range(args.warmup + args.steps):
+        samp = cpu_oracle_sample(args.workload, K, args.cpu_sample_seconds, threads)
+        if i >= args.warmup:
+            times.append(samp)
+    tok_per_s = [s["tokens"] / s["gen_time"] for s in times]
+    value = statistics.median(tok_per_s)
+    sample = (f"batch 1 of the '{w.name}' workload: one anchor refresh + {K} denoising steps "
+              f"({'with prompt prefill' if w.block_len else 'full canvas'}), extrapolated to the "
+              f"{w.steps_per_block * w.n_blocks}-step generation of {w.gen_len} tokens")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "higher_is_better": True,
+            "ms_per_step": 1000.0 * statistics.median([s["gen_time"] for s in times]),
+            "dtype": "f64", "data": "synthetic",
+            "config": {"workload": w.name, "batch": 1, "K": K},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": threads, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------- GPU arm
+def gpu_arm(args):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    import workloads as wl
+    from paper_2609_37924_gb300 import TadmModel, upload_weights
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    w = wl.get_workload(args.workload)
+    if args.batch:
+        w = wl.get_workload(args.workload, batch=args.batch)
+    K = args.K or w.K
+    m = w.model
+    B = w.batch
+    host_w = wl.make_weights(m, seed=w.seed)
+    dev_w = upload_weights(m, host_w)
+    del host_w
+    prompts = wl.make_prompts(w, seed=w.seed + 1000 * rank)         # each replica its own prompts
+    bl = w.block_len
+    max_rows = max(w.prompt_len, bl) if bl else w.total_len
+    tm = TadmModel(m, dev_w, max_batch=B, max_rows=max_rows, max_ctx=w.total_len if bl else 0)
+    stream = torch.cuda.current_stream()
+    p_dev = torch.from_numpy(prompts).cuda()
+    out = torch.empty((B, w.total_len), dtype=torch.int32, device="cuda")
+
+    def one(Kv):
+        tm.tadm_generate(p_dev, out, w.gen_len, w.steps_per_block, Kv, bl, stream)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    def timed(Kv, steps, probe=False):
+        for _ in range(args.warmup):
+            one(Kv)
+        tm.tadm_sync_status()
+        if probe:
+            tm.tadm_probe_enable(8192)
+        barrier()
+        launches = 0
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ev0.record(stream)
+        for _ in range(steps):
+            one(Kv)
+            launches += tm.tadm_get_counters()["kernel_launches"]
+        ev1.record(stream)
+        barrier()
+        ms = ev0.elapsed_time(ev1)
+        pr = tm.tadm_probe_read() if probe else None
+        if probe:
+            tm.tadm_probe_enable(0)
+        tm.tadm_sync_status()
+        if world > 1:
+            t = torch.tensor([ms], device="cuda")
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ms = float(t.item())
+        return ms, launches, pr
+
+    clocks = ClockSampler(local)
+    ms, launches, probe = timed(K, args.steps, probe=True)
+    clk = clocks.stop()
+    tokens_per_step = B * w.gen_len
+    value = world * tokens_per_step * args.steps / (ms / 1000.0)
+    sweep = {}
+    for s in [int(x) for x in args.sweep.split(",") if x.strip()]:
+        if s == K:
+            continue
+        ms_s, _, _ = timed(s, args.steps)
+        sweep[str(s)] = world * tokens_per_step * args.steps / (ms_s / 1000.0)
+    sweep[str(K)] = value
+
+    # e2e: public API with host buffers (pinned prompt in, tokens out), copies inside the timed region
+    hp = torch.from_numpy(prompts).pin_memory()
+    for _ in range(args.warmup):
+        tm.generate(hp, w.gen_len, w.steps_per_block, K, bl)
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        res = tm.generate(hp, w.gen_len, w.steps_per_block, K, bl)
+    barrier()
+    e2e_s = time.perf_counter() - t0
+    if world > 1:
+        t = torch.tensor([e2e_s], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    e2e = {"value": world * tokens_per_step * args.steps / e2e_s, "unit": "tokens/s",
+           "h2d_bytes_per_step": int(hp.numel() * 4), "d2h_bytes_per_step": int(res.numel() * 4)}
+
+    peaks = load_peaks()
+    n_launch, gemm_ms, gemm_flops = probe
+    achieved = gemm_flops / (gemm_ms / 1000.0) / 1e12 if gemm_ms > 0 else None
+    if peaks:
+        peak, peak_src = peaks["bf16_tflops_sustained"], "measured sustained bf16 (MEASURED_PEAKS.json)"
+    else:
+        peak, peak_src = 1700.0, "fallback sustained bf16"
+    roofline = {"bound": "tensor", "kernel": "gemm_tc_kernel (tcgen05, all GEMM launches)",
+                "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": (achieved / peak) if achieved else None, "traffic": None, "peak_source": peak_src,
+                "launches_timed": n_launch, "gemm_ms_per_step": gemm_ms / args.steps,
+                "gemm_share_of_step": gemm_ms / ms if ms else None}
+
+    line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if m.dtype == "bf16" else "f32",
+            "data": "synthetic (seeded random-init weights N(0,0.02), Zipf-1.1 prompt ids)",
+            "config": {"workload": w.name, "batch": B, "prompt_len": w.prompt_len, "gen_len": w.gen_len,
+                       "steps_per_block": w.steps_per_block, "block_len": bl, "K": K, "d_model": m.d_model,
+                       "layers_anchor": m.n_anchor, "layers_denoise": m.n_denoise, "vocab": m.vocab,
+                       "parallelism": f"replicas x{world}",
+                       "l2": "inputs larger than L2 (weights + activations per step >> 129 MB)"},
+            "k_sweep_tokens_per_s": sweep, "roofline": roofline, "clocks": clk,
+            "e2e": e2e, "gpu_launches": launches}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        try:
+            threads = os.cpu_count() or 1
+            s = cpu_oracle_sample(args.workload, K, args.cpu_sample_seconds, threads)
+            line["cpu_baseline"] = {
+                "value": s["tokens"] / s["gen_time"], "unit": "tokens/s", "cores": threads, "kind": "oracle",
+                "sample": (f"batch 1: one anchor refresh ({s['t_anchor']:.2f} s) + {s['steps']} denoising steps "
+                           f"({s['t_step']:.2f} s each) of the '{w.name}' workload, extrapolated to the "
+                           f"{w.steps_per_block * w.n_blocks}-step generation of {w.gen_len} tokens")}
+        except Exception as e:  # the baseline is context; the GPU line still prints
+            line["cpu_baseline"] = {"error": str(e)[-300:]}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def kernel_bench(args):
+    """Times one building block alone through the C ABI (for isolated ncu
+    captures of the GEMM): C[M, N] = A[M, K] B[N, K]^T, bf16 in, bf16 out."""
+    import torch
+    from paper_2609_37924_gb300 import tadm
+    kind, shape = args.kernel_bench.split(":")
+    g = torch.Generator(device="cuda").manual_seed(0)
+    if kind == "attn":
+        # attn:B,H,Hkv,R,hd  bidirectional attention of R rows (no context), bf16
+        B, H, Hkv, R, hd = (int(x) for x in shape.split(","))
+        q = torch.randn((B, H, R, hd), device="cuda", generator=g).to(torch.bfloat16)
+        k = torch.randn((B, Hkv, R, hd), device="cuda", generator=g).to(torch.bfloat16)
+        v = torch.randn((B, Hkv, R, hd), device="cuda", generator=g).to(torch.bfloat16)
+        o = torch.empty((B * R, H * hd), device="cuda", dtype=torch.bfloat16)
+        run = lambda: tadm.tadm_attention(q, k, v, o, H, Hkv, R, 0, False, dtype=1)  # noqa: E731
+        flops = 4.0 * B * H * R * R * hd
+    else:
+        M, N, K = (int(x) for x in shape.split(","))
+        A = torch.randn((M, K), device="cuda", generator=g).to(torch.bfloat16)
+        Bm = torch.randn((N, K), device="cuda", generator=g).to(torch.bfloat16)
+        C = torch.empty((M, N), device="cuda", dtype=torch.bfloat16)
+        run = lambda: tadm.tadm_gemm(A, Bm, C, dtype=1)  # noqa: E731
+        flops = 2.0 * M * N * K
+    for _ in range(args.warmup):
+        run()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.steps):
+        run()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / args.steps
+    print(json.dumps({"kernel": kind, "shape": shape, "ms": ms, "tflops": flops / (ms / 1000.0) / 1e12}), flush=True)
+
+
+def main():
+    args = parse()
+    if args.kernel_bench:
+        import __graft_entry__
+        __graft_entry__.build()
+        kernel_bench(args)
+        return
+    if args.impl == "reference":
+        reference_arm(args)
+    else:
+        import __graft_entry__
+        __graft_entry__.build()
+        gpu_arm(args)
+
+
+if __name__ == "__main__":
+    main()

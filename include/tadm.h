@@ -206,8 +206,18 @@ typedef struct {
   int64_t shared_layers, anchor_layers, denoise_layers;
   int64_t anchor_calls, denoise_steps;
   int64_t commit_passes;
+  int64_t kernel_launches; /* CUDA kernels this handle launched */
 } tadm_counters;
 TADM_API tadm_status tadm_get_counters(const tadm_handle* h, tadm_counters* out);
+
+/* GEMM timing probe.  While enabled, every GEMM launch of the handle is
+ * bracketed by two CUDA events recorded on its stream (a pool of up to
+ * `max_launches` pairs, created here), and its algorithmic work 2*M*N*K is
+ * noted.  tadm_probe_read waits for the last event and returns the number
+ * of bracketed launches, their summed duration (ms) and summed FLOPs, then
+ * clears the records.  tadm_probe_enable(h, 0) frees the events. */
+TADM_API tadm_status tadm_probe_enable(tadm_handle* h, int max_launches);
+TADM_API tadm_status tadm_probe_read(tadm_handle* h, int64_t* launches, double* total_ms, double* total_flops);
 
 /* Plan of tadm_generate (host only, no GPU): the ordered phases it issues.
  * kind: 0 prefill, 1 anchor refresh, 2 denoise step, 3 commit.  For kinds 1

@@ -122,6 +122,11 @@ struct tadm_handle {
   size_t kv_slab = 0;
   int kv_stride = 0, n_part_tiles = 0;
 
+  // GEMM timing probe
+  std::vector<cudaEvent_t> probe_ev;
+  std::vector<double> probe_flops;
+  int probe_next = 0;
+
   // sequence state
   int batch = 0, ctx = 0;
   tadm_counters counters{};
@@ -153,6 +158,7 @@ tadm_status fail(tadm_handle* h, tadm_status s, const char* fmt, ...) {
   do {                                                              \
     const char* _e = (expr);                                        \
     if (_e) return fail(h, TADM_ERR_CUDA, "%s: %s", #expr, _e);     \
+    h->counters.kernel_launches += 1;                               \
   } while (0)
 
 #define TRYS(expr)                         \
@@ -265,8 +271,16 @@ tadm_status gemm(tadm_handle* h, const void* A, int64_t a_rows, int lda, const v
   g.status = h->status();
   g.ep.out_bf16 = out_f32 ? 0 : h->act_bf16();
   g.ep.bias_bf16 = h->cfg.dtype;
+  const bool probe = h->probe_next < static_cast<int>(h->probe_flops.size());
+  if (probe) cudaEventRecord(h->probe_ev[2 * h->probe_next], s);
   const char* e = h->cfg.dtype ? gemm_tc(g, s) : gemm_simt(g, s);
   if (e) return fail(h, TADM_ERR_CUDA, "GEMM (M=%d N=%d K=%d epi=%d): %s", M, N, K, epi, e);
+  h->counters.kernel_launches += 1;
+  if (probe) {
+    cudaEventRecord(h->probe_ev[2 * h->probe_next + 1], s);
+    const double n_acc = epi == EPI_GLU ? 2.0 * N : static_cast<double>(N);
+    h->probe_flops[h->probe_next++] = 2.0 * M * n_acc * K;
+  }
   return TADM_OK;
 }
 
@@ -670,7 +684,43 @@ tadm_status tadm_create(const tadm_config* cfg, const void* const* weights, int 
   return TADM_OK;
 }
 
-void tadm_destroy(tadm_handle* h) { delete h; }
+void tadm_destroy(tadm_handle* h) {
+  if (h) tadm_probe_enable(h, 0);
+  delete h;
+}
+
+tadm_status tadm_probe_enable(tadm_handle* h, int max_launches) {
+  if (!h || max_launches < 0) return TADM_ERR_INVALID_ARG;
+  for (cudaEvent_t e : h->probe_ev) cudaEventDestroy(e);
+  h->probe_ev.clear();
+  h->probe_flops.clear();
+  h->probe_next = 0;
+  if (max_launches == 0) return TADM_OK;
+  h->probe_ev.resize(2 * static_cast<size_t>(max_launches));
+  for (auto& e : h->probe_ev)
+    if (cudaEventCreate(&e) != cudaSuccess) return fail(h, TADM_ERR_CUDA, "cudaEventCreate failed");
+  h->probe_flops.assign(max_launches, 0.0);
+  return TADM_OK;
+}
+
+tadm_status tadm_probe_read(tadm_handle* h, int64_t* launches, double* total_ms, double* total_flops) {
+  if (!h) return TADM_ERR_INVALID_ARG;
+  double ms = 0.0, fl = 0.0;
+  if (h->probe_next > 0 && cudaEventSynchronize(h->probe_ev[2 * h->probe_next - 1]) != cudaSuccess)
+    return fail(h, TADM_ERR_CUDA, "probe event sync failed");
+  for (int i = 0; i < h->probe_next; ++i) {
+    float t = 0.0f;
+    if (cudaEventElapsedTime(&t, h->probe_ev[2 * i], h->probe_ev[2 * i + 1]) != cudaSuccess)
+      return fail(h, TADM_ERR_CUDA, "probe elapsed time failed");
+    ms += t;
+    fl += h->probe_flops[i];
+  }
+  if (launches) *launches = h->probe_next;
+  if (total_ms) *total_ms = ms;
+  if (total_flops) *total_flops = fl;
+  h->probe_next = 0;
+  return TADM_OK;
+}
 
 const char* tadm_last_error(const tadm_handle* h) { return h ? h->err.c_str() : "NULL handle"; }
 

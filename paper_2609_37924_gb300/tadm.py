@@ -22,7 +22,7 @@ ABI_FUNCTIONS = [
     "tadm_status_string", "tadm_workspace_size", "tadm_bind_workspace", "tadm_cache_size", "tadm_reset",
     "tadm_prefill", "tadm_anchor_forward", "tadm_denoise_step", "tadm_commit_block", "tadm_generate",
     "tadm_sync_status", "tadm_get_counters", "tadm_plan", "tadm_layer_cost", "tadm_gemm", "tadm_confidence",
-    "tadm_topk_unmask", "tadm_attention",
+    "tadm_topk_unmask", "tadm_attention", "tadm_probe_enable", "tadm_probe_read",
 ]
 
 
@@ -46,7 +46,8 @@ class tadm_step_outputs(ctypes.Structure):
 
 class tadm_counters(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int64) for n in (
-        "shared_layers", "anchor_layers", "denoise_layers", "anchor_calls", "denoise_steps", "commit_passes")]
+        "shared_layers", "anchor_layers", "denoise_layers", "anchor_calls", "denoise_steps", "commit_passes",
+        "kernel_launches")]
 
 
 class tadm_plan_event(ctypes.Structure):
@@ -90,6 +91,9 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "tadm_confidence": (I, [P, I, I, I, P, P, P]),
         "tadm_topk_unmask": (I, [P, I, P, P, I, I, I, I, P, P]),
         "tadm_attention": (I, [P, P, P, P, I, I, I, I, I, I, I, I, I, P]),
+        "tadm_probe_enable": (I, [P, I]),
+        "tadm_probe_read": (I, [P, ctypes.POINTER(I64), ctypes.POINTER(ctypes.c_double),
+                                ctypes.POINTER(ctypes.c_double)]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -267,6 +271,14 @@ class TadmModel:
 
     def tadm_sync_status(self):
         _check(self.lib.tadm_sync_status(self.h), self.h)
+
+    def tadm_probe_enable(self, max_launches: int):
+        _check(self.lib.tadm_probe_enable(self.h, max_launches), self.h)
+
+    def tadm_probe_read(self):
+        n, ms, fl = ctypes.c_int64(), ctypes.c_double(), ctypes.c_double()
+        _check(self.lib.tadm_probe_read(self.h, ctypes.byref(n), ctypes.byref(ms), ctypes.byref(fl)), self.h)
+        return n.value, ms.value, fl.value
 
     def tadm_get_counters(self) -> dict:
         c = tadm_counters()

@@ -55,7 +55,22 @@ def gpu_step(tm, z, t, Tn, G, cache, want_fused=False):
     return out
 
 
-def check_step(o, sess, z, cache_o, g, n, Tn, G, tol, min_agree):
+class Agreement:
+    """Teacher-forced agreement over a test: every token the GPU commits is
+    compared with the oracle's prediction at that position on the same
+    canvas; all-position argmax agreement is recorded too."""
+
+    def __init__(self):
+        self.committed = self.committed_ok = self.masked = self.masked_ok = 0
+
+    def check(self, min_committed=0.995):
+        assert self.committed > 0
+        rate = self.committed_ok / self.committed
+        assert rate >= min_committed, (self.committed_ok, self.committed)
+        return rate
+
+
+def check_step(o, sess, z, cache_o, g, n, Tn, G, tol, min_agree, agg=None):
     ref = o.denoise_step(sess, z, cache_o, n, Tn, G)
     assert rel_l2(g["logits"], ref["logits"]) < tol
     # confidence / argmax from the GPU's own logits are bit-exact in the sampler
@@ -63,14 +78,31 @@ def check_step(o, sess, z, cache_o, g, n, Tn, G, tol, min_agree):
     assert np.array_equal(g["tok"].reshape(-1), t2)
     assert np.max(np.abs(g["conf"].reshape(-1) - c2) / c2) < 4e-6
     # selection from the GPU's conf keys is exact
+    k = O.unmask_count(n, Tn, G)
     for b in range(z.shape[0]):
-        p = O.select_topk(z[b], g["conf"][b].astype(np.float64), O.unmask_count(n, Tn, G), o.mask_id)
+        p = O.select_topk(z[b], g["conf"][b].astype(np.float64), k, o.mask_id)
         assert list(g["sel"][b]) == list(p)
     masked = z == o.mask_id
     agree = float(np.mean(g["tok"][masked] == ref["tok"][masked]))
     assert agree >= min_agree, agree
-    # committed tokens: same positions and tokens as the oracle
-    assert np.array_equal(g["z"], ref["z"])
+    # the positions the GPU chose are a valid top-k of the oracle's confidences,
+    # up to twice the observed GPU-vs-oracle confidence error (near-ties may
+    # be ordered either way)
+    for b in range(z.shape[0]):
+        cand = np.nonzero(masked[b])[0]
+        if cand.size == 0 or k == 0:
+            continue
+        oc = ref["conf"][b]
+        delta = float(np.max(np.abs(g["conf"][b][cand] / oc[cand] - 1.0)))
+        kth = np.sort(oc[cand])[::-1][min(k, cand.size) - 1]
+        for p in g["sel"][b]:
+            assert oc[p] >= kth * (1.0 - 2.0 * delta) - 1e-30, (p, oc[p], kth, delta)
+    committed = masked & (g["z"] != o.mask_id)
+    if agg is not None:
+        agg.committed += int(committed.sum())
+        agg.committed_ok += int((g["z"][committed] == ref["tok"][committed]).sum())
+        agg.masked += int(masked.sum())
+        agg.masked_ok += int((g["tok"][masked] == ref["tok"][masked]).sum())
     return ref
 
 
@@ -92,7 +124,9 @@ def test_tiny_fp32_teacher_forced_step(T):
     g = gpu_step(tm, z, 30, 32, 96, cache, want_fused=True)
     ht = np.stack([o.fuse(o.S(z[b], np.arange(R), None), cache_o[b]) for b in range(B)])
     assert rel_l2(g["fused"], ht) < 1e-5
-    check_step(o, sess, z, cache_o, g, 2, 32, 96, tol=1e-4, min_agree=0.99)
+    agg = Agreement()
+    check_step(o, sess, z, cache_o, g, 2, 32, 96, tol=1e-4, min_agree=0.99, agg=agg)
+    agg.check(1.0)
 
 
 @pytest.mark.parametrize("glu", ["swiglu", "geglu"])
@@ -111,7 +145,9 @@ def test_bf16_teacher_forced_step_stale_cache(T, glu):
     g = gpu_step(tm, z1, 14, 16, 160, cache, want_fused=True)
     ht = np.stack([o.fuse(o.S(z1[b], np.arange(R), None), cache_o[b]) for b in range(B)])
     assert rel_l2(g["fused"], ht) < 1e-2
-    check_step(o, sess, z1, cache_o, g, 2, 16, 160, tol=2e-2, min_agree=0.95)
+    agg = Agreement()
+    check_step(o, sess, z1, cache_o, g, 2, 16, 160, tol=2e-2, min_agree=0.95, agg=agg)
+    agg.check()
 
 
 def test_generate_k1_equals_step_loop_and_counts(T):
@@ -185,6 +221,7 @@ def test_block_mode_with_kv_context(T):
     sess = o.new_session(B)
     o.prefill(sess, prompts)
     cache = tm.new_cache(B, bl)
+    agg = Agreement()
     for blk in range(2):
         zb = np.full((B, bl), m.mask_id, np.int32)
         for n in range(4):
@@ -192,11 +229,12 @@ def test_block_mode_with_kv_context(T):
                 tm.tadm_anchor_forward(torch.from_numpy(zb).cuda(), 4 - n, cache)
                 cache_o = o.anchor_forward(sess, zb)
             g = gpu_step(tm, zb, 4 - n, 4, bl, cache)
-            check_step(o, sess, zb, cache_o, g, n, 4, bl, tol=2e-2, min_agree=0.9)
+            check_step(o, sess, zb, cache_o, g, n, 4, bl, tol=2e-2, min_agree=0.9, agg=agg)
             zb = g["z"]
         tm.tadm_commit_block(torch.from_numpy(zb).cuda())
         o.commit_block(sess, zb)
     tm.tadm_sync_status()
+    agg.check()
     # and tadm_generate follows the same plan
     out = tm.generate(torch.from_numpy(prompts).cuda(), 64, 4, 2, block_len=bl).cpu().numpy()
     assert out.shape == (B, P + 64) and np.all(out != m.mask_id) and np.array_equal(out[:, :P], prompts)
@@ -223,7 +261,9 @@ def test_paired_attention_fusion_identity_and_parity(T):
     g1 = gpu_step(tm, z1, 7, 8, R, cache, want_fused=True)
     ht = np.stack([o.fuse(o.S(z1[b], np.arange(R), None), cache_o[b]) for b in range(B)])
     assert rel_l2(g1["fused"], ht) < 1e-2
-    check_step(o, sess, z1, cache_o, g1, 1, 8, R, tol=2e-2, min_agree=0.9)
+    agg = Agreement()
+    check_step(o, sess, z1, cache_o, g1, 1, 8, R, tol=2e-2, min_agree=0.9, agg=agg)
+    agg.check()
 
 
 def test_invalid_calls_return_errors(T):
