@@ -256,6 +256,20 @@ TADM_API tadm_status tadm_confidence(const float* logits, int rows, int vocab, i
 TADM_API tadm_status tadm_topk_unmask(int32_t* z, int ldz, const float* conf, const int32_t* tok, int batch,
                              int rows, int k, int mask_id, int32_t* selected, tadm_stream stream);
 
+/* Fused output head + confidence (the sampler's input, paper App. B.1.1
+ * zero-masking): for each row of x [rows, d], logits = x W^T over W
+ * [vocab, d] are reduced inside the GEMM epilogue to per-column-tile
+ * (max, sum exp, argmax) partials, which a second kernel merges into
+ * tok = argmax over ids != mask_id (lowest id on ties) and
+ * conf = 1 / sum_v exp(l_v - l_tok).  The logits never reach memory.
+ * dtype 1: x, W bf16 (tcgen05); 0: fp32.  scratch: device, at least
+ * tadm_head_scratch_size() bytes, holds the partials; it needs no
+ * initialisation and its contents are meaningless after the call. */
+TADM_API tadm_status tadm_head_scratch_size(int rows, int vocab, int dtype, size_t* bytes);
+TADM_API tadm_status tadm_head_confidence(const void* x, const void* w, int rows, int d, int vocab, int mask_id,
+                                          int dtype, void* scratch, size_t scratch_bytes, float* conf,
+                                          int32_t* tok, tadm_stream stream);
+
 /* softmax(Q K^T / sqrt(hd)) V for queries at positions ctx .. ctx+rows-1 over
  * keys 0 .. ctx+rows-1 (keys < ctx always visible; the rest bidirectional,
  * or causal if `causal`).  dtype 1: bf16, 0: fp32.

@@ -912,6 +912,38 @@ tadm_status tadm_topk_unmask(int32_t* z, int ldz, const float* conf, const int32
   return topk_unmask(z, ldz, conf, tok, batch, rows, k, mask_id, selected, stream) ? TADM_ERR_CUDA : TADM_OK;
 }
 
+tadm_status tadm_head_scratch_size(int rows, int vocab, int dtype, size_t* bytes) {
+  if (!bytes || rows < 0 || vocab < 2 || (dtype != 0 && dtype != 1)) return TADM_ERR_INVALID_ARG;
+  const int tiles = dtype ? gemm_tc_tiles_n(vocab, EPI_LMHEAD) : gemm_simt_tiles_n(vocab, EPI_LMHEAD);
+  *bytes = static_cast<size_t>(rows) * tiles * 3 * sizeof(float);
+  return TADM_OK;
+}
+
+tadm_status tadm_head_confidence(const void* x, const void* w, int rows, int d, int vocab, int mask_id, int dtype,
+                                 void* scratch, size_t scratch_bytes, float* conf, int32_t* tok, tadm_stream stream) {
+  size_t need = 0;
+  if (tadm_head_scratch_size(rows, vocab, dtype, &need) != TADM_OK) return TADM_ERR_INVALID_ARG;
+  if (!x || !w || !conf || !tok || d <= 0 || mask_id < 0 || mask_id >= vocab) return TADM_ERR_INVALID_ARG;
+  if (rows == 0) return TADM_OK;
+  if (!scratch || scratch_bytes < need) return TADM_ERR_INVALID_ARG;
+  GemmCall g{};
+  g.A = x;
+  g.B = w;
+  g.M = rows;
+  g.N = vocab;
+  g.K = d;
+  g.lda = d;
+  g.ldb = d;
+  g.epi = EPI_LMHEAD;
+  g.ep.part = static_cast<float*>(scratch);
+  g.ep.mask_id = mask_id;
+  const char* e = dtype ? gemm_tc(g, stream) : gemm_simt(g, stream);
+  if (e) return TADM_ERR_CUDA;
+  const int tiles = dtype ? gemm_tc_tiles_n(vocab, EPI_LMHEAD) : gemm_simt_tiles_n(vocab, EPI_LMHEAD);
+  return combine_partials(static_cast<const float*>(scratch), rows, tiles, conf, tok, stream) ? TADM_ERR_CUDA
+                                                                                               : TADM_OK;
+}
+
 tadm_status tadm_attention(const void* q, const void* k, const void* v, void* o, int batch, int n_heads, int n_kv_heads,
                            int head_dim, int rows, int ctx, int kv_stride, int causal, int dtype, tadm_stream stream) {
   if (!q || !k || !v || !o || batch < 0 || n_heads <= 0 || n_kv_heads <= 0 || rows < 0 || ctx < 0)

@@ -22,7 +22,8 @@ ABI_FUNCTIONS = [
     "tadm_status_string", "tadm_workspace_size", "tadm_bind_workspace", "tadm_cache_size", "tadm_reset",
     "tadm_prefill", "tadm_anchor_forward", "tadm_denoise_step", "tadm_commit_block", "tadm_generate",
     "tadm_sync_status", "tadm_get_counters", "tadm_plan", "tadm_layer_cost", "tadm_gemm", "tadm_confidence",
-    "tadm_topk_unmask", "tadm_attention", "tadm_probe_enable", "tadm_probe_read",
+    "tadm_topk_unmask", "tadm_attention", "tadm_probe_enable", "tadm_probe_read", "tadm_head_scratch_size",
+    "tadm_head_confidence",
 ]
 
 
@@ -91,6 +92,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "tadm_confidence": (I, [P, I, I, I, P, P, P]),
         "tadm_topk_unmask": (I, [P, I, P, P, I, I, I, I, P, P]),
         "tadm_attention": (I, [P, P, P, P, I, I, I, I, I, I, I, I, I, P]),
+        "tadm_head_scratch_size": (I, [I, I, I, ctypes.POINTER(SZ)]),
+        "tadm_head_confidence": (I, [P, P, I, I, I, I, I, P, SZ, P, P, P]),
         "tadm_probe_enable": (I, [P, I]),
         "tadm_probe_read": (I, [P, ctypes.POINTER(I64), ctypes.POINTER(ctypes.c_double),
                                 ctypes.POINTER(ctypes.c_double)]),
@@ -176,6 +179,20 @@ def tadm_topk_unmask(z, conf, tok, k: int, mask_id: int, selected=None, stream=N
     batch, rows = conf.shape
     _check(load_library().tadm_topk_unmask(_ptr(z), z.stride(0), _ptr(conf), _ptr(tok), batch, rows, k, mask_id,
                                            _ptr(selected), _stream(stream)))
+
+
+def tadm_head_scratch_size(rows: int, vocab: int, dtype: int) -> int:
+    n = ctypes.c_size_t()
+    _check(load_library().tadm_head_scratch_size(rows, vocab, dtype, ctypes.byref(n)))
+    return n.value
+
+
+def tadm_head_confidence(x, w, mask_id: int, conf, tok, scratch, dtype: int, stream=None):
+    rows, d = x.shape
+    vocab = w.shape[0]
+    _check(load_library().tadm_head_confidence(_ptr(x), _ptr(w), rows, d, vocab, mask_id, dtype, _ptr(scratch),
+                                               scratch.numel() * scratch.element_size(), _ptr(conf), _ptr(tok),
+                                               _stream(stream)))
 
 
 def tadm_attention(q, k, v, o, n_heads: int, n_kv_heads: int, rows: int, ctx: int, causal: bool, dtype: int,

@@ -136,3 +136,22 @@ def test_topk_unmask_bit_exact_from_same_keys(T):
             zr[p] = tok[b, p]
             assert np.array_equal(zg[b], zr)
             assert list(sg[b, : p.size]) == list(p) and np.all(sg[b, p.size:] == -1)
+
+
+@pytest.mark.parametrize("rows,d,V,dtype", [(300, 768, 32768, 1), (129, 256, 5000, 1), (70, 256, 1024, 0)])
+def test_head_confidence_fused(T, rows, d, V, dtype):
+    mk = bf16_tensor if dtype else f32_tensor
+    x, xd = mk((rows, d), 12)
+    w, wd = mk((V, d), 13, std=0.05)
+    conf = torch.empty(rows, dtype=torch.float32, device="cuda")
+    tok = torch.empty(rows, dtype=torch.int32, device="cuda")
+    scratch = torch.empty(T.tadm_head_scratch_size(rows, V, dtype), dtype=torch.uint8, device="cuda")
+    T.tadm_head_confidence(x, w, V - 1, conf, tok, scratch, dtype)
+    logits = torch.empty((rows, V), dtype=torch.float32, device="cuda")
+    T.tadm_gemm(x, w, logits, dtype=dtype)          # same accumulation, materialised
+    torch.cuda.synchronize()
+    rc, rt = O.confidence(logits.cpu().numpy().astype(np.float64), V - 1)
+    assert np.array_equal(tok.cpu().numpy(), rt)
+    assert np.max(np.abs(conf.cpu().numpy() - rc) / rc) < 4e-6
+    lf = xd @ wd.T                                   # fp64 from the same inputs
+    assert np.linalg.norm(logits.cpu().numpy() - lf) / np.linalg.norm(lf) < 1e-5
