@@ -270,6 +270,31 @@ TADM_API tadm_status tadm_head_confidence(const void* x, const void* w, int rows
                                           int dtype, void* scratch, size_t scratch_bytes, float* conf,
                                           int32_t* tok, tadm_stream stream);
 
+/* tadm_head_confidence without caller scratch, for callers that cannot
+ * allocate device memory: for example code inside a host framework that
+ * owns every device allocation and passes in only input and output
+ * buffers, or latency-critical paths that forbid cudaMalloc because it can
+ * synchronise the device.  The paper has no counterpart; this is a library
+ * convenience.  Arguments and results are those of tadm_head_confidence.
+ *  - The partials live in a fixed device array of
+ *    TADM_HEAD_STATIC_SCRATCH_BYTES (8 MiB) inside the library, which every
+ *    GPU that loads the library holds until the process exits.  Calls that
+ *    need more (rows * ceil(vocab / 256) * 12 bytes for dtype 1,
+ *    rows * ceil(vocab / 64) * 12 bytes for dtype 0) return
+ *    TADM_ERR_INVALID_ARG and do nothing.
+ *  - The first call on each device looks up the array's device address
+ *    (cudaGetSymbolAddress, with that device current); make that first call
+ *    before any stream capture.  Later calls on the device only launch.
+ *  - No allocation of any kind: no cudaMalloc / cudaFree, no allocating
+ *    library routine.
+ *  - Every call shares the one array and leaves its partials there; nothing
+ *    in it needs to start at zero.  Calls whose work overlaps on the GPU
+ *    (other streams, other host threads) race on the array: serialise them. */
+#define TADM_HEAD_STATIC_SCRATCH_BYTES (8u << 20)
+TADM_API tadm_status tadm_head_confidence_static(const void* x, const void* w, int rows, int d, int vocab,
+                                                 int mask_id, int dtype, float* conf, int32_t* tok,
+                                                 tadm_stream stream);
+
 /* softmax(Q K^T / sqrt(hd)) V for queries at positions ctx .. ctx+rows-1 over
  * keys 0 .. ctx+rows-1 (keys < ctx always visible; the rest bidirectional,
  * or causal if `causal`).  dtype 1: bf16, 0: fp32.

@@ -23,7 +23,7 @@ ABI_FUNCTIONS = [
     "tadm_prefill", "tadm_anchor_forward", "tadm_denoise_step", "tadm_commit_block", "tadm_generate",
     "tadm_sync_status", "tadm_get_counters", "tadm_plan", "tadm_layer_cost", "tadm_gemm", "tadm_confidence",
     "tadm_topk_unmask", "tadm_attention", "tadm_probe_enable", "tadm_probe_read", "tadm_head_scratch_size",
-    "tadm_head_confidence",
+    "tadm_head_confidence", "tadm_head_confidence_static",
 ]
 
 
@@ -94,6 +94,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "tadm_attention": (I, [P, P, P, P, I, I, I, I, I, I, I, I, I, P]),
         "tadm_head_scratch_size": (I, [I, I, I, ctypes.POINTER(SZ)]),
         "tadm_head_confidence": (I, [P, P, I, I, I, I, I, P, SZ, P, P, P]),
+        "tadm_head_confidence_static": (I, [P, P, I, I, I, I, I, P, P, P]),
         "tadm_probe_enable": (I, [P, I]),
         "tadm_probe_read": (I, [P, ctypes.POINTER(I64), ctypes.POINTER(ctypes.c_double),
                                 ctypes.POINTER(ctypes.c_double)]),
@@ -193,6 +194,15 @@ def tadm_head_confidence(x, w, mask_id: int, conf, tok, scratch, dtype: int, str
     _check(load_library().tadm_head_confidence(_ptr(x), _ptr(w), rows, d, vocab, mask_id, dtype, _ptr(scratch),
                                                scratch.numel() * scratch.element_size(), _ptr(conf), _ptr(tok),
                                                _stream(stream)))
+
+
+def tadm_head_confidence_static(x, w, mask_id: int, conf, tok, dtype: int, stream=None):
+    """The same result as tadm_head_confidence, with the partials in the
+    library's fixed device array instead of caller scratch (no allocation)."""
+    rows, d = x.shape
+    vocab = w.shape[0]
+    _check(load_library().tadm_head_confidence_static(_ptr(x), _ptr(w), rows, d, vocab, mask_id, dtype, _ptr(conf),
+                                                      _ptr(tok), _stream(stream)))
 
 
 def tadm_attention(q, k, v, o, n_heads: int, n_kv_heads: int, rows: int, ctx: int, causal: bool, dtype: int,
