@@ -279,8 +279,7 @@ TADM_API tadm_status tadm_head_confidence(const void* x, const void* w, int rows
  *  - The partials live in a fixed device array of
  *    TADM_HEAD_STATIC_SCRATCH_BYTES (8 MiB) inside the library, which every
  *    GPU that loads the library holds until the process exits.  Calls that
- *    need more (rows * ceil(vocab / 256) * 12 bytes for dtype 1,
- *    rows * ceil(vocab / 64) * 12 bytes for dtype 0) return
+ *    need more than that (tadm_head_scratch_size) return
  *    TADM_ERR_INVALID_ARG and do nothing.
  *  - The first call on each device looks up the array's device address
  *    (cudaGetSymbolAddress, with that device current); make that first call
@@ -298,8 +297,9 @@ TADM_API tadm_status tadm_head_confidence_static(const void* x, const void* w, i
 /* softmax(Q K^T / sqrt(hd)) V for queries at positions ctx .. ctx+rows-1 over
  * keys 0 .. ctx+rows-1 (keys < ctx always visible; the rest bidirectional,
  * or causal if `causal`).  dtype 1: bf16, 0: fp32.
- * q: [batch, n_heads, rows, hd]; k, v: [batch, n_kv_heads, kv_stride, hd];
- * o: [batch*rows, n_heads*hd]. */
+ * q: [batch, n_heads, rows, hd]; k: [batch, n_kv_heads, kv_stride, hd];
+ * v transposed: [batch, n_kv_heads, hd, kv_stride]; o: [batch*rows, n_heads*hd].
+ * K and V entries at positions >= ctx + rows must hold finite values. */
 TADM_API tadm_status tadm_attention(const void* q, const void* k, const void* v, void* o, int batch,
                            int n_heads, int n_kv_heads, int head_dim, int rows, int ctx,
                            int kv_stride, int causal, int dtype, tadm_stream stream);

@@ -2,19 +2,348 @@
 //   o = softmax(q k^T / sqrt(hd)) v
 // Queries are the rows of the current canvas at absolute positions
 // ctx .. ctx+rows-1; keys are positions 0 .. ctx+rows-1 of the layer's K/V
-// buffer.  Keys below ctx (committed context) are always visible; the active
+// buffers.  Keys below ctx (committed context) are always visible; the active
 // rows see each other bidirectionally, or causally for commit / prefill
 // passes.  Query head h reads KV head h / (n_heads / n_kv_heads).
+// Layouts: q [B, Hq, rows, hd]; k [B, Hkv, kv_stride, hd];
+// v transposed [B, Hkv, hd, kv_stride]; o [B*rows, Hq*hd].
 //
-// bf16: flash-attention style, one CTA = 64 query rows of one (batch, head),
-// 4 warps x 16 rows, key tiles of 64 double-buffered with cp.async,
-// QK^T and PV on mma.sync m16n8k16 (fp32 accumulate), online softmax in fp32.
+// bf16, rows >= 128 (attn_tc_kernel): tcgen05.  One CTA = 128 query rows of
+//   one (batch, head).  Warp 0 streams Q once and K / V^T tiles of 128 keys
+//   (2-stage ring) with TMA; warp 1 issues S = Q K^T into TMEM and, once the
+//   probabilities are in shared memory, O_tile = P V into TMEM; warps 2..5
+//   own one query row per thread: masked online softmax on the S row, P as
+//   bf16 into the 128-byte-swizzled operand layout, and O accumulated in
+//   registers with the running-max correction.
+// bf16, short rows (attn_bf16_kernel): mma.sync m16n8k16 flash attention.
 // fp32: one warp per query row on the CUDA cores.
+#include <cudaTypedefs.h>
+#include <mutex>
+
 #include "kernels.h"
 
 namespace tadm {
 namespace {
 
+// =============================================================== tcgen05 path
+constexpr int TQ = 128;      // query rows per CTA
+constexpr int TKV = 128;     // keys per tile
+
+template <int HD>
+struct AttnTcCfg {
+  static constexpr int Q_BYTES = HD / 64 * 16384;       // HD/64 swizzle atoms of 128 x 64
+  static constexpr int K_BYTES = HD / 64 * 16384;
+  static constexpr int V_BYTES = 2 * HD * 128;           // two 64-key atoms of HD rows
+  static constexpr int P_BYTES = 2 * 16384;              // two 64-key atoms of 128 rows
+  static constexpr int STAGES = 2;
+  // hd 64 runs two CTAs per SM, which leaves no room for re-alignment slack:
+  // the kernel then requires (and checks) a 1024-byte aligned dynamic base.
+  static constexpr int SLACK = HD == 64 ? 0 : 1024;
+  static constexpr int SMEM = SLACK + Q_BYTES + STAGES * (K_BYTES + V_BYTES) + P_BYTES + 256;
+  static constexpr int TMEM_COLS = 256;                  // S: [0,128), O tile: [128, 128+HD)
+  static constexpr int MIN_BLOCKS = HD == 64 ? 2 : 1;
+};
+
+struct AttnTcArgs {
+  int rows, ctx, kv_len, n_heads, n_kv_heads, causal;
+  float scale_log2;
+  bf16* o;
+  int* status;
+};
+
+template <int HD>
+__global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
+    attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+                   const __grid_constant__ CUtensorMap tmV, const AttnTcArgs args) {
+  using C = AttnTcCfg<HD>;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = smem_raw;
+  if (C::SLACK) {
+    smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  } else if (smem_u32(smem_raw) & 1023) {
+    // the swizzled operand layout needs 1024-byte alignment: refuse (uniform exit, nothing started)
+    if (threadIdx.x == 0 && args.status) atomicOr(args.status, kErrLayout);
+    return;
+  }
+  uint8_t* sQ = smem;
+  uint8_t* sK = sQ + C::Q_BYTES;
+  uint8_t* sV = sK + C::STAGES * C::K_BYTES;
+  uint8_t* sP = sV + C::STAGES * C::V_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + C::P_BYTES);
+  uint64_t* q_full = bars;
+  uint64_t* kv_full = bars + 1;       // [2]
+  uint64_t* kv_empty = bars + 3;      // [2]
+  uint64_t* s_full = bars + 5;
+  uint64_t* s_free = bars + 6;
+  uint64_t* p_full = bars + 7;
+  uint64_t* o_full = bars + 8;
+  uint64_t* o_free = bars + 9;
+  uint64_t* drain = bars + 10;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 11);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int m0 = blockIdx.x * TQ, h = blockIdx.y, b = blockIdx.z;
+  const int hk = h / (args.n_heads / args.n_kv_heads);
+  const int kv_end = args.causal ? min(args.kv_len, args.ctx + min(m0 + TQ, args.rows)) : args.kv_len;
+  const int n_tiles = (kv_end + TKV - 1) / TKV;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&kv_full[s], 1);
+      mbar_init(&kv_empty[s], 1);
+    }
+    mbar_init(s_full, 1);
+    mbar_init(s_free, 128);
+    mbar_init(p_full, 128);
+    mbar_init(o_full, 1);
+    mbar_init(o_free, 128);
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    tma_prefetch_desc(&tmQ);
+    tma_prefetch_desc(&tmK);
+    tma_prefetch_desc(&tmV);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, C::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t t_s = tmem, t_o = tmem + 128;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------------------- producer
+      int issued0 = 0, issued1 = 0;
+      mbar_arrive_expect_tx(q_full, C::Q_BYTES);
+      for (int s = 0; s < HD / 64; ++s) tma_load_3d(sQ + s * 16384, &tmQ, q_full, 64 * s, m0, b * args.n_heads + h);
+      for (int j = 0; j < n_tiles; ++j) {
+        const int st = j & 1;
+        if (!mbar_wait_bounded(&kv_empty[st], ((j >> 1) & 1) ^ 1, abort_flag, args.status)) break;
+        mbar_arrive_expect_tx(&kv_full[st], C::K_BYTES + C::V_BYTES);
+        const int z = b * args.n_kv_heads + hk;
+        for (int s = 0; s < HD / 64; ++s)
+          tma_load_3d(sK + st * C::K_BYTES + s * 16384, &tmK, &kv_full[st], 64 * s, j * TKV, z);
+        for (int s = 0; s < 2; ++s)
+          tma_load_3d(sV + st * C::V_BYTES + s * HD * 128, &tmV, &kv_full[st], j * TKV + 64 * s, 0, z);
+        if (st) ++issued1; else ++issued0;
+      }
+      // every copy started here has landed before the CTA may exit
+      volatile int never = 0;
+      mbar_wait_bounded(q_full, 0, &never, args.status);
+      if (issued0 > 0) mbar_wait_bounded(&kv_full[0], (issued0 - 1) & 1, &never, args.status);
+      if (issued1 > 0) mbar_wait_bounded(&kv_full[1], (issued1 - 1) & 1, &never, args.status);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ------------------------------------------------------------- MMA issuer
+      constexpr uint32_t idesc_s = idesc_bf16_f32(TQ, TKV);
+      constexpr uint32_t idesc_o = idesc_bf16_f32(TQ, HD);
+      bool ok = mbar_wait_bounded(q_full, 0, abort_flag, args.status);
+      const uint32_t q0 = smem_u32(sQ), p0 = smem_u32(sP);
+      for (int j = 0; ok && j < n_tiles; ++j) {
+        const int st = j & 1;
+        if (!mbar_wait_bounded(&kv_full[st], (j >> 1) & 1, abort_flag, args.status)) break;
+        if (j > 0 && !mbar_wait_bounded(s_free, (j - 1) & 1, abort_flag, args.status)) break;
+        tc_fence_after();
+        const uint32_t k0 = smem_u32(sK + st * C::K_BYTES), v0 = smem_u32(sV + st * C::V_BYTES);
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk)
+          umma_bf16(t_s, sdesc_kmajor_sw128(q0 + (kk >> 2) * 16384 + (kk & 3) * 32),
+                    sdesc_kmajor_sw128(k0 + (kk >> 2) * 16384 + (kk & 3) * 32), idesc_s, kk != 0);
+        umma_commit(s_full);
+        if (!mbar_wait_bounded(p_full, j & 1, abort_flag, args.status)) break;
+        if (j > 0 && !mbar_wait_bounded(o_free, (j - 1) & 1, abort_flag, args.status)) break;
+        tc_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < TKV / 16; ++kk)
+          umma_bf16(t_o, sdesc_kmajor_sw128(p0 + (kk >> 2) * 16384 + (kk & 3) * 32),
+                    sdesc_kmajor_sw128(v0 + (kk >> 2) * (HD * 128) + (kk & 3) * 32), idesc_o, kk != 0);
+        umma_commit(o_full);
+        umma_commit(&kv_empty[st]);
+      }
+      umma_commit(drain);
+      volatile int never = 0;
+      mbar_wait_bounded(drain, 0, &never, args.status);
+    }
+  } else {
+    // --------------------------------------------------------------- softmax
+    const int quad = warp & 3;
+    const int row = quad * 32 + lane;                 // row within the tile = TMEM lane
+    const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+    const int qpos = args.ctx + m0 + row;
+    float o_acc[HD];
+#pragma unroll
+    for (int i = 0; i < HD; ++i) o_acc[i] = 0.0f;
+    float m_run = -INFINITY, l_run = 0.0f, alpha_prev = 0.0f;
+    bool ok = true;
+    uint8_t* prow0 = sP + row * 128;
+    for (int j = 0; j < n_tiles; ++j) {
+      if (!warp_wait_bounded(s_full, j & 1, abort_flag, args.status)) { ok = false; break; }
+      tc_fence_after();
+      const int key0 = j * TKV;
+      // keys visible to this row: key < kv_hi (kv_end, or the causal bound)
+      const int kv_hi = args.causal ? min(kv_end, qpos + 1) : kv_end;
+      const int lim = kv_hi - key0;                                   // visible keys of this tile
+      const bool masked = __any_sync(0xffffffffu, lim < TKV);         // warp-uniform path choice
+      float v[16];
+      float mx = -INFINITY;
+#pragma unroll
+      for (int c = 0; c < TKV / 16; ++c) {
+        tmem_ld16(t_s + lane_off + 16 * c, v);
+        if (masked) {
+#pragma unroll
+          for (int i = 0; i < 16; ++i) mx = fmaxf(mx, 16 * c + i < lim ? v[i] : -INFINITY);
+        } else {
+#pragma unroll
+          for (int i = 0; i < 16; ++i) mx = fmaxf(mx, v[i]);
+        }
+      }
+      const float m_new = fmaxf(m_run, mx * args.scale_log2);
+      const float alpha = (m_run == -INFINITY) ? 0.0f : ex2_approx(m_run - m_new);
+      if (j > 0) {
+        // O of the previous tile is ready: fold it in with its correction
+        if (!warp_wait_bounded(o_full, (j - 1) & 1, abort_flag, args.status)) { ok = false; break; }
+        tc_fence_after();
+#pragma unroll
+        for (int c = 0; c < HD / 16; ++c) {
+          tmem_ld16(t_o + lane_off + 16 * c, v);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) o_acc[16 * c + i] = fmaf(o_acc[16 * c + i], alpha_prev, v[i]);
+        }
+        tc_fence_before();
+        mbar_arrive(o_free);
+      }
+      // P = 2^(s * scale - m_new) as bf16 into the swizzled A-operand layout
+      float psum = 0.0f;
+#pragma unroll
+      for (int c = 0; c < TKV / 16; ++c) {
+        tmem_ld16(t_s + lane_off + 16 * c, v);
+        uint32_t pk[8];
+#pragma unroll
+        for (int i = 0; i < 16; i += 2) {
+          float p0 = ex2_approx(fmaf(v[i], args.scale_log2, -m_new));
+          float p1 = ex2_approx(fmaf(v[i + 1], args.scale_log2, -m_new));
+          if (masked) {
+            p0 = 16 * c + i < lim ? p0 : 0.0f;
+            p1 = 16 * c + i + 1 < lim ? p1 : 0.0f;
+          }
+          psum += p0 + p1;
+          __nv_bfloat162 t = __floats2bfloat162_rn(p0, p1);
+          pk[i / 2] = *reinterpret_cast<uint32_t*>(&t);
+        }
+        // keys 16c .. 16c+15: atom (16c / 64), 16-byte chunks (16c % 64) / 8 and +1
+        uint8_t* atom = prow0 + (c >> 2) * 16384;
+        const int chunk = (c & 3) * 2;
+        *reinterpret_cast<uint4*>(atom + ((chunk ^ (row & 7)) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+        *reinterpret_cast<uint4*>(atom + (((chunk + 1) ^ (row & 7)) << 4)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+      }
+      l_run = l_run * alpha + psum;
+      m_run = m_new;
+      alpha_prev = alpha;
+      tc_fence_before();
+      fence_proxy_async_smem();
+      mbar_arrive(s_free);
+      mbar_arrive(p_full);
+    }
+    if (ok && n_tiles > 0 && warp_wait_bounded(o_full, (n_tiles - 1) & 1, abort_flag, args.status)) {
+      tc_fence_after();
+      float v[16];
+#pragma unroll
+      for (int c = 0; c < HD / 16; ++c) {
+        tmem_ld16(t_o + lane_off + 16 * c, v);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) o_acc[16 * c + i] = fmaf(o_acc[16 * c + i], alpha_prev, v[i]);
+      }
+      const int grow = m0 + row;
+      if (grow < args.rows) {
+        const float inv = l_run > 0.0f ? 1.0f / l_run : 0.0f;
+        bf16* orow = args.o + (static_cast<size_t>(b) * args.rows + grow) * args.n_heads * HD +
+                     static_cast<size_t>(h) * HD;
+#pragma unroll
+        for (int i = 0; i < HD; i += 8) {
+          __nv_bfloat162 t0 = __floats2bfloat162_rn(o_acc[i] * inv, o_acc[i + 1] * inv);
+          __nv_bfloat162 t1 = __floats2bfloat162_rn(o_acc[i + 2] * inv, o_acc[i + 3] * inv);
+          __nv_bfloat162 t2 = __floats2bfloat162_rn(o_acc[i + 4] * inv, o_acc[i + 5] * inv);
+          __nv_bfloat162 t3 = __floats2bfloat162_rn(o_acc[i + 6] * inv, o_acc[i + 7] * inv);
+          *reinterpret_cast<uint4*>(orow + i) =
+              make_uint4(*reinterpret_cast<uint32_t*>(&t0), *reinterpret_cast<uint32_t*>(&t1),
+                         *reinterpret_cast<uint32_t*>(&t2), *reinterpret_cast<uint32_t*>(&t3));
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 g_enc = nullptr;
+std::once_flag g_enc_once;
+
+bool encoder() {
+  std::call_once(g_enc_once, [] {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      g_enc = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  });
+  return g_enc != nullptr;
+}
+
+// 3-D bf16 map: dims {d0 (contiguous), d1, d2}, byte strides {s1, s2}, box {64, box1, 1}, 128-byte swizzle.
+bool map3d(CUtensorMap* m, const void* ptr, uint64_t d0, uint64_t d1, uint64_t d2, uint64_t s1, uint64_t s2,
+           uint32_t box1) {
+  cuuint64_t dims[3] = {d0, d1, d2};
+  cuuint64_t strides[2] = {s1, s2};
+  cuuint32_t box[3] = {64, box1, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return g_enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int HD>
+const char* launch_tc(const AttnCall& a, int* status, cudaStream_t s) {
+  using C = AttnTcCfg<HD>;
+  if (!encoder()) return "cuTensorMapEncodeTiled is unavailable";
+  const int kv_len = a.ctx + a.rows;
+  CUtensorMap mq, mk, mv;
+  // Q: {hd, rows, B*Hq}; K: {hd, kv_len, B*Hkv}; V^T: {kv_len, hd, B*Hkv} -- positions past kv_len read zeros
+  if (!map3d(&mq, a.q, HD, a.rows, static_cast<uint64_t>(a.batch) * a.n_heads, HD * 2ull,
+             static_cast<uint64_t>(a.rows) * HD * 2, TQ) ||
+      !map3d(&mk, a.k, HD, kv_len, static_cast<uint64_t>(a.batch) * a.n_kv_heads, HD * 2ull,
+             static_cast<uint64_t>(a.kv_stride) * HD * 2, TKV) ||
+      !map3d(&mv, a.v, kv_len, HD, static_cast<uint64_t>(a.batch) * a.n_kv_heads, a.kv_stride * 2ull,
+             static_cast<uint64_t>(a.kv_stride) * HD * 2, HD))
+    return "attention tensor map encode failed";
+  static bool attr = false;
+  if (!attr) {
+    if (cudaFuncSetAttribute(attn_tc_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM) !=
+        cudaSuccess)
+      return "attention smem attribute failed";
+    attr = true;
+  }
+  AttnTcArgs args{a.rows, a.ctx, kv_len, a.n_heads, a.n_kv_heads, a.causal,
+                  1.4426950408889634f / sqrtf(static_cast<float>(HD)), static_cast<bf16*>(a.o), status};
+  dim3 grid((a.rows + TQ - 1) / TQ, a.n_heads, a.batch);
+  attn_tc_kernel<HD><<<grid, 192, C::SMEM, s>>>(mq, mk, mv, args);
+  cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
+}
+
+// ============================================================= mma.sync path
 constexpr int AM = 64, AN = 64;
 
 __device__ __forceinline__ void cp_async16(void* dst, const void* src, bool pred) {
@@ -27,11 +356,6 @@ __device__ __forceinline__ void cp_async_wait() { asm volatile("cp.async.wait_gr
 
 __device__ __forceinline__ void ldsm_x4(uint32_t (&r)[4], const void* p) {
   asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(smem_u32(p)));
-}
-__device__ __forceinline__ void ldsm_x4_t(uint32_t (&r)[4], const void* p) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
                : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
                : "r"(smem_u32(p)));
 }
@@ -49,26 +373,27 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 
 template <int HD>
 __global__ void __launch_bounds__(128) attn_bf16_kernel(const bf16* __restrict__ q, const bf16* __restrict__ k,
-                                                        const bf16* __restrict__ v, bf16* __restrict__ o,
+                                                        const bf16* __restrict__ vt, bf16* __restrict__ o,
                                                         int n_heads, int n_kv_heads, int rows, int ctx,
                                                         int kv_stride, int causal, float scale_log2) {
-  constexpr int LD = HD + 8;  // padded smem row (bf16), keeps ldmatrix rows 16-byte aligned
+  constexpr int LD = HD + 8;   // padded smem row of Q / K (bf16)
+  constexpr int LDV = AN + 8;  // padded smem row of V^T (one head dim, AN keys)
   extern __shared__ __align__(16) uint8_t smem_raw[];
   bf16* sQ = reinterpret_cast<bf16*>(smem_raw);
   bf16* sK = sQ + AM * LD;          // [2][AN][LD]
-  bf16* sV = sK + 2 * AN * LD;      // [2][AN][LD]
+  bf16* sV = sK + 2 * AN * LD;      // [2][HD][LDV]
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int m0 = blockIdx.x * AM, h = blockIdx.y, b = blockIdx.z;
   const int hk = h / (n_heads / n_kv_heads);
   const bf16* qb = q + (static_cast<size_t>(b) * n_heads + h) * rows * HD;
   const bf16* kb = k + (static_cast<size_t>(b) * n_kv_heads + hk) * kv_stride * HD;
-  const bf16* vb = v + (static_cast<size_t>(b) * n_kv_heads + hk) * kv_stride * HD;
+  const bf16* vb = vt + (static_cast<size_t>(b) * n_kv_heads + hk) * HD * kv_stride;
   const int kv_len = ctx + rows;
   const int kv_end = causal ? min(kv_len, ctx + min(m0 + AM, rows)) : kv_len;
   const int n_tiles = (kv_end + AN - 1) / AN;
 
-  constexpr int CPR = HD / 8;  // 16-byte chunks per row
+  constexpr int CPR = HD / 8;  // 16-byte chunks per Q / K row
   for (int i = tid; i < AM * CPR; i += 128) {
     const int r = i / CPR, c = i % CPR;
     const bool ok = m0 + r < rows;
@@ -79,9 +404,22 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const bf16* __restrict__
     for (int i = tid; i < AN * CPR; i += 128) {
       const int r = i / CPR, c = i % CPR;
       const bool ok = n0 + r < kv_end;
-      const size_t off = static_cast<size_t>(ok ? n0 + r : 0) * HD + c * 8;
-      cp_async16(sK + (buf * AN + r) * LD + c * 8, kb + off, ok);
-      cp_async16(sV + (buf * AN + r) * LD + c * 8, vb + off, ok);
+      cp_async16(sK + (buf * AN + r) * LD + c * 8, kb + static_cast<size_t>(ok ? n0 + r : 0) * HD + c * 8, ok);
+    }
+    if ((kv_stride & 7) == 0) {
+      for (int i = tid; i < HD * (AN / 8); i += 128) {
+        const int dd = i / (AN / 8), c = i % (AN / 8);
+        const bool ok = n0 + c * 8 < kv_end;   // keys past kv_end inside a chunk get P = 0
+        cp_async16(sV + (buf * HD + dd) * LDV + c * 8,
+                   vb + static_cast<size_t>(dd) * kv_stride + (ok ? n0 + c * 8 : 0), ok);
+      }
+    } else {
+      // rows of V^T are not 16-byte aligned: element loads, zeros past kv_end
+      for (int i = tid; i < HD * AN; i += 128) {
+        const int dd = i / AN, c = i % AN;
+        sV[(buf * HD + dd) * LDV + c] =
+            n0 + c < kv_end ? vb[static_cast<size_t>(dd) * kv_stride + n0 + c] : __float2bfloat16_rn(0.0f);
+      }
     }
   };
   if (n_tiles > 0) load_kv(0, 0);
@@ -92,7 +430,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const bf16* __restrict__
   for (int j = 0; j < HD / 8; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.0f;
   float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.0f, 0.0f};
   const int g = lane >> 2, t4 = lane & 3;
-  const int qpos0 = ctx + m0 + warp * 16 + g;  // absolute position of this thread's first row
+  const int qpos0 = ctx + m0 + warp * 16 + g;
   uint32_t qf[HD / 16][4];
 
   for (int t = 0; t < n_tiles; ++t) {
@@ -107,8 +445,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const bf16* __restrict__
         ldsm_x4(qf[kk], sQ + (warp * 16 + (lane & 15)) * LD + kk * 16 + (lane >> 4) * 8);
     }
     const bf16* Kt = sK + buf * AN * LD;
-    const bf16* Vt = sV + buf * AN * LD;
-    // S = Q K^T : 16 x 64 per warp
+    const bf16* Vt = sV + buf * HD * LDV;
     float s[AN / 8][4];
 #pragma unroll
     for (int j = 0; j < AN / 8; ++j) s[j][0] = s[j][1] = s[j][2] = s[j][3] = 0.0f;
@@ -124,7 +461,6 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const bf16* __restrict__
         mma_bf16_16816(s[2 * jj + 1], qf[kk], bfr[2], bfr[3]);
       }
     }
-    // mask and online softmax (rows g and g+8 of the warp's 16)
     const int n0 = t * AN;
     float tmax[2] = {-INFINITY, -INFINITY};
 #pragma unroll
@@ -166,7 +502,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const bf16* __restrict__
       acc[j][0] *= corr[0]; acc[j][1] *= corr[0];
       acc[j][2] *= corr[1]; acc[j][3] *= corr[1];
     }
-    // O += P V
+    // O += P V, V^T tile [dim][key] is the col-major B operand
 #pragma unroll
     for (int kk = 0; kk < AN / 16; ++kk) {
       uint32_t pa[4];
@@ -177,16 +513,15 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const bf16* __restrict__
 #pragma unroll
       for (int jj = 0; jj < HD / 16; ++jj) {
         uint32_t vfr[4];
-        const int key = kk * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
-        const int dim = jj * 16 + (lane >> 4) * 8;
-        ldsm_x4_t(vfr, Vt + key * LD + dim);
+        const int dim = jj * 16 + (lane & 7) + (lane >> 4) * 8;
+        const int key = kk * 16 + ((lane >> 3) & 1) * 8;
+        ldsm_x4(vfr, Vt + dim * LDV + key);
         mma_bf16_16816(acc[2 * jj], pa, vfr[0], vfr[1]);
         mma_bf16_16816(acc[2 * jj + 1], pa, vfr[2], vfr[3]);
       }
     }
     __syncthreads();
   }
-  // finish: row sums across the quad, normalise, store
 #pragma unroll
   for (int r = 0; r < 2; ++r) {
     lrow[r] += __shfl_xor_sync(0xffffffffu, lrow[r], 1);
@@ -210,7 +545,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const bf16* __restrict__
 // fp32: one warp per (query row, head, batch); each lane owns hd/32 dims.
 template <int HD>
 __global__ void __launch_bounds__(128) attn_f32_kernel(const float* __restrict__ q, const float* __restrict__ k,
-                                                       const float* __restrict__ v, float* __restrict__ o,
+                                                       const float* __restrict__ vt, float* __restrict__ o,
                                                        int n_heads, int n_kv_heads, int rows, int ctx,
                                                        int kv_stride, int causal, float scale) {
   constexpr int PL = HD / 32;
@@ -221,7 +556,7 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const float* __restrict__
   const int hk = h / (n_heads / n_kv_heads);
   const float* qr = q + ((static_cast<size_t>(b) * n_heads + h) * rows + row) * HD;
   const float* kb = k + (static_cast<size_t>(b) * n_kv_heads + hk) * kv_stride * HD;
-  const float* vb = v + (static_cast<size_t>(b) * n_kv_heads + hk) * kv_stride * HD;
+  const float* vb = vt + (static_cast<size_t>(b) * n_kv_heads + hk) * HD * kv_stride;
   float qv[PL], acc[PL];
 #pragma unroll
   for (int i = 0; i < PL; ++i) { qv[i] = qr[lane + 32 * i]; acc[i] = 0.0f; }
@@ -237,7 +572,7 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const float* __restrict__
     const float c = expf(m - mn), p = expf(d - mn);
     l = l * c + p;
 #pragma unroll
-    for (int i = 0; i < PL; ++i) acc[i] = acc[i] * c + p * vb[static_cast<size_t>(j) * HD + lane + 32 * i];
+    for (int i = 0; i < PL; ++i) acc[i] = acc[i] * c + p * vb[static_cast<size_t>(lane + 32 * i) * kv_stride + j];
     m = mn;
   }
   float* orow = o + (static_cast<size_t>(b) * rows + row) * n_heads * HD + static_cast<size_t>(h) * HD;
@@ -247,8 +582,8 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const float* __restrict__
 
 template <int HD>
 cudaError_t launch_bf16(const AttnCall& a, cudaStream_t s) {
-  constexpr int LD = HD + 8;
-  const size_t smem = static_cast<size_t>(AM + 4 * AN) * LD * sizeof(bf16);
+  const size_t smem = static_cast<size_t>(AM + 2 * AN) * (HD + 8) * sizeof(bf16) +
+                      static_cast<size_t>(2 * HD) * (AN + 8) * sizeof(bf16);
   static bool attr = false;
   if (!attr) {
     cudaError_t e = cudaFuncSetAttribute(attn_bf16_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -279,17 +614,17 @@ const char* attention(const AttnCall& a, cudaStream_t s) {
   if (a.rows <= 0 || a.batch <= 0) return nullptr;
   if (a.n_kv_heads <= 0 || a.n_heads % a.n_kv_heads) return "n_heads must be a multiple of n_kv_heads";
   if (a.kv_stride < a.ctx + a.rows) return "kv_stride smaller than ctx + rows";
-  cudaError_t e;
   if (a.bf16) {
-    if (a.head_dim == 64) e = launch_bf16<64>(a, s);
-    else if (a.head_dim == 128) e = launch_bf16<128>(a, s);
-    else return "bf16 attention supports head_dim 64 and 128";
-  } else {
-    if (a.head_dim == 32) e = launch_f32<32>(a, s);
-    else if (a.head_dim == 64) e = launch_f32<64>(a, s);
-    else if (a.head_dim == 128) e = launch_f32<128>(a, s);
-    else return "fp32 attention supports head_dim 32, 64 and 128";
+    const bool tc = a.rows >= TQ && a.kv_stride % 8 == 0;
+    if (a.head_dim == 64) return tc ? launch_tc<64>(a, a.status, s) : (launch_bf16<64>(a, s) == cudaSuccess ? nullptr : "attention launch failed");
+    if (a.head_dim == 128) return tc ? launch_tc<128>(a, a.status, s) : (launch_bf16<128>(a, s) == cudaSuccess ? nullptr : "attention launch failed");
+    return "bf16 attention supports head_dim 64 and 128";
   }
+  cudaError_t e;
+  if (a.head_dim == 32) e = launch_f32<32>(a, s);
+  else if (a.head_dim == 64) e = launch_f32<64>(a, s);
+  else if (a.head_dim == 128) e = launch_f32<128>(a, s);
+  else return "fp32 attention supports head_dim 32, 64 and 128";
   return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
 }
 

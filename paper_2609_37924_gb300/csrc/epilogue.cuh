@@ -12,7 +12,7 @@ namespace tadm {
 enum EpiKind : int {
   EPI_STORE = 0,     // out = acc
   EPI_RESID = 1,     // resid += acc (+ bias)
-  EPI_QKV = 2,       // split into Q / K / V heads, optional RoPE, K/V into the cache
+  EPI_QKV = 2,       // split into Q / K / V heads, optional RoPE, K and V^T into the cache
   EPI_GLU = 3,       // out = act(gate) * up (gate and up are the two halves of the tile)
   EPI_FUSION1 = 4,   // [g | hidden] = [sigmoid(acc + b) | GELU(acc + b)]
   EPI_FUSION2 = 5,   // out = h + g * (acc + b)
@@ -33,7 +33,7 @@ struct EpiParams {
   int ldb;
   const void* bias;         // [N] weights dtype
   int bias_bf16;
-  // EPI_QKV
+  // EPI_QKV: q [B, Hq, R, hd], k [B, Hkv, kv_stride, hd], v transposed [B, Hkv, hd, kv_stride]
   void *q, *k, *v;
   int R, ctx, kv_stride, n_heads, n_kv_heads, head_dim, rope;
   const float2* rope_tab;   // [position][head_dim / 2] = (cos, sin)
@@ -101,6 +101,21 @@ __device__ __forceinline__ void store32(void* base, int bf, size_t off, const fl
   }
 }
 
+// Stores 32 values of one row as one column of a transposed layout: element i
+// goes to base[off + i * stride].  Across a warp whose lanes hold consecutive
+// rows, each of the 32 stores writes 32 consecutive elements.
+__device__ __forceinline__ void store_col32(void* base, int bf, size_t off, int stride, const float (&v)[32]) {
+  if (bf) {
+    bf16* p = static_cast<bf16*>(base) + off;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) p[static_cast<size_t>(i) * stride] = __float2bfloat16_rn(v[i]);
+  } else {
+    float* p = static_cast<float*>(base) + off;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) p[static_cast<size_t>(i) * stride] = v[i];
+  }
+}
+
 __device__ __forceinline__ void load32f(const float* p, int n_valid, float (&v)[32]) {
   if (n_valid >= 32 && (reinterpret_cast<uintptr_t>(p) & 15) == 0) {
     const float4* p4 = reinterpret_cast<const float4*>(p);
@@ -127,14 +142,23 @@ __device__ __forceinline__ void load32a(const void* p, int bf, size_t off, int n
 // of 64) are available from src.load(chunk, v); the tile's first output column
 // is n_blk * ncols (n_blk * ncols / 2 for EPI_GLU).  Control flow is uniform
 // across a warp except for the stores (src.load may be warp-collective).
+//
+// The tile's columns may be split between `nsplit` threads per row (one per
+// warp of a lane quadrant); split `part` handles its share: chunks
+// [part * nch / nsplit, (part + 1) * nch / nsplit) (for EPI_GLU the same share
+// of gate chunks and their up partners; for EPI_QKV whole heads; EPI_LMHEAD
+// writes one partial per split, indexed n_blk * nsplit + part; EPI_PA_GATE
+// needs nsplit == 1).
 template <int EPI, class Src>
-__device__ __forceinline__ void epilogue_row(const EpiParams& p, int m, int n_blk, int ncols, Src& src) {
+__device__ __forceinline__ void epilogue_row(const EpiParams& p, int m, int n_blk, int ncols, Src& src,
+                                             int part = 0, int nsplit = 1) {
   const bool row_ok = m < p.M;
   const int nch = ncols / 32;
+  const int c_lo = part * nch / nsplit, c_hi = (part + 1) * nch / nsplit;
   float v[32];
   if constexpr (EPI == EPI_STORE || EPI == EPI_RESID || EPI == EPI_SILU || EPI == EPI_ADD ||
                 EPI == EPI_FUSION1 || EPI == EPI_FUSION2 || EPI == EPI_PA_UP) {
-    for (int c = 0; c < nch; ++c) {
+    for (int c = c_lo; c < c_hi; ++c) {
       src.load(c, v);
       const int n0 = n_blk * ncols + 32 * c;
       const int nv = min(32, p.N - n0);
@@ -197,7 +221,8 @@ __device__ __forceinline__ void epilogue_row(const EpiParams& p, int m, int n_bl
     }
   } else if constexpr (EPI == EPI_GLU) {
     const int half = ncols / 2;
-    for (int c = 0; c < half / 32; ++c) {
+    const int g_lo = part * (half / 32) / nsplit, g_hi = (part + 1) * (half / 32) / nsplit;
+    for (int c = g_lo; c < g_hi; ++c) {
       float u[32];
       src.load(c, v);
       src.load(c + half / 32, u);
@@ -213,20 +238,21 @@ __device__ __forceinline__ void epilogue_row(const EpiParams& p, int m, int n_bl
     const int hpt = ncols / hd;       // heads per tile
     const int b = m / p.R, r = m - (m / p.R) * p.R;
     const int pos = p.ctx + r;
-    for (int hh = 0; hh < hpt; ++hh) {
+    for (int hh = part * hpt / nsplit; hh < (part + 1) * hpt / nsplit; ++hh) {
       const int nb = n_blk * ncols + hh * hd;
       const int gh = nb / hd;
       int region = 2, head = gh - p.n_heads - p.n_kv_heads;
       if (gh < p.n_heads) { region = 0; head = gh; }
       else if (gh < p.n_heads + p.n_kv_heads) { region = 1; head = gh - p.n_heads; }
       void* dst;
-      size_t off;
+      size_t off, vt_off = 0;
       if (region == 0) {
         dst = p.q;
         off = ((static_cast<size_t>(b) * p.n_heads + head) * p.R + r) * hd;
       } else {
         dst = region == 1 ? p.k : p.v;
         off = ((static_cast<size_t>(b) * p.n_kv_heads + head) * p.kv_stride + pos) * hd;
+        vt_off = (static_cast<size_t>(b) * p.n_kv_heads + head) * hd * p.kv_stride + pos;
       }
       const bool ok = row_ok && nb < p.N;
       if (hd == 32) {  // rotate-half pairs (i, i + 16) inside one chunk
@@ -242,7 +268,11 @@ __device__ __forceinline__ void epilogue_row(const EpiParams& p, int m, int n_bl
             v[i + 16] = c2 * cs.x + a * cs.y;
           }
         }
-        store32(dst, p.out_bf16, off, v, 32);
+        if (region == 2) {
+          store_col32(dst, p.out_bf16, vt_off, p.kv_stride, v);
+        } else {
+          store32(dst, p.out_bf16, off, v, 32);
+        }
         continue;
       }
       for (int j2 = 0; j2 < hd / 64; ++j2) {
@@ -261,14 +291,21 @@ __device__ __forceinline__ void epilogue_row(const EpiParams& p, int m, int n_bl
             w[i] = c2 * cs.x + a * cs.y;
           }
         }
-        store32(dst, p.out_bf16, off + 32 * j2, v, 32);
-        store32(dst, p.out_bf16, off + hd / 2 + 32 * j2, w, 32);
+        if (region == 2) {   // V is stored transposed: [b][head][dim][position]
+          store_col32(dst, p.out_bf16, vt_off + static_cast<size_t>(32 * j2) * p.kv_stride, p.kv_stride, v);
+          store_col32(dst, p.out_bf16, vt_off + static_cast<size_t>(hd / 2 + 32 * j2) * p.kv_stride, p.kv_stride, w);
+        } else {
+          store32(dst, p.out_bf16, off + 32 * j2, v, 32);
+          store32(dst, p.out_bf16, off + hd / 2 + 32 * j2, w, 32);
+        }
       }
     }
   } else if constexpr (EPI == EPI_LMHEAD) {
+    // sum of exp(l - max) as exp2((l - max) * log2 e)
+    constexpr float kLog2e = 1.4426950408889634f;
     float mx = -INFINITY, sum = 0.0f;
     int arg = -1;
-    for (int c = 0; c < nch; ++c) {
+    for (int c = c_lo; c < c_hi; ++c) {
       src.load(c, v);
       const int n0 = n_blk * ncols + 32 * c;
       const int nv = min(32, p.N - n0);
@@ -283,18 +320,19 @@ __device__ __forceinline__ void epilogue_row(const EpiParams& p, int m, int n_bl
       }
       if (carg < 0) continue;
       const float nm = fmaxf(mx, cmx);
-      float s = (mx == -INFINITY) ? 0.0f : sum * expf(mx - nm);
+      const float nms = nm * kLog2e;
+      float s = (mx == -INFINITY) ? 0.0f : sum * exp2f(fmaf(mx, kLog2e, -nms));
 #pragma unroll
       for (int i = 0; i < 32; ++i) {
         const int n = n0 + i;
-        if (i < nv && n != p.mask_id) s += expf(v[i] - nm);
+        if (i < nv && n != p.mask_id) s += exp2f(fmaf(v[i], kLog2e, -nms));
       }
       if (cmx > mx) arg = carg;
       mx = nm;
       sum = s;
     }
     if (row_ok) {
-      float* o = p.part + (static_cast<size_t>(m) * p.n_tiles + n_blk) * 3;
+      float* o = p.part + (static_cast<size_t>(m) * p.n_tiles + n_blk * nsplit + part) * 3;
       o[0] = mx;
       o[1] = sum;
       o[2] = __int_as_float(arg);

@@ -7,9 +7,10 @@
 //               shared-memory ring (128-byte swizzle);
 //   warp 1      allocates 512 TMEM columns (two 128 x 256 fp32 accumulators)
 //               and one thread issues tcgen05.mma (M=128, N=256, K=16);
-//   warps 2..5  epilogue: tcgen05.ld the accumulator rows (one TMEM lane per
-//               thread) and run the fused epilogue of epilogue.cuh, while the
-//               MMA warp fills the other accumulator.
+//   warps 2..9  epilogue: tcgen05.ld the accumulator rows (one TMEM lane per
+//               thread; two warps per lane quadrant, each taking half of the
+//               256 columns) and run the fused epilogue of epilogue.cuh, while
+//               the MMA warp fills the other accumulator.
 // Every mbarrier wait is bounded (mbar_wait_bounded): a role that gives up
 // raises a shared abort flag and the device status word, and the CTA drains
 // its in-flight copies and MMAs, frees TMEM and exits.
@@ -27,7 +28,8 @@ constexpr int A_BYTES = BM * BK * 2;   // 16 KB
 constexpr int B_BYTES = BN * BK * 2;   // 32 KB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = 512;
-constexpr int NUM_THREADS = 192;
+constexpr int EPI_WARPS = 8;
+constexpr int NUM_THREADS = 64 + 32 * EPI_WARPS;
 constexpr size_t SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;
 
 struct TmemSrc {
@@ -70,7 +72,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
-      mbar_init(&tempty[a], 128);
+      mbar_init(&tempty[a], 32 * EPI_WARPS);
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -161,15 +163,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
   } else {
     // ------------------------------------------------------------------ epilogue
-    const int quad = warp & 3;   // TMEM lanes 32*quad .. 32*quad+31
+    const int quad = warp & 3;               // TMEM lanes 32*quad .. 32*quad+31 (hardware rule)
+    const int part = (warp - 2) / 4;         // which half of the columns
+    constexpr int nsplit = EPI == EPI_PA_GATE ? 1 : 2;
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
-      if (!mbar_wait_bounded(&tfull[acc], acc_phase, abort_flag, args.status)) break;
+      if (!warp_wait_bounded(&tfull[acc], acc_phase, abort_flag, args.status)) break;
       tc_fence_after();
       const int mb = tile % num_m, nb = tile / num_m;
       TmemSrc src{tmem_base + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(quad * 32) << 16)};
-      epilogue_row<EPI>(args.ep, mb * BM + quad * 32 + lane, nb, BN, src);
+      if (part < nsplit) epilogue_row<EPI>(args.ep, mb * BM + quad * 32 + lane, nb, BN, src, part, nsplit);
       tc_fence_before();
       mbar_arrive(&tempty[acc]);
       if (++acc == 2) { acc = 0; acc_phase ^= 1; }
@@ -257,7 +261,7 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
   a.ep = g.ep;
   a.ep.M = g.M;
   a.ep.N = g.N;
-  a.ep.n_tiles = a.n_tiles_n;
+  a.ep.n_tiles = a.n_tiles_n * (g.epi == EPI_LMHEAD ? 2 : 1);   // one partial per column half
   const int tiles = ((g.M + BM - 1) / BM) * a.n_tiles_n;
   const int grid = tiles < g_num_sms ? tiles : g_num_sms;
   cudaError_t e;
@@ -278,6 +282,9 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
   return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
 }
 
-int gemm_tc_tiles_n(int N, int epi) { return epi == EPI_GLU ? (N + 127) / 128 : (N + 255) / 256; }
+int gemm_tc_tiles_n(int N, int epi) {
+  if (epi == EPI_LMHEAD) return 2 * ((N + 255) / 256);   // partials: one per half tile
+  return epi == EPI_GLU ? (N + 127) / 128 : (N + 255) / 256;
+}
 
 }  // namespace tadm

@@ -25,11 +25,13 @@ int gemm_tc_tiles_n(int N, int epi);
 const char* gemm_simt(const GemmCall& g, cudaStream_t s);
 int gemm_simt_tiles_n(int N, int epi);
 
+// q [B, Hq, rows, hd]; k [B, Hkv, kv_stride, hd]; v transposed [B, Hkv, hd, kv_stride]
 struct AttnCall {
   const void *q, *k, *v;
   void* o;
   int batch, n_heads, n_kv_heads, head_dim, rows, ctx, kv_stride, causal;
   int bf16;
+  int* status;   // device status word (may be null)
 };
 const char* attention(const AttnCall& a, cudaStream_t s);
 

@@ -210,7 +210,7 @@ void layout(tadm_handle* h) {
     o = align_up(o + bytes, 256);
     return at;
   };
-  h->kv_stride = h->max_ctx > 0 ? h->max_ctx : h->max_rows;
+  h->kv_stride = static_cast<int>(align_up(static_cast<size_t>(h->max_ctx > 0 ? h->max_ctx : h->max_rows), 8));
   const int n_pos = h->kv_stride + h->max_rows;
   h->n_part_tiles = c.dtype ? gemm_tc_tiles_n(c.vocab, EPI_LMHEAD) : gemm_simt_tiles_n(c.vocab, EPI_LMHEAD);
   auto& f = h->off;
@@ -313,7 +313,7 @@ tadm_status layer_fwd(tadm_handle* h, int li, float* x, int B, int R, int ctx, i
   ep.rope_tab = h->at<const float2>(h->off.rope);
   TRYS(gemm(h, norm, Mmax, d, L.wqkv, d, M, nqkv, d, EPI_QKV, ep, s));
   AttnCall a{ep.q, ep.k, ep.v, h->at(h->off.attn), B, c.n_heads, c.n_kv_heads, hd, R, ctx, h->kv_stride, causal,
-             h->act_bf16()};
+             h->act_bf16(), h->status()};
   TRY(attention(a, s));
   EpiParams er{};
   er.resid = x;
@@ -363,7 +363,7 @@ tadm_status mixer(tadm_handle* h, const float* Z, const float* U, int B, int R, 
   eq.head_dim = hd;
   eq.rope = 0;
   TRYS(gemm(h, J, Mmax, 2 * r, h->fw[2], 2 * r, M, 3 * r, 2 * r, EPI_QKV, eq, s));
-  AttnCall a{eq.q, eq.k, eq.v, h->at(h->off.pa_mo), B, fh, fh, hd, R, 0, R, 0, h->act_bf16()};
+  AttnCall a{eq.q, eq.k, eq.v, h->at(h->off.pa_mo), B, fh, fh, hd, R, 0, R, 0, h->act_bf16(), h->status()};
   TRY(attention(a, s));
   EpiParams e1{};
   e1.base = Z;
@@ -740,6 +740,9 @@ tadm_status tadm_bind_workspace(tadm_handle* h, void* dev_ptr, size_t bytes) {
   cudaStream_t s = nullptr;
   TRY(rope_table(h->at<float2>(h->off.rope), n_pos, h->cfg.head_dim, h->cfg.rope_theta, s));
   if (cudaMemsetAsync(h->status(), 0, 256, s) != cudaSuccess) return fail(h, TADM_ERR_CUDA, "memset failed");
+  // K / V positions that were never written are read with zero weight; keep them finite
+  if (cudaMemsetAsync(h->at(h->off.kv), 0, h->off.attn - h->off.kv, s) != cudaSuccess)
+    return fail(h, TADM_ERR_CUDA, "memset failed");
   if (cudaStreamSynchronize(s) != cudaSuccess) return fail(h, TADM_ERR_CUDA, "bind: %s", cudaGetErrorString(cudaGetLastError()));
   return TADM_OK;
 }
@@ -870,6 +873,7 @@ tadm_status tadm_sync_status(tadm_handle* h) {
   if (cudaMemcpy(&st, h->status(), sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess)
     return fail(h, TADM_ERR_CUDA, "status read failed");
   if (st & kErrTimeout) return fail(h, TADM_ERR_TIMEOUT, "a kernel gave up a bounded wait (status 0x%x)", st);
+  if (st & kErrLayout) return fail(h, TADM_ERR_CUDA, "a kernel found its shared memory misaligned (status 0x%x)", st);
   return TADM_OK;
 }
 
@@ -948,7 +952,7 @@ tadm_status tadm_attention(const void* q, const void* k, const void* v, void* o,
                            int head_dim, int rows, int ctx, int kv_stride, int causal, int dtype, tadm_stream stream) {
   if (!q || !k || !v || !o || batch < 0 || n_heads <= 0 || n_kv_heads <= 0 || rows < 0 || ctx < 0)
     return TADM_ERR_INVALID_ARG;
-  AttnCall a{q, k, v, o, batch, n_heads, n_kv_heads, head_dim, rows, ctx, kv_stride, causal, dtype};
+  AttnCall a{q, k, v, o, batch, n_heads, n_kv_heads, head_dim, rows, ctx, kv_stride, causal, dtype, nullptr};
   return attention(a, stream) ? TADM_ERR_CUDA : TADM_OK;
 }
 

@@ -63,14 +63,17 @@ def test_gemm_f32_cuda_cores(T, M, N, K):
 
 
 # -------------------------------------------------------------------------- attention
-@pytest.mark.parametrize("hd,Hq,Hkv,rows,ctx,causal", [
-    (64, 4, 4, 70, 0, False), (64, 4, 2, 64, 0, True), (128, 4, 2, 32, 37, False), (128, 2, 1, 100, 130, True),
-    (64, 12, 12, 1024, 0, False)])
-def test_attention_bf16(T, hd, Hq, Hkv, rows, ctx, causal):
-    B, stride = 2, ctx + rows + 5
+# rows >= 128 with kv_stride % 8 == 0 run the tcgen05 kernel, the others mma.sync
+@pytest.mark.parametrize("hd,Hq,Hkv,rows,ctx,causal,pad", [
+    (64, 4, 4, 70, 0, False, 5), (64, 4, 2, 64, 0, True, 5), (128, 4, 2, 32, 37, False, 5),
+    (128, 2, 1, 100, 130, True, 5), (64, 12, 12, 1024, 0, False, 0), (64, 4, 2, 300, 77, True, 3),
+    (128, 4, 2, 260, 0, False, 4), (128, 2, 2, 512, 200, True, 0), (64, 2, 1, 200, 0, False, 1)])
+def test_attention_bf16(T, hd, Hq, Hkv, rows, ctx, causal, pad):
+    B, stride = 2, ctx + rows + pad
     q, qd = bf16_tensor((B, Hq, rows, hd), 5)
     k, kd = bf16_tensor((B, Hkv, stride, hd), 6)
-    v, vd = bf16_tensor((B, Hkv, stride, hd), 7)
+    vt, vtd = bf16_tensor((B, Hkv, hd, stride), 7)       # V is passed transposed
+    v, vd = vt, vtd.transpose(0, 1, 3, 2)
     o = torch.empty((B * rows, Hq * hd), dtype=torch.bfloat16, device="cuda")
     T.tadm_attention(q, k, v, o, Hq, Hkv, rows, ctx, causal, dtype=1)
     torch.cuda.synchronize()
@@ -91,7 +94,8 @@ def test_attention_f32(T, hd, causal):
     stride = ctx + rows
     q, qd = f32_tensor((B, Hq, rows, hd), 8)
     k, kd = f32_tensor((B, Hkv, stride, hd), 9)
-    v, vd = f32_tensor((B, Hkv, stride, hd), 10)
+    v, vtd = f32_tensor((B, Hkv, hd, stride), 10)        # V is passed transposed
+    vd = vtd.transpose(0, 1, 3, 2)
     o = torch.empty((B * rows, Hq * hd), dtype=torch.float32, device="cuda")
     T.tadm_attention(q, k, v, o, Hq, Hkv, rows, ctx, causal, dtype=0)
     torch.cuda.synchronize()
