@@ -42,6 +42,9 @@ def parse():
     ap.add_argument("--batch", type=int, default=None)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-sample-seconds", type=float, default=20.0)
+    ap.add_argument("--T", type=int, default=None,
+                    help="override reverse steps per block (short runs for launch-list profiles)")
+    ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
     ap.add_argument("--kernel-bench", default=None,
                     help="time one building block alone instead, e.g. gemm:16384,32768,768")
     return ap.parse_args()
@@ -201,9 +204,12 @@ def gpu_arm(args):
     torch.cuda.set_device(local)
     if world > 1:
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-    w = wl.get_workload(args.workload)
+    over = {}
     if args.batch:
-        w = wl.get_workload(args.workload, batch=args.batch)
+        over["batch"] = args.batch
+    if args.T:
+        over["steps_per_block"] = args.T
+    w = wl.get_workload(args.workload, **over)
     K = args.K or w.K
     m = w.model
     B = w.batch
@@ -231,7 +237,7 @@ def gpu_arm(args):
             one(Kv)
         tm.tadm_sync_status()
         if probe:
-            tm.tadm_probe_enable(8192)
+            tm.tadm_probe_enable(40000)
         barrier()
         launches = 0
         ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -242,7 +248,8 @@ def gpu_arm(args):
         ev1.record(stream)
         barrier()
         ms = ev0.elapsed_time(ev1)
-        pr = tm.tadm_probe_read() if probe else None
+        brk = tm.tadm_probe_breakdown() if probe else None
+        pr = (tm.tadm_probe_read(), brk) if probe else None
         if probe:
             tm.tadm_probe_enable(0)
         tm.tadm_sync_status()
@@ -267,23 +274,24 @@ def gpu_arm(args):
 
     # e2e: public API with host buffers (pinned prompt in, tokens out), copies inside the timed region
     hp = torch.from_numpy(prompts).pin_memory()
-    for _ in range(args.warmup):
+    for _ in range(0 if args.no_e2e else args.warmup):
         tm.generate(hp, w.gen_len, w.steps_per_block, K, bl)
     barrier()
     t0 = time.perf_counter()
-    for _ in range(args.steps):
+    res = out
+    for _ in range(0 if args.no_e2e else args.steps):
         res = tm.generate(hp, w.gen_len, w.steps_per_block, K, bl)
     barrier()
-    e2e_s = time.perf_counter() - t0
+    e2e_s = max(time.perf_counter() - t0, 1e-9)
     if world > 1:
         t = torch.tensor([e2e_s], device="cuda")
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         e2e_s = float(t.item())
-    e2e = {"value": world * tokens_per_step * args.steps / e2e_s, "unit": "tokens/s",
+    e2e = None if args.no_e2e else {"value": world * tokens_per_step * args.steps / e2e_s, "unit": "tokens/s",
            "h2d_bytes_per_step": int(hp.numel() * 4), "d2h_bytes_per_step": int(res.numel() * 4)}
 
     peaks = load_peaks()
-    n_launch, gemm_ms, gemm_flops = probe
+    (n_launch, gemm_ms, gemm_flops), gemm_kinds = probe
     achieved = gemm_flops / (gemm_ms / 1000.0) / 1e12 if gemm_ms > 0 else None
     if peaks:
         peak, peak_src = peaks["bf16_tflops_sustained"], "measured sustained bf16 (MEASURED_PEAKS.json)"
@@ -293,7 +301,10 @@ def gpu_arm(args):
                 "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                 "frac": (achieved / peak) if achieved else None, "traffic": None, "peak_source": peak_src,
                 "launches_timed": n_launch, "gemm_ms_per_step": gemm_ms / args.steps,
-                "gemm_share_of_step": gemm_ms / ms if ms else None}
+                "gemm_share_of_step": gemm_ms / ms if ms else None,
+                "by_epilogue": {k: {"ms_per_step": v["ms"] / args.steps, "tflops": round(v["tflops"], 1),
+                                    "launches_per_step": v["launches"] / args.steps}
+                                for k, v in gemm_kinds.items()}}
 
     line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,

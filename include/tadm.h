@@ -218,6 +218,12 @@ TADM_API tadm_status tadm_get_counters(const tadm_handle* h, tadm_counters* out)
  * clears the records.  tadm_probe_enable(h, 0) frees the events. */
 TADM_API tadm_status tadm_probe_enable(tadm_handle* h, int max_launches);
 TADM_API tadm_status tadm_probe_read(tadm_handle* h, int64_t* launches, double* total_ms, double* total_flops);
+/* The same records split by GEMM epilogue kind (0 plain, 1 residual, 2 QKV +
+ * RoPE, 3 GLU, 4 fusion gate/hidden, 5 fusion output, 6 output head,
+ * 7..10 paired-attention fusion): arrays of n_kinds entries.  Call before
+ * tadm_probe_read, which clears the records. */
+TADM_API tadm_status tadm_probe_breakdown(tadm_handle* h, int n_kinds, int64_t* launches, double* ms,
+                                          double* flops);
 
 /* Plan of tadm_generate (host only, no GPU): the ordered phases it issues.
  * kind: 0 prefill, 1 anchor refresh, 2 denoise step, 3 commit.  For kinds 1

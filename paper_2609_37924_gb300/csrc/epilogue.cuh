@@ -36,7 +36,8 @@ struct EpiParams {
   // EPI_QKV: q [B, Hq, R, hd], k [B, Hkv, kv_stride, hd], v transposed [B, Hkv, hd, kv_stride]
   void *q, *k, *v;
   int R, ctx, kv_stride, n_heads, n_kv_heads, head_dim, rope;
-  const float2* rope_tab;   // [position][head_dim / 2] = (cos, sin)
+  const float2* rope_tab;   // [head_dim / 2][n_pos] = (cos, sin): a warp's consecutive positions read consecutive entries
+  int rope_npos;
   // EPI_GLU
   int glu;                  // 0 SiLU, 1 tanh-GELU
   // EPI_FUSION1 / EPI_ADD
@@ -156,6 +157,75 @@ __device__ __forceinline__ void epilogue_row(const EpiParams& p, int m, int n_bl
   const int nch = ncols / 32;
   const int c_lo = part * nch / nsplit, c_hi = (part + 1) * nch / nsplit;
   float v[32];
+  // Sources that can stage (tensor-core path) write bf16 outputs 64 columns at
+  // a time through shared memory with one TMA store per warp (full lines).
+  if constexpr (Src::kStaged && (EPI == EPI_STORE || EPI == EPI_FUSION1)) {
+    if (src.staged()) {
+      float w[32];
+      for (int c = c_lo; c + 1 < c_hi; c += 2) {
+        src.load(c, v);
+        src.load(c + 1, w);
+        const int n0 = n_blk * ncols + 32 * c;
+        int which = 0, x = n0;
+        if constexpr (EPI == EPI_FUSION1) {
+          const bool gate = n0 < p.d_split;     // d_split is a multiple of 64
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const float b0 = n0 + i < p.N ? ld_param(p.bias, p.bias_bf16, n0 + i) : 0.0f;
+            const float b1 = n0 + 32 + i < p.N ? ld_param(p.bias, p.bias_bf16, n0 + 32 + i) : 0.0f;
+            v[i] = gate ? sigmoid_f(v[i] + b0) : gelu_erf_f(v[i] + b0);
+            w[i] = gate ? sigmoid_f(w[i] + b1) : gelu_erf_f(w[i] + b1);
+          }
+          which = gate ? 0 : 1;
+          x = gate ? n0 : n0 - p.d_split;
+        }
+        src.store64(which, x, v, w);
+      }
+      return;
+    }
+  }
+  // fp32 read-modify-write epilogues on the tensor-core path: the warp's 32 x 32
+  // accumulator chunk is transposed through its shared-memory box so that each
+  // global access instruction covers 32 consecutive columns of one row.
+  if constexpr (Src::kStaged && (EPI == EPI_RESID || EPI == EPI_FUSION2)) {
+    if (src.has_box()) {
+      const int lane = threadIdx.x & 31;
+      for (int c = c_lo; c < c_hi; ++c) {
+        src.load(c, v);
+        src.put_row(v);
+        const int n = n_blk * ncols + 32 * c + lane;
+        const bool col_ok = n < p.N;
+        const float bias = (p.bias && col_ok) ? ld_param(p.bias, p.bias_bf16, n) : 0.0f;
+        const int nrows = min(32, p.M - src.row0);
+#pragma unroll
+        for (int h0 = 0; h0 < 32; h0 += 16) {     // 16 rows at a time: loads first, then the stores
+          float xv[16], gv[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const size_t m_i = static_cast<size_t>(src.row0 + h0 + i);
+            const bool ok = h0 + i < nrows && col_ok;
+            if constexpr (EPI == EPI_RESID) {
+              xv[i] = ok ? p.resid[m_i * p.ldr + n] : 0.0f;
+            } else {
+              xv[i] = ok ? p.base[m_i * p.ldb + n] : 0.0f;
+              gv[i] = ok ? ld_param(p.gate, p.out_bf16, static_cast<int>(m_i * p.ldg + n)) : 0.0f;
+            }
+          }
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            const size_t m_i = static_cast<size_t>(src.row0 + h0 + i);
+            if (h0 + i < nrows && col_ok) {
+              const float a = src.get(h0 + i);
+              if constexpr (EPI == EPI_RESID) p.resid[m_i * p.ldr + n] = xv[i] + a + bias;
+              else static_cast<float*>(p.out)[m_i * p.ldo + n] = xv[i] + gv[i] * (a + bias);
+            }
+          }
+        }
+        __syncwarp();   // the box is rewritten by the next chunk
+      }
+      return;
+    }
+  }
   if constexpr (EPI == EPI_STORE || EPI == EPI_RESID || EPI == EPI_SILU || EPI == EPI_ADD ||
                 EPI == EPI_FUSION1 || EPI == EPI_FUSION2 || EPI == EPI_PA_UP) {
     for (int c = c_lo; c < c_hi; ++c) {
@@ -222,6 +292,23 @@ __device__ __forceinline__ void epilogue_row(const EpiParams& p, int m, int n_bl
   } else if constexpr (EPI == EPI_GLU) {
     const int half = ncols / 2;
     const int g_lo = part * (half / 32) / nsplit, g_hi = (part + 1) * (half / 32) / nsplit;
+    if constexpr (Src::kStaged) {
+      if (src.staged()) {
+        float w[32], u[32];
+        for (int c = g_lo; c + 1 < g_hi; c += 2) {
+          src.load(c, v);
+          src.load(c + half / 32, u);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] = (p.glu ? gelu_tanh_f(v[i]) : silu_f(v[i])) * u[i];
+          src.load(c + 1, w);
+          src.load(c + 1 + half / 32, u);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) w[i] = (p.glu ? gelu_tanh_f(w[i]) : silu_f(w[i])) * u[i];
+          src.store64(0, n_blk * half + 32 * c, v, w);
+        }
+        return;
+      }
+    }
     for (int c = g_lo; c < g_hi; ++c) {
       float u[32];
       src.load(c, v);
@@ -259,10 +346,10 @@ __device__ __forceinline__ void epilogue_row(const EpiParams& p, int m, int n_bl
         src.load(hh, v);
         if (!ok) continue;
         if (p.rope && region < 2) {
-          const float2* tab = p.rope_tab + static_cast<size_t>(pos) * 16;
+          const float2* tab = p.rope_tab + pos;
 #pragma unroll
           for (int i = 0; i < 16; ++i) {
-            const float2 cs = tab[i];
+            const float2 cs = tab[static_cast<size_t>(i) * p.rope_npos];
             const float a = v[i], c2 = v[i + 16];
             v[i] = a * cs.x - c2 * cs.y;
             v[i + 16] = c2 * cs.x + a * cs.y;
@@ -282,10 +369,10 @@ __device__ __forceinline__ void epilogue_row(const EpiParams& p, int m, int n_bl
         src.load(cb, w);
         if (!ok) continue;
         if (p.rope && region < 2) {
-          const float2* tab = p.rope_tab + static_cast<size_t>(pos) * (hd / 2) + 32 * j2;
+          const float2* tab = p.rope_tab + static_cast<size_t>(32 * j2) * p.rope_npos + pos;
 #pragma unroll
           for (int i = 0; i < 32; ++i) {
-            const float2 cs = tab[i];
+            const float2 cs = tab[static_cast<size_t>(i) * p.rope_npos];
             const float a = v[i], c2 = w[i];
             v[i] = a * cs.x - c2 * cs.y;
             w[i] = c2 * cs.x + a * cs.y;

@@ -10,6 +10,9 @@ namespace {
 constexpr int TM = 64, TN = 64, TK = 16;
 
 struct SmemSrc {
+  static constexpr bool kStaged = false;
+  __device__ bool staged() const { return false; }
+  __device__ void store64(int, int, const float (&)[32], const float (&)[32]) {}
   const float* row;  // accumulator row in shared memory
   __device__ __forceinline__ void load(int chunk, float (&v)[32]) {
 #pragma unroll

@@ -30,33 +30,104 @@ constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = 512;
 constexpr int EPI_WARPS = 8;
 constexpr int NUM_THREADS = 64 + 32 * EPI_WARPS;
-constexpr size_t SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 256;
+constexpr int STAGE_OUT_BYTES = 32 * 128;   // per epilogue warp: 32 rows x 64 bf16
+constexpr size_t SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + EPI_WARPS * STAGE_OUT_BYTES + 256;
 
+// Accumulator rows of one warp (32 TMEM lanes) plus, when bf16 outputs are
+// staged, the warp's 4 KB shared-memory box and the output tensor maps.
 struct TmemSrc {
+  static constexpr bool kStaged = true;
   uint32_t taddr;
+  uint8_t* stage;                      // 32 rows x 128 B, 128-byte swizzle; null: direct stores
+  const CUtensorMap* tm_out[2];
+  int row0;                            // first of the warp's 32 output rows
+  __device__ __forceinline__ bool staged() const { return stage != nullptr; }
+  __device__ __forceinline__ bool has_box() const { return stage != nullptr; }
+  // row `lane` of a 32 x 32 fp32 box (128-byte rows, 16-byte chunks XOR-swizzled by row)
+  __device__ __forceinline__ void put_row(const float (&v)[32]) {
+    const int lane = threadIdx.x & 31;
+    __syncwarp();
+    float4* row = reinterpret_cast<float4*>(stage + lane * 128);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) row[q ^ (lane & 7)] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+    __syncwarp();
+  }
+  // element (row i, column lane) of that box
+  __device__ __forceinline__ float get(int i) const {
+    const int lane = threadIdx.x & 31;
+    return reinterpret_cast<const float*>(stage + i * 128)[(((lane >> 2) ^ (i & 7)) << 2) | (lane & 3)];
+  }
   __device__ __forceinline__ void load(int chunk, float (&v)[32]) {
     __syncwarp();  // tcgen05.ld is warp-collective: reconverge after divergent stores
     tmem_ld32(taddr + 32 * chunk, v);
+  }
+  // bf16 of a[0..31] and b[0..31] (output columns x .. x+63 of this lane's row)
+  // into the box, then one TMA store of the warp's 32 x 64 block; rows and
+  // columns outside the output are clipped by the tensor map.
+  __device__ __forceinline__ void store64(int which, int x, const float (&a)[32], const float (&b)[32]) {
+    const int lane = threadIdx.x & 31;
+    if (lane == 0) bulk_wait_read0();   // the previous store has read the box
+    __syncwarp();
+    uint8_t* row = stage + lane * 128;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const float* src = q < 4 ? &a[8 * q] : &b[8 * (q - 4)];
+      __nv_bfloat162 t0 = __floats2bfloat162_rn(src[0], src[1]);
+      __nv_bfloat162 t1 = __floats2bfloat162_rn(src[2], src[3]);
+      __nv_bfloat162 t2 = __floats2bfloat162_rn(src[4], src[5]);
+      __nv_bfloat162 t3 = __floats2bfloat162_rn(src[6], src[7]);
+      *reinterpret_cast<uint4*>(row + ((q ^ (lane & 7)) << 4)) =
+          make_uint4(*reinterpret_cast<uint32_t*>(&t0), *reinterpret_cast<uint32_t*>(&t1),
+                     *reinterpret_cast<uint32_t*>(&t2), *reinterpret_cast<uint32_t*>(&t3));
+    }
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      tma_store_2d(tm_out[which], stage, x, row0);
+      bulk_commit();
+    }
   }
 };
 
 struct TcArgs {
   int M, N_acc, K;         // N_acc: accumulator columns in total (2F for GLU)
+  int staged;              // bf16 outputs go through the per-warp boxes and TMA stores
   int b_split;             // >0: B tile = 128 rows at n*128 and 128 rows at b_split + n*128
   int n_tiles_n;
   int* status;
   EpiParams ep;
 };
 
+// Tiles run N-fastest: the CTAs in flight share A tiles (activations, the
+// large operand) through L2, and every weight matrix of the model fits in L2.
+// At the start of a tile the producer asks L2 for the global rows its
+// epilogue will read (residual stream, h, gate), so the epilogue does not wait
+// on DRAM latency.
+template <int EPI>
+__device__ __forceinline__ void prefetch_epilogue_inputs(const TcArgs& a, int mb, int nb) {
+  const EpiParams& p = a.ep;
+  const float* src = nullptr;
+  int ld = 0;
+  if constexpr (EPI == EPI_RESID) { src = p.resid; ld = p.ldr; }
+  else if constexpr (EPI == EPI_FUSION2 || EPI == EPI_ADD || EPI == EPI_PA_UP) { src = p.base; ld = p.ldb; }
+  if (!src) return;
+  const int n0 = nb * BN, ncol = min(BN, p.N - n0);
+  if (ncol <= 0 || (ld & 3) || (n0 & 3)) return;
+  const uint32_t bytes = static_cast<uint32_t>(ncol) * 4u & ~15u;
+  for (int r = mb * BM; r < min(mb * BM + BM, p.M); ++r) prefetch_l2(src + static_cast<size_t>(r) * ld + n0, bytes);
+}
+
 template <int EPI>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmC2,
                    const TcArgs args) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + STAGES * A_BYTES;
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + STAGES * STAGE_BYTES);
+  uint8_t* sOut = smem + STAGES * STAGE_BYTES;          // EPI_WARPS boxes of 4 KB
+  uint64_t* full = reinterpret_cast<uint64_t*>(sOut + EPI_WARPS * STAGE_OUT_BYTES);
   uint64_t* empty = full + STAGES;
   uint64_t* tfull = empty + STAGES;
   uint64_t* tempty = tfull + 2;
@@ -101,7 +172,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       int issued[STAGES];
       for (int s = 0; s < STAGES; ++s) issued[s] = 0;
       for (int tile = blockIdx.x; tile < tiles && !*abort_flag; tile += gridDim.x) {
-        const int mb = tile % num_m, nb = tile / num_m;
+        const int nb = tile % args.n_tiles_n, mb = tile / args.n_tiles_n;
+        prefetch_epilogue_inputs<EPI>(args, mb, nb);
         bool ok = true;
         for (int kb = 0; kb < kblocks; ++kb) {
           if (!mbar_wait_bounded(&empty[stage], phase ^ 1, abort_flag, args.status)) { ok = false; break; }
@@ -171,13 +243,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
       if (!warp_wait_bounded(&tfull[acc], acc_phase, abort_flag, args.status)) break;
       tc_fence_after();
-      const int mb = tile % num_m, nb = tile / num_m;
-      TmemSrc src{tmem_base + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(quad * 32) << 16)};
+      const int nb = tile % args.n_tiles_n, mb = tile / args.n_tiles_n;
+      TmemSrc src{tmem_base + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(quad * 32) << 16),
+                  args.staged ? sOut + (warp - 2) * STAGE_OUT_BYTES : nullptr, {&tmC, &tmC2}, mb * BM + quad * 32};
       if (part < nsplit) epilogue_row<EPI>(args.ep, mb * BM + quad * 32 + lane, nb, BN, src, part, nsplit);
       tc_fence_before();
       mbar_arrive(&tempty[acc]);
       if (++acc == 2) { acc = 0; acc_phase ^= 1; }
     }
+    if (args.staged && lane == 0) bulk_wait0();   // every TMA store of this warp (if any) is complete
   }
 
   tc_fence_before();
@@ -222,8 +296,20 @@ bool make_map(CUtensorMap* m, const void* ptr, int64_t rows, int64_t cols, int64
   return r == CUDA_SUCCESS;
 }
 
+// 2-D bf16 output map over rows x cols (row stride ld), box 32 rows x 64, 128-byte swizzle.
+bool make_out_map(CUtensorMap* m, const void* ptr, int64_t rows, int64_t cols, int64_t ld) {
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld * 2)};
+  cuuint32_t box[2] = {64, 32};
+  cuuint32_t estr[2] = {1, 1};
+  return g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 template <int EPI>
-cudaError_t launch_epi(const CUtensorMap& ta, const CUtensorMap& tb, const TcArgs& a, int grid, cudaStream_t s) {
+cudaError_t launch_epi(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc, const CUtensorMap& tc2,
+                       const TcArgs& a, int grid, cudaStream_t s) {
   static bool attr_set = false;
   if (!attr_set) {
     cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -231,7 +317,7 @@ cudaError_t launch_epi(const CUtensorMap& ta, const CUtensorMap& tb, const TcArg
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  gemm_tc_kernel<EPI><<<grid, NUM_THREADS, SMEM_BYTES, s>>>(ta, tb, a);
+  gemm_tc_kernel<EPI><<<grid, NUM_THREADS, SMEM_BYTES, s>>>(ta, tb, tc, tc2, a);
   return cudaGetLastError();
 }
 
@@ -262,21 +348,35 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
   a.ep.M = g.M;
   a.ep.N = g.N;
   a.ep.n_tiles = a.n_tiles_n * (g.epi == EPI_LMHEAD ? 2 : 1);   // one partial per column half
+  // bf16 outputs of the plain, GLU and fusion-gate epilogues go out through TMA stores
+  CUtensorMap tc{}, tc2{};
+  a.staged = 0;
+  auto aligned = [](const void* p, int ld) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0 && ld % 8 == 0; };
+  if (g.epi == EPI_RESID || g.epi == EPI_FUSION2) {
+    a.staged = 1;   // the boxes serve as transpose scratch; no output map
+  } else if (g.ep.out_bf16 && (g.epi == EPI_STORE || g.epi == EPI_GLU)) {
+    if (aligned(g.ep.out, g.ep.ldo) && make_out_map(&tc, g.ep.out, g.M, g.N, g.ep.ldo)) a.staged = 1;
+  } else if (g.ep.out_bf16 && g.epi == EPI_FUSION1 && g.ep.d_split % 64 == 0) {
+    if (aligned(g.ep.out, g.ep.ldo) && aligned(g.ep.out2, g.ep.ldo2) &&
+        make_out_map(&tc, g.ep.out, g.M, g.ep.d_split, g.ep.ldo) &&
+        make_out_map(&tc2, g.ep.out2, g.M, g.N - g.ep.d_split, g.ep.ldo2))
+      a.staged = 1;
+  }
   const int tiles = ((g.M + BM - 1) / BM) * a.n_tiles_n;
   const int grid = tiles < g_num_sms ? tiles : g_num_sms;
   cudaError_t e;
   switch (g.epi) {
-    case EPI_STORE: e = launch_epi<EPI_STORE>(ta, tb, a, grid, s); break;
-    case EPI_RESID: e = launch_epi<EPI_RESID>(ta, tb, a, grid, s); break;
-    case EPI_QKV: e = launch_epi<EPI_QKV>(ta, tb, a, grid, s); break;
-    case EPI_GLU: e = launch_epi<EPI_GLU>(ta, tb, a, grid, s); break;
-    case EPI_FUSION1: e = launch_epi<EPI_FUSION1>(ta, tb, a, grid, s); break;
-    case EPI_FUSION2: e = launch_epi<EPI_FUSION2>(ta, tb, a, grid, s); break;
-    case EPI_LMHEAD: e = launch_epi<EPI_LMHEAD>(ta, tb, a, grid, s); break;
-    case EPI_PA_UP: e = launch_epi<EPI_PA_UP>(ta, tb, a, grid, s); break;
-    case EPI_SILU: e = launch_epi<EPI_SILU>(ta, tb, a, grid, s); break;
-    case EPI_ADD: e = launch_epi<EPI_ADD>(ta, tb, a, grid, s); break;
-    case EPI_PA_GATE: e = launch_epi<EPI_PA_GATE>(ta, tb, a, grid, s); break;
+    case EPI_STORE: e = launch_epi<EPI_STORE>(ta, tb, tc, tc2, a, grid, s); break;
+    case EPI_RESID: e = launch_epi<EPI_RESID>(ta, tb, tc, tc2, a, grid, s); break;
+    case EPI_QKV: e = launch_epi<EPI_QKV>(ta, tb, tc, tc2, a, grid, s); break;
+    case EPI_GLU: e = launch_epi<EPI_GLU>(ta, tb, tc, tc2, a, grid, s); break;
+    case EPI_FUSION1: e = launch_epi<EPI_FUSION1>(ta, tb, tc, tc2, a, grid, s); break;
+    case EPI_FUSION2: e = launch_epi<EPI_FUSION2>(ta, tb, tc, tc2, a, grid, s); break;
+    case EPI_LMHEAD: e = launch_epi<EPI_LMHEAD>(ta, tb, tc, tc2, a, grid, s); break;
+    case EPI_PA_UP: e = launch_epi<EPI_PA_UP>(ta, tb, tc, tc2, a, grid, s); break;
+    case EPI_SILU: e = launch_epi<EPI_SILU>(ta, tb, tc, tc2, a, grid, s); break;
+    case EPI_ADD: e = launch_epi<EPI_ADD>(ta, tb, tc, tc2, a, grid, s); break;
+    case EPI_PA_GATE: e = launch_epi<EPI_PA_GATE>(ta, tb, tc, tc2, a, grid, s); break;
     default: return "unknown epilogue";
   }
   return e == cudaSuccess ? nullptr : cudaGetErrorString(e);

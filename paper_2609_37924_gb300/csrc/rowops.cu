@@ -164,11 +164,11 @@ __global__ void sub_kernel(const float* __restrict__ a, const float* __restrict_
     o[i] = a[i] - b[i];
 }
 
-// tab[pos][j] = (cos, sin)(pos * theta^(-2j/hd)), angles evaluated in double
+// tab[j][pos] = (cos, sin)(pos * theta^(-2j/hd)), angles evaluated in double
 __global__ void rope_table_kernel(float2* tab, int n_pos, int half, int hd, double theta) {
   const size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x;
   if (i >= static_cast<size_t>(n_pos) * half) return;
-  const int pos = static_cast<int>(i / half), j = static_cast<int>(i % half);
+  const int j = static_cast<int>(i / n_pos), pos = static_cast<int>(i % n_pos);
   const double inv = pow(theta, -2.0 * j / hd);
   const double ang = static_cast<double>(pos) * inv;
   tab[i] = make_float2(static_cast<float>(cos(ang)), static_cast<float>(sin(ang)));

@@ -125,6 +125,7 @@ struct tadm_handle {
   // GEMM timing probe
   std::vector<cudaEvent_t> probe_ev;
   std::vector<double> probe_flops;
+  std::vector<int> probe_kind;
   int probe_next = 0;
 
   // sequence state
@@ -279,6 +280,7 @@ tadm_status gemm(tadm_handle* h, const void* A, int64_t a_rows, int lda, const v
   if (probe) {
     cudaEventRecord(h->probe_ev[2 * h->probe_next + 1], s);
     const double n_acc = epi == EPI_GLU ? 2.0 * N : static_cast<double>(N);
+    h->probe_kind[h->probe_next] = epi;
     h->probe_flops[h->probe_next++] = 2.0 * M * n_acc * K;
   }
   return TADM_OK;
@@ -311,6 +313,7 @@ tadm_status layer_fwd(tadm_handle* h, int li, float* x, int B, int R, int ctx, i
   ep.head_dim = hd;
   ep.rope = 1;
   ep.rope_tab = h->at<const float2>(h->off.rope);
+  ep.rope_npos = h->kv_stride + h->max_rows;
   TRYS(gemm(h, norm, Mmax, d, L.wqkv, d, M, nqkv, d, EPI_QKV, ep, s));
   AttnCall a{ep.q, ep.k, ep.v, h->at(h->off.attn), B, c.n_heads, c.n_kv_heads, hd, R, ctx, h->kv_stride, causal,
              h->act_bf16(), h->status()};
@@ -700,6 +703,28 @@ tadm_status tadm_probe_enable(tadm_handle* h, int max_launches) {
   for (auto& e : h->probe_ev)
     if (cudaEventCreate(&e) != cudaSuccess) return fail(h, TADM_ERR_CUDA, "cudaEventCreate failed");
   h->probe_flops.assign(max_launches, 0.0);
+  h->probe_kind.assign(max_launches, 0);
+  return TADM_OK;
+}
+
+tadm_status tadm_probe_breakdown(tadm_handle* h, int n_kinds, int64_t* launches, double* ms, double* flops) {
+  if (!h || n_kinds <= 0 || !launches || !ms || !flops) return TADM_ERR_INVALID_ARG;
+  for (int k = 0; k < n_kinds; ++k) {
+    launches[k] = 0;
+    ms[k] = flops[k] = 0.0;
+  }
+  if (h->probe_next > 0 && cudaEventSynchronize(h->probe_ev[2 * h->probe_next - 1]) != cudaSuccess)
+    return fail(h, TADM_ERR_CUDA, "probe event sync failed");
+  for (int i = 0; i < h->probe_next; ++i) {
+    const int k = h->probe_kind[i];
+    if (k < 0 || k >= n_kinds) continue;
+    float t = 0.0f;
+    if (cudaEventElapsedTime(&t, h->probe_ev[2 * i], h->probe_ev[2 * i + 1]) != cudaSuccess)
+      return fail(h, TADM_ERR_CUDA, "probe elapsed time failed");
+    launches[k] += 1;
+    ms[k] += t;
+    flops[k] += h->probe_flops[i];
+  }
   return TADM_OK;
 }
 

@@ -23,7 +23,7 @@ ABI_FUNCTIONS = [
     "tadm_prefill", "tadm_anchor_forward", "tadm_denoise_step", "tadm_commit_block", "tadm_generate",
     "tadm_sync_status", "tadm_get_counters", "tadm_plan", "tadm_layer_cost", "tadm_gemm", "tadm_confidence",
     "tadm_topk_unmask", "tadm_attention", "tadm_probe_enable", "tadm_probe_read", "tadm_head_scratch_size",
-    "tadm_head_confidence", "tadm_head_confidence_static",
+    "tadm_head_confidence", "tadm_head_confidence_static", "tadm_probe_breakdown",
 ]
 
 
@@ -96,6 +96,8 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "tadm_head_confidence": (I, [P, P, I, I, I, I, I, P, SZ, P, P, P]),
         "tadm_head_confidence_static": (I, [P, P, I, I, I, I, I, P, P, P]),
         "tadm_probe_enable": (I, [P, I]),
+        "tadm_probe_breakdown": (I, [P, I, ctypes.POINTER(I64), ctypes.POINTER(ctypes.c_double),
+                                     ctypes.POINTER(ctypes.c_double)]),
         "tadm_probe_read": (I, [P, ctypes.POINTER(I64), ctypes.POINTER(ctypes.c_double),
                                 ctypes.POINTER(ctypes.c_double)]),
     }
@@ -301,6 +303,16 @@ class TadmModel:
 
     def tadm_probe_enable(self, max_launches: int):
         _check(self.lib.tadm_probe_enable(self.h, max_launches), self.h)
+
+    EPI_NAMES = ["plain", "residual", "qkv_rope", "glu", "fusion_gate_hidden", "fusion_out", "output_head",
+                 "pa_up", "pa_silu", "pa_add", "pa_gate"]
+
+    def tadm_probe_breakdown(self) -> dict:
+        n = len(self.EPI_NAMES)
+        L, ms, fl = (ctypes.c_int64 * n)(), (ctypes.c_double * n)(), (ctypes.c_double * n)()
+        _check(self.lib.tadm_probe_breakdown(self.h, n, L, ms, fl), self.h)
+        return {self.EPI_NAMES[k]: {"launches": L[k], "ms": ms[k], "tflops": fl[k] / (ms[k] / 1e3) / 1e12}
+                for k in range(n) if L[k] > 0}
 
     def tadm_probe_read(self):
         n, ms, fl = ctypes.c_int64(), ctypes.c_double(), ctypes.c_double()
