@@ -45,6 +45,9 @@ def parse():
     ap.add_argument("--T", type=int, default=None,
                     help="override reverse steps per block (short runs for launch-list profiles)")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
+    ap.add_argument("--sweep-workloads", default=None,
+                    help="comma list of workloads: print one JSON line per (workload, batch, K) instead")
+    ap.add_argument("--sweep-batches", default="", help="batches for the 'sweep' workload (default 1,8,32,128)")
     ap.add_argument("--kernel-bench", default=None,
                     help="time one building block alone instead, e.g. gemm:16384,32768,768")
     return ap.parse_args()
@@ -370,8 +373,63 @@ def kernel_bench(args):
     print(json.dumps({"kernel": kind, "shape": shape, "ms": ms, "tflops": flops / (ms / 1000.0) / 1e12}), flush=True)
 
 
+def workload_sweep(args):
+    """Generated tokens/s of each workload for every K of its sweep (one line each)."""
+    import torch
+
+    import workloads as wl
+    from paper_2609_37924_gb300 import TadmModel, upload_weights
+
+    torch.cuda.set_device(0)
+    for name in args.sweep_workloads.split(","):
+        base = wl.get_workload(name)
+        batches = [base.batch]
+        if name == "sweep":
+            batches = [int(b) for b in (args.sweep_batches or "1,8,32,128").split(",")]
+        m = base.model
+        t0 = time.perf_counter()
+        dev_w = upload_weights(m, wl.make_weights(m, seed=base.seed))
+        t_w = time.perf_counter() - t0
+        for B in batches:
+            w = wl.get_workload(name, batch=B)
+            bl = w.block_len
+            tm = TadmModel(m, dev_w, max_batch=B, max_rows=max(w.prompt_len, bl) if bl else w.total_len,
+                           max_ctx=w.total_len if bl else 0)
+            p = torch.from_numpy(wl.make_prompts(w)).cuda()
+            out = torch.empty((B, w.total_len), dtype=torch.int32, device="cuda")
+            res = {}
+            for K in (w.k_sweep or (w.K,)):
+                for _ in range(max(1, args.warmup)):
+                    tm.tadm_generate(p, out, w.gen_len, w.steps_per_block, K, bl)
+                tm.tadm_sync_status()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                torch.cuda.synchronize()
+                e0.record()
+                for _ in range(args.steps):
+                    tm.tadm_generate(p, out, w.gen_len, w.steps_per_block, K, bl)
+                e1.record()
+                tm.tadm_sync_status()
+                ms = e0.elapsed_time(e1) / args.steps
+                c = tm.tadm_get_counters()
+                res[K] = B * w.gen_len / (ms / 1000.0)
+                print(json.dumps({"workload": name, "batch": B, "K": K, "tokens_per_s": res[K], "ms_per_generation": ms,
+                                  "vs_K1": res[K] / res[1] if 1 in res else None, "anchor_calls": c["anchor_calls"],
+                                  "denoise_steps": c["denoise_steps"], "commit_passes": c["commit_passes"],
+                                  "gpu_launches": c["kernel_launches"], "weights_s": round(t_w, 1)}), flush=True)
+            tm.close()
+            del tm
+            torch.cuda.empty_cache()
+        del dev_w
+        torch.cuda.empty_cache()
+
+
 def main():
     args = parse()
+    if args.sweep_workloads:
+        import __graft_entry__
+        __graft_entry__.build()
+        workload_sweep(args)
+        return
     if args.kernel_bench:
         import __graft_entry__
         __graft_entry__.build()

@@ -56,3 +56,71 @@ def test_small_workload_sampled_sequence(request):
     agree = float(np.mean(gt[masked] == ref["tok"][0][masked]))
     assert agree >= 0.95, agree
     print(f"[fullsize small] logits rel-L2 {rel:.3e}, argmax agreement {agree:.4f}, committed 6/6")
+
+
+def _block_case(m, B, P, bl, seed, T=16):
+    """GPU: prefill, refresh + one stale step on block 0; oracle: the last sequence."""
+    import __graft_entry__ as g
+    g.build()
+    from paper_2609_37924_gb300 import TadmModel, upload_weights
+    w = wl.Workload("fullsize", m, batch=B, prompt_len=P, gen_len=4 * bl, steps_per_block=T, K=4, block_len=bl,
+                    seed=seed)
+    host = wl.make_weights(m, seed=seed)
+    tm = TadmModel(m, upload_weights(m, host), max_batch=B, max_rows=max(P, bl), max_ctx=P + 4 * bl)
+    prompts = wl.make_prompts(w)
+    z0 = np.full((B, bl), m.mask_id, np.int32)
+    z1 = wl.random_canvas(w, B, bl, 0.6, seed=seed + 1)
+    tm.tadm_reset(B)
+    tm.tadm_prefill(torch.from_numpy(prompts).cuda())
+    cache = tm.new_cache(B, bl)
+    tm.tadm_anchor_forward(torch.from_numpy(z0).cuda(), T, cache)
+    zt = torch.from_numpy(z1).cuda()
+    logits = torch.empty((B * bl, m.vocab), dtype=torch.float32, device="cuda")
+    conf = torch.empty(B * bl, dtype=torch.float32, device="cuda")
+    tok = torch.empty(B * bl, dtype=torch.int32, device="cuda")
+    tm.tadm_denoise_step(zt, T - 1, T, bl, cache, logits=logits, conf=conf, tok=tok)
+    tm.tadm_sync_status()
+    b = B - 1
+    gl = logits[b * bl:(b + 1) * bl].cpu().numpy().astype(np.float64)
+    gt = tok.cpu().numpy().reshape(B, bl)[b]
+    gz = zt.cpu().numpy()[b]
+    del tm, logits
+    torch.cuda.empty_cache()
+    o = O.Oracle(m, host)
+    sess = o.new_session(1)
+    o.prefill(sess, prompts[b:b + 1])
+    cache_o = o.anchor_forward(sess, z0[b:b + 1])
+    ref = o.denoise_step(sess, z1[b:b + 1], cache_o, 1, T, bl)
+    rel = np.linalg.norm(gl - ref["logits"][0]) / np.linalg.norm(ref["logits"][0])
+    masked = z1[b] == m.mask_id
+    committed = masked & (gz != m.mask_id)
+    agree = float(np.mean(gt[masked] == ref["tok"][0][masked]))
+    return rel, agree, committed, gz, ref
+
+
+def test_block_workload_full_size_sampled_sequence():
+    """'block' workload dims and launch configuration: batch 32, d_model 2048,
+    16 + 6 layers, GQA 16/8 heads of 128, vocab 128000, 512-token causal
+    prefill, blocks of 32."""
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    w = wl.WORKLOADS["block"]
+    rel, agree, committed, gz, ref = _block_case(w.model, w.batch, w.prompt_len, w.block_len, seed=w.seed)
+    assert rel < 2e-2, rel
+    assert np.array_equal(gz[committed], ref["tok"][0][committed])
+    assert agree >= 0.9, agree
+    print(f"[fullsize block] logits rel-L2 {rel:.3e}, argmax agreement {agree:.4f}, committed {committed.sum()}")
+
+
+def test_posttrain_full_width_reduced_depth():
+    """'posttrain' widths (d_model 5376, 32/16 heads of 128, FFN 21504 GeGLU,
+    vocab 262144, tied head, paired-attention fusion r = 256) with 1 + 2 + 1
+    layers and a 64-token prompt, batch 8."""
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    m = wl.get_workload("posttrain", model_n_shared=1, model_n_anchor=2, model_n_denoise=1).model
+    rel, agree, committed, gz, ref = _block_case(m, 8, 64, 32, seed=3, T=32)
+    assert rel < 2e-2, rel
+    assert np.array_equal(gz[committed], ref["tok"][0][committed])
+    assert agree >= 0.9, agree
+    print(f"[fullsize posttrain] logits rel-L2 {rel:.3e}, argmax agreement {agree:.4f}, committed {committed.sum()}")

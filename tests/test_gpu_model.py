@@ -279,3 +279,31 @@ def test_invalid_calls_return_errors(T):
         tm.tadm_prefill(z[:2, :8])                              # no KV context configured
     with pytest.raises(T.TadmError):
         tm.tadm_generate(z[:2, :8], torch.empty((2, 70), dtype=torch.int32, device="cuda"), 62, 4, 1, block_len=31)
+
+
+def test_block_mode_fp32_positions_and_context_exact(T):
+    """The fp32 path shares all of block mode's host logic (positions, KV
+    context, prefill / commit passes) and computes in fp32: it must match the
+    oracle to 1e-4 through prefill, two blocks and a commit."""
+    m = wl.ModelConfig(vocab=512, d_model=256, n_heads=4, n_kv_heads=2, head_dim=64, ffn=512, n_anchor=2,
+                       n_denoise=2, dtype="f32")
+    B, P, bl = 2, 40, 32
+    w = wl.Workload("t", m, batch=B, prompt_len=P, gen_len=64, steps_per_block=4, K=2, block_len=bl)
+    tm, o = setup(T, m, B, max(P, bl), max_ctx=P + 64)
+    prompts = wl.make_prompts(w, batch=B, seed=13)
+    tm.tadm_reset(B)
+    tm.tadm_prefill(torch.from_numpy(prompts).cuda())
+    sess = o.new_session(B)
+    o.prefill(sess, prompts)
+    cache = tm.new_cache(B, bl)
+    for blk in range(2):
+        zb = wl.random_canvas(w, B, bl, 0.7, seed=20 + blk)
+        tm.tadm_anchor_forward(torch.from_numpy(zb).cuda(), 4, cache)
+        cache_o = o.anchor_forward(sess, zb)
+        g = gpu_step(tm, zb, 4, 4, bl, cache)
+        ref = o.denoise_step(sess, zb, cache_o, 0, 4, bl)
+        assert rel_l2(g["logits"], ref["logits"]) < 1e-4
+        assert np.array_equal(g["z"], ref["z"])
+        tm.tadm_commit_block(torch.from_numpy(g["z"]).cuda())
+        o.commit_block(sess, g["z"])
+    tm.tadm_sync_status()
