@@ -44,6 +44,7 @@ def parse():
     ap.add_argument("--cpu-sample-seconds", type=float, default=20.0)
     ap.add_argument("--T", type=int, default=None,
                     help="override reverse steps per block (short runs for launch-list profiles)")
+    ap.add_argument("--G", type=int, default=None, help="override the generation length (short profiling runs)")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
     ap.add_argument("--sweep-workloads", default=None,
                     help="comma list of workloads: print one JSON line per (workload, batch, K) instead")
@@ -212,6 +213,8 @@ def gpu_arm(args):
         over["batch"] = args.batch
     if args.T:
         over["steps_per_block"] = args.T
+    if args.G:
+        over["gen_len"] = args.G
     w = wl.get_workload(args.workload, **over)
     K = args.K or w.K
     m = w.model

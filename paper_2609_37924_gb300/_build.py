@@ -9,7 +9,7 @@ PKG = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(PKG, "csrc")
 LIBDIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(LIBDIR, "libtadm.so")
-SOURCES = ["gemm_tc.cu", "gemm_simt.cu", "attention.cu", "rowops.cu", "sampler.cu", "tadm_api.cu", "head_static.cu"]
+SOURCES = ["gemm_tc.cu", "gemm_simt.cu", "attention.cu", "rowops.cu", "sampler.cu", "tadm_api.cu", "head_static.cu", "splitk.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden"]
 

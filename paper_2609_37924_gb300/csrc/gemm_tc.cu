@@ -15,6 +15,7 @@
 // raises a shared abort flag and the device status word, and the CTA drains
 // its in-flight copies and MMAs, frees TMEM and exits.
 #include <cudaTypedefs.h>
+#include <algorithm>
 #include <mutex>
 
 #include "epilogue.cuh"
@@ -91,6 +92,10 @@ struct TmemSrc {
 
 struct TcArgs {
   int M, N_acc, K;         // N_acc: accumulator columns in total (2F for GLU)
+  int splits, kb_per_split;  // split-K: unit = (tile, K slice); partials [split][M][ldp] fp32
+  float* part;
+  size_t part_stride;
+  int ldp;
   int staged;              // bf16 outputs go through the per-warp boxes and TMA stores
   int b_split;             // >0: B tile = 128 rows at n*128 and 128 rows at b_split + n*128
   int n_tiles_n;
@@ -162,6 +167,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
   const int num_m = (args.M + BM - 1) / BM;
   const int tiles = num_m * args.n_tiles_n;
+  const int units = tiles * args.splits;
   const int kblocks = (args.K + BK - 1) / BK;
 
   if (warp == 0) {
@@ -171,11 +177,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       uint32_t phase = 0;
       int issued[STAGES];
       for (int s = 0; s < STAGES; ++s) issued[s] = 0;
-      for (int tile = blockIdx.x; tile < tiles && !*abort_flag; tile += gridDim.x) {
+      for (int unit = blockIdx.x; unit < units && !*abort_flag; unit += gridDim.x) {
+        const int tile = unit / args.splits, ks = unit % args.splits;
         const int nb = tile % args.n_tiles_n, mb = tile / args.n_tiles_n;
-        prefetch_epilogue_inputs<EPI>(args, mb, nb);
+        const int kb0 = ks * args.kb_per_split, kb1 = min(kblocks, kb0 + args.kb_per_split);
+        if (args.splits == 1) prefetch_epilogue_inputs<EPI>(args, mb, nb);
         bool ok = true;
-        for (int kb = 0; kb < kblocks; ++kb) {
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait_bounded(&empty[stage], phase ^ 1, abort_flag, args.status)) { ok = false; break; }
           mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
           tma_load_2d(sA + stage * A_BYTES, &tmA, &full[stage], kb * BK, mb * BM);
@@ -206,12 +214,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
       uint32_t phase = 0;
       int acc = 0;
       uint32_t acc_phase = 0;
-      for (int tile = blockIdx.x; tile < tiles && !*abort_flag; tile += gridDim.x) {
+      for (int unit = blockIdx.x; unit < units && !*abort_flag; unit += gridDim.x) {
+        const int ks = unit % args.splits;
+        const int kb0 = ks * args.kb_per_split, kb1 = min(kblocks, kb0 + args.kb_per_split);
         if (!mbar_wait_bounded(&tempty[acc], acc_phase ^ 1, abort_flag, args.status)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * BN;
         bool ok = true;
-        for (int kb = 0; kb < kblocks; ++kb) {
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait_bounded(&full[stage], phase, abort_flag, args.status)) { ok = false; break; }
           tc_fence_after();
           const uint32_t a0 = smem_u32(sA + stage * A_BYTES);
@@ -219,7 +229,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k) {
             umma_bf16(d_tmem, sdesc_kmajor_sw128(a0 + 32 * k), sdesc_kmajor_sw128(b0 + 32 * k), idesc,
-                      (kb | k) != 0);
+                      (kb != kb0) || (k != 0));
           }
           umma_commit(&empty[stage]);
           if (++stage == STAGES) { stage = 0; phase ^= 1; }
@@ -240,13 +250,25 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     constexpr int nsplit = EPI == EPI_PA_GATE ? 1 : 2;
     int acc = 0;
     uint32_t acc_phase = 0;
-    for (int tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
+    for (int unit = blockIdx.x; unit < units; unit += gridDim.x) {
       if (!warp_wait_bounded(&tfull[acc], acc_phase, abort_flag, args.status)) break;
       tc_fence_after();
+      const int tile = unit / args.splits, ks = unit % args.splits;
       const int nb = tile % args.n_tiles_n, mb = tile / args.n_tiles_n;
       TmemSrc src{tmem_base + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(quad * 32) << 16),
                   args.staged ? sOut + (warp - 2) * STAGE_OUT_BYTES : nullptr, {&tmC, &tmC2}, mb * BM + quad * 32};
-      if (part < nsplit) epilogue_row<EPI>(args.ep, mb * BM + quad * 32 + lane, nb, BN, src, part, nsplit);
+      const int m = mb * BM + quad * 32 + lane;
+      if (args.splits > 1) {
+        // raw fp32 partial of this K slice, tile-local column order
+        float v[32];
+        float* dst = args.part + ks * args.part_stride + static_cast<size_t>(m) * args.ldp + nb * BN;
+        for (int c = part * (BN / 64); c < (part + 1) * (BN / 64); ++c) {
+          src.load(c, v);
+          if (m < args.M) store32(dst, 0, 32 * c, v, 32);
+        }
+      } else if (part < nsplit) {
+        epilogue_row<EPI>(args.ep, m, nb, BN, src, part, nsplit);
+      }
       tc_fence_before();
       mbar_arrive(&tempty[acc]);
       if (++acc == 2) { acc = 0; acc_phase ^= 1; }
@@ -363,7 +385,26 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
       a.staged = 1;
   }
   const int tiles = ((g.M + BM - 1) / BM) * a.n_tiles_n;
-  const int grid = tiles < g_num_sms ? tiles : g_num_sms;
+  // split-K when the tiles cannot fill the SMs and K is long: fixed-order
+  // reduction afterwards, so results do not depend on the split
+  const int kblocks = (g.K + BK - 1) / BK;
+  a.splits = 1;
+  a.kb_per_split = kblocks;
+  a.ldp = a.n_tiles_n * BN;
+  if (g.split_buf && tiles * 3 < g_num_sms * 2 && kblocks >= 8) {
+    int sp = std::min(std::min(g_num_sms / tiles, kblocks / 4), 16);
+    const size_t per = static_cast<size_t>(g.M) * a.ldp * sizeof(float);
+    while (sp > 1 && sp * per > g.split_bytes) --sp;
+    if (sp > 1) {
+      a.kb_per_split = (kblocks + sp - 1) / sp;
+      a.splits = (kblocks + a.kb_per_split - 1) / a.kb_per_split;
+      a.part = g.split_buf;
+      a.part_stride = static_cast<size_t>(g.M) * a.ldp;
+      a.staged = 0;
+    }
+  }
+  const int units = tiles * a.splits;
+  const int grid = units < g_num_sms ? units : g_num_sms;
   cudaError_t e;
   switch (g.epi) {
     case EPI_STORE: e = launch_epi<EPI_STORE>(ta, tb, tc, tc2, a, grid, s); break;
@@ -379,7 +420,19 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
     case EPI_PA_GATE: e = launch_epi<EPI_PA_GATE>(ta, tb, tc, tc2, a, grid, s); break;
     default: return "unknown epilogue";
   }
-  return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
+  if (e != cudaSuccess) return cudaGetErrorString(e);
+  const_cast<GemmCall&>(g).launched = 1;
+  if (a.splits > 1) {
+    const char* r = splitk_reduce(g.epi, a.ep, a.part, a.part_stride, a.ldp, a.splits, a.n_tiles_n, s);
+    if (r) return r;
+    const_cast<GemmCall&>(g).launched = 3;
+  }
+  return nullptr;
+}
+
+size_t gemm_tc_split_bytes() {
+  get_encoder();
+  return static_cast<size_t>(g_num_sms > 0 ? g_num_sms : 160) * BM * BN * sizeof(float);
 }
 
 int gemm_tc_tiles_n(int N, int epi) {

@@ -16,11 +16,20 @@ struct GemmCall {
   int epi;
   EpiParams ep;
   int* status;
+  float* split_buf;      // fp32 partials for split-K (null: no split)
+  size_t split_bytes;
+  int launched;          // out: kernels launched
 };
+
+// Split-K partial buffer that covers every GEMM (units x 128 x 256 fp32 for at most one unit per SM).
+size_t gemm_tc_split_bytes();
 
 // tcgen05 path (bf16 operands)
 const char* gemm_tc(const GemmCall& g, cudaStream_t s);
 int gemm_tc_tiles_n(int N, int epi);
+// fixed-order sum of split-K partials followed by the GEMM's epilogue
+const char* splitk_reduce(int epi, const EpiParams& ep, const float* part, size_t part_stride, int ldp, int splits,
+                          int n_tiles_n, cudaStream_t s);
 // CUDA-core path (fp32 operands)
 const char* gemm_simt(const GemmCall& g, cudaStream_t s);
 int gemm_simt_tiles_n(int N, int epi);

@@ -50,6 +50,36 @@ __global__ void embed_kernel(const int32_t* __restrict__ z, int ldz, int rows, i
   }
 }
 
+// out = x / sqrt(mean(x^2) + eps) * gain, one 256-thread block per row (few rows)
+template <class T>
+__global__ void __launch_bounds__(256) rmsnorm_block_kernel(const float* __restrict__ x, int d,
+                                                            const void* __restrict__ gain, int w_bf16, float eps,
+                                                            void* __restrict__ out, int ldo) {
+  __shared__ float red[8];
+  const int m = blockIdx.x;
+  const float* xr = x + static_cast<size_t>(m) * d;
+  float ss = 0.0f;
+  for (int j = threadIdx.x * 4; j < d; j += 1024) {
+    const float4 v = *reinterpret_cast<const float4*>(xr + j);
+    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+  }
+  ss = warp_sum(ss);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  float tot = 0.0f;
+#pragma unroll
+  for (int w = 0; w < 8; ++w) tot += red[w];
+  const float inv = rsqrtf(tot / static_cast<float>(d) + eps);
+  for (int j = threadIdx.x * 4; j < d; j += 1024) {
+    const float4 v = *reinterpret_cast<const float4*>(xr + j);
+    const size_t o = static_cast<size_t>(m) * ldo + j;
+    store_act<T>(out, o + 0, v.x * inv * ldw(gain, w_bf16, j + 0));
+    store_act<T>(out, o + 1, v.y * inv * ldw(gain, w_bf16, j + 1));
+    store_act<T>(out, o + 2, v.z * inv * ldw(gain, w_bf16, j + 2));
+    store_act<T>(out, o + 3, v.w * inv * ldw(gain, w_bf16, j + 3));
+  }
+}
+
 // out = x / sqrt(mean(x^2) + eps) * gain
 template <class T>
 __global__ void rmsnorm_kernel(const float* __restrict__ x, int M, int d, const void* __restrict__ gain, int w_bf16,
@@ -208,6 +238,13 @@ const char* embed_rows(const int32_t* z, int ldz, int batch, int rows, const voi
 const char* rmsnorm_rows(const float* x, int M, int d, const void* gain, int w_bf16, float eps, void* out, int ldo,
                          int act_bf16, cudaStream_t s) {
   if (M <= 0) return nullptr;
+  if (M < 1024) {   // few rows: a block per row keeps enough SMs busy
+    if (act_bf16)
+      rmsnorm_block_kernel<bf16><<<M, 256, 0, s>>>(x, d, gain, w_bf16, eps, out, ldo);
+    else
+      rmsnorm_block_kernel<float><<<M, 256, 0, s>>>(x, d, gain, w_bf16, eps, out, ldo);
+    return err();
+  }
   if (act_bf16)
     rmsnorm_kernel<bf16><<<rows_grid(M), WPB * 32, 0, s>>>(x, M, d, gain, w_bf16, eps, out, ldo);
   else

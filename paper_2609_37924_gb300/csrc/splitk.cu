@@ -1,0 +1,100 @@
+// Split-K reduction for the tcgen05 GEMM: sums the fp32 partials of the K
+// slices in slice order (deterministic) into slice 0, then runs the GEMM's own
+// epilogue on that sum, one thread per (output row, column group) of a
+// 256-column tile.
+#include "kernels.h"
+
+namespace tadm {
+namespace {
+
+struct PartSrc {
+  static constexpr bool kStaged = false;
+  const float* row;      // partial row of slice 0 at this tile's first column
+  size_t stride;         // between slices
+  int splits;
+  __device__ __forceinline__ void load(int chunk, float (&v)[32]) {
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = 0.0f;
+    for (int ks = 0; ks < splits; ++ks) {
+      const float4* p = reinterpret_cast<const float4*>(row + ks * stride + 32 * chunk);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const float4 t = p[q];
+        v[4 * q] += t.x; v[4 * q + 1] += t.y; v[4 * q + 2] += t.z; v[4 * q + 3] += t.w;
+      }
+    }
+  }
+};
+
+// Column groups one thread may take without changing the epilogue's result:
+// the output head keeps the tensor-core path's two partials per tile, the
+// paired-attention gate needs whole rows, GLU pairs gate / up chunks, QKV
+// whole heads; the rest is independent per 32-column chunk.
+template <int EPI>
+__device__ __forceinline__ int reduce_groups(const EpiParams& ep) {
+  if constexpr (EPI == EPI_PA_GATE) return 1;
+  else if constexpr (EPI == EPI_LMHEAD) return 2;
+  else if constexpr (EPI == EPI_GLU) return 4;
+  else if constexpr (EPI == EPI_QKV) return 256 / ep.head_dim;
+  else return 8;
+}
+
+// block: 32 rows x 8 group slots; thread (row, slot) runs group `slot` if it exists
+template <int EPI>
+__global__ void __launch_bounds__(256) splitk_reduce_kernel(EpiParams ep, const float* __restrict__ part,
+                                                            size_t stride, int ldp, int splits) {
+  const int m = blockIdx.x * 32 + (threadIdx.x & 31), slot = threadIdx.x >> 5, nb = blockIdx.y;
+  const int groups = reduce_groups<EPI>(ep);
+  if (m >= ep.M || slot >= groups) return;
+  PartSrc src{part + static_cast<size_t>(m) * ldp + nb * 256, stride, splits};
+  epilogue_row<EPI>(ep, m, nb, 256, src, slot, groups);
+}
+
+// Phase 1: slice 0 <- sum of all slices in slice order, one float4 per thread.
+__global__ void __launch_bounds__(256) splitk_sum_kernel(float* __restrict__ part, size_t stride, size_t n4,
+                                                         int splits) {
+  const size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x;
+  if (i >= n4) return;
+  float4* p = reinterpret_cast<float4*>(part);
+  float4 a = p[i];
+  for (int ks = 1; ks < splits; ++ks) {
+    const float4 t = p[i + ks * (stride / 4)];
+    a.x += t.x; a.y += t.y; a.z += t.z; a.w += t.w;
+  }
+  p[i] = a;
+}
+
+// Phase 2: the epilogue on slice 0.
+template <int EPI>
+cudaError_t launch(const EpiParams& ep, const float* part, size_t stride, int ldp, int splits, int n_tiles_n,
+                   cudaStream_t s) {
+  const size_t n4 = static_cast<size_t>(ep.M) * ldp / 4;
+  splitk_sum_kernel<<<static_cast<unsigned>((n4 + 255) / 256), 256, 0, s>>>(const_cast<float*>(part), stride, n4,
+                                                                            splits);
+  dim3 grid((ep.M + 31) / 32, n_tiles_n);
+  splitk_reduce_kernel<EPI><<<grid, 256, 0, s>>>(ep, part, stride, ldp, 1);
+  return cudaGetLastError();
+}
+}  // namespace
+
+const char* splitk_reduce(int epi, const EpiParams& ep, const float* part, size_t stride, int ldp, int splits,
+                          int n_tiles_n, cudaStream_t s) {
+  cudaError_t e;
+  switch (epi) {
+    case EPI_STORE: e = launch<EPI_STORE>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
+    case EPI_RESID: e = launch<EPI_RESID>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
+    case EPI_QKV: e = launch<EPI_QKV>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
+    case EPI_GLU: e = launch<EPI_GLU>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
+    case EPI_FUSION1: e = launch<EPI_FUSION1>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
+    case EPI_FUSION2: e = launch<EPI_FUSION2>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
+    case EPI_LMHEAD: e = launch<EPI_LMHEAD>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
+    case EPI_PA_UP: e = launch<EPI_PA_UP>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
+    case EPI_SILU: e = launch<EPI_SILU>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
+    case EPI_ADD: e = launch<EPI_ADD>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
+    case EPI_PA_GATE: e = launch<EPI_PA_GATE>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
+    default: return "unknown epilogue";
+  }
+  return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
+}
+
+}  // namespace tadm

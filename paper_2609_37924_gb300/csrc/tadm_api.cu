@@ -116,7 +116,7 @@ struct tadm_handle {
   char* ws = nullptr;
   size_t ws_bytes = 0, ws_need = 0;
   struct Off {
-    size_t status, rope, c, x, h_int, norm, qbuf, kv, attn, glu, f_g, f_hid, f_pre, part, conf, tok;
+    size_t status, rope, c, x, h_int, norm, qbuf, kv, attn, glu, f_g, f_hid, f_pre, part, conf, tok, split;
     size_t pa_z, pa_j, pa_mq, pa_mk, pa_mv, pa_mo, pa_r, pa_rb, pa_hid, pa_phi, pa_m, pa_dz, pa_f, pa_g, pa_mb;
   } off{};
   size_t kv_slab = 0;
@@ -250,6 +250,7 @@ void layout(tadm_handle* h) {
     f.pa_mb = take(M * r * es);
   }
   f.part = take(M * h->n_part_tiles * 3 * 4);
+  f.split = c.dtype ? take(gemm_tc_split_bytes()) : take(0);
   f.conf = take(M * 4);
   f.tok = take(M * 4);
   h->ws_need = o;
@@ -270,13 +271,17 @@ tadm_status gemm(tadm_handle* h, const void* A, int64_t a_rows, int lda, const v
   g.epi = epi;
   g.ep = ep;
   g.status = h->status();
+  if (h->cfg.dtype) {
+    g.split_buf = h->at<float>(h->off.split);
+    g.split_bytes = gemm_tc_split_bytes();
+  }
   g.ep.out_bf16 = out_f32 ? 0 : h->act_bf16();
   g.ep.bias_bf16 = h->cfg.dtype;
   const bool probe = h->probe_next < static_cast<int>(h->probe_flops.size());
   if (probe) cudaEventRecord(h->probe_ev[2 * h->probe_next], s);
   const char* e = h->cfg.dtype ? gemm_tc(g, s) : gemm_simt(g, s);
   if (e) return fail(h, TADM_ERR_CUDA, "GEMM (M=%d N=%d K=%d epi=%d): %s", M, N, K, epi, e);
-  h->counters.kernel_launches += 1;
+  h->counters.kernel_launches += h->cfg.dtype ? g.launched : 1;
   if (probe) {
     cudaEventRecord(h->probe_ev[2 * h->probe_next + 1], s);
     const double n_acc = epi == EPI_GLU ? 2.0 * N : static_cast<double>(N);
