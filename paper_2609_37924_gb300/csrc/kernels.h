@@ -48,7 +48,11 @@ const char* attention(const AttnCall& a, cudaStream_t s);
 const char* embed_rows(const int32_t* z, int ldz, int batch, int rows, const void* E, int e_bf16, int d,
                        int vocab, float* out, float* out2, cudaStream_t s);
 const char* rmsnorm_rows(const float* x, int M, int d, const void* gain, int w_bf16, float eps, void* out,
-                         int ldo, int act_bf16, cudaStream_t s);
+                         int ldo, int act_bf16, cudaStream_t s, const int32_t* rows_idx = nullptr);
+// per sequence: the rows still holding MASK (first `per_seq` of them, in order) -> idx[b * per_seq + j]
+// (global row b * rows + r); conf of every row set to -inf so that rows left out are never selected
+const char* masked_rows(const int32_t* z, int ldz, int batch, int rows, int mask_id, int per_seq, int32_t* idx,
+                        float* conf, cudaStream_t s);
 const char* ln_pair_rows(const float* c, const float* h, int M, int d, const void* wc, const void* bc,
                          const void* wh, const void* bh, int w_bf16, float eps, void* u, int act_bf16,
                          cudaStream_t s);
@@ -69,7 +73,7 @@ const char* copy_rows_i32(const int32_t* src, int lds, int32_t* dst, int ldd, in
 const char* confidence_rows(const float* logits, int rows, int vocab, int ld, int mask_id, float* conf,
                             int32_t* tok, cudaStream_t s);
 const char* combine_partials(const float* part, int rows, int n_tiles, float* conf, int32_t* tok,
-                             cudaStream_t s);
+                             cudaStream_t s, const int32_t* rows_idx = nullptr);
 const char* topk_unmask(int32_t* z, int ldz, const float* conf, const int32_t* tok, int batch, int rows, int k,
                         int mask_id, int32_t* selected, cudaStream_t s);
 

@@ -54,10 +54,11 @@ __global__ void embed_kernel(const int32_t* __restrict__ z, int ldz, int rows, i
 template <class T>
 __global__ void __launch_bounds__(256) rmsnorm_block_kernel(const float* __restrict__ x, int d,
                                                             const void* __restrict__ gain, int w_bf16, float eps,
-                                                            void* __restrict__ out, int ldo) {
+                                                            void* __restrict__ out, int ldo,
+                                                            const int32_t* __restrict__ rows_idx) {
   __shared__ float red[8];
   const int m = blockIdx.x;
-  const float* xr = x + static_cast<size_t>(m) * d;
+  const float* xr = x + static_cast<size_t>(rows_idx ? rows_idx[m] : m) * d;
   float ss = 0.0f;
   for (int j = threadIdx.x * 4; j < d; j += 1024) {
     const float4 v = *reinterpret_cast<const float4*>(xr + j);
@@ -83,10 +84,10 @@ __global__ void __launch_bounds__(256) rmsnorm_block_kernel(const float* __restr
 // out = x / sqrt(mean(x^2) + eps) * gain
 template <class T>
 __global__ void rmsnorm_kernel(const float* __restrict__ x, int M, int d, const void* __restrict__ gain, int w_bf16,
-                               float eps, void* __restrict__ out, int ldo) {
+                               float eps, void* __restrict__ out, int ldo, const int32_t* __restrict__ rows_idx) {
   const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (m >= M) return;
-  const float* xr = x + static_cast<size_t>(m) * d;
+  const float* xr = x + static_cast<size_t>(rows_idx ? rows_idx[m] : m) * d;
   float ss = 0.0f;
   for (int j = lane * 4; j < d; j += 128) {
     const float4 v = *reinterpret_cast<const float4*>(xr + j);
@@ -236,19 +237,19 @@ const char* embed_rows(const int32_t* z, int ldz, int batch, int rows, const voi
 }
 
 const char* rmsnorm_rows(const float* x, int M, int d, const void* gain, int w_bf16, float eps, void* out, int ldo,
-                         int act_bf16, cudaStream_t s) {
+                         int act_bf16, cudaStream_t s, const int32_t* rows_idx) {
   if (M <= 0) return nullptr;
   if (M < 1024) {   // few rows: a block per row keeps enough SMs busy
     if (act_bf16)
-      rmsnorm_block_kernel<bf16><<<M, 256, 0, s>>>(x, d, gain, w_bf16, eps, out, ldo);
+      rmsnorm_block_kernel<bf16><<<M, 256, 0, s>>>(x, d, gain, w_bf16, eps, out, ldo, rows_idx);
     else
-      rmsnorm_block_kernel<float><<<M, 256, 0, s>>>(x, d, gain, w_bf16, eps, out, ldo);
+      rmsnorm_block_kernel<float><<<M, 256, 0, s>>>(x, d, gain, w_bf16, eps, out, ldo, rows_idx);
     return err();
   }
   if (act_bf16)
-    rmsnorm_kernel<bf16><<<rows_grid(M), WPB * 32, 0, s>>>(x, M, d, gain, w_bf16, eps, out, ldo);
+    rmsnorm_kernel<bf16><<<rows_grid(M), WPB * 32, 0, s>>>(x, M, d, gain, w_bf16, eps, out, ldo, rows_idx);
   else
-    rmsnorm_kernel<float><<<rows_grid(M), WPB * 32, 0, s>>>(x, M, d, gain, w_bf16, eps, out, ldo);
+    rmsnorm_kernel<float><<<rows_grid(M), WPB * 32, 0, s>>>(x, M, d, gain, w_bf16, eps, out, ldo, rows_idx);
   return err();
 }
 

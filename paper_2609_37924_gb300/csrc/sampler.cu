@@ -76,7 +76,7 @@ __global__ void __launch_bounds__(256) confidence_kernel(const float* __restrict
 // One warp per row: merge the per-column-tile (max, sum exp, argmax) partials
 // written by the output-head GEMM epilogue.
 __global__ void combine_kernel(const float* __restrict__ part, int rows, int n_tiles, float* __restrict__ conf,
-                               int32_t* __restrict__ tok) {
+                               int32_t* __restrict__ tok, const int32_t* __restrict__ rows_idx) {
   const int r = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (r >= rows) return;
   const float* p = part + static_cast<size_t>(r) * n_tiles * 3;
@@ -100,9 +100,45 @@ __global__ void combine_kernel(const float* __restrict__ part, int rows, int n_t
   }
   s = warp_sum(s);
   if (lane == 0) {
-    conf[r] = 1.0f / s;
-    tok[r] = arg;
+    const int dst = rows_idx ? rows_idx[r] : r;   // compacted rows scatter back to their positions
+    conf[dst] = 1.0f / s;
+    tok[dst] = arg;
   }
+}
+
+// One block per sequence: ordered list of the rows that still hold MASK.
+__global__ void __launch_bounds__(256) masked_rows_kernel(const int32_t* __restrict__ z, int ldz, int rows,
+                                                          int mask_id, int per_seq, int32_t* __restrict__ idx,
+                                                          float* __restrict__ conf) {
+  __shared__ int base;
+  __shared__ int wsum[8];
+  const int b = blockIdx.x;
+  const int32_t* zb = z + static_cast<size_t>(b) * ldz;
+  if (threadIdx.x == 0) base = 0;
+  __syncthreads();
+  for (int r0 = 0; r0 < rows; r0 += 256) {
+    const int r = r0 + threadIdx.x;
+    const bool m = r < rows && zb[r] == mask_id;
+    if (r < rows) conf[static_cast<size_t>(b) * rows + r] = -INFINITY;
+    const unsigned ballot = __ballot_sync(0xffffffffu, m);
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    if (lane == 0) wsum[w] = __popc(ballot);
+    __syncthreads();
+    int before = base;
+    for (int i = 0; i < w; ++i) before += wsum[i];
+    const int j = before + __popc(ballot & ((1u << lane) - 1u));
+    if (m && j < per_seq) idx[static_cast<size_t>(b) * per_seq + j] = b * rows + r;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int t = 0;
+      for (int i = 0; i < 8; ++i) t += wsum[i];
+      base += t;
+    }
+    __syncthreads();
+  }
+  // sequences with fewer masked rows than per_seq: pad with their last row (results overwritten identically)
+  if (threadIdx.x == 0)
+    for (int j = base; j < per_seq; ++j) idx[static_cast<size_t>(b) * per_seq + j] = b * rows + (rows - 1);
 }
 
 // One block per sequence: k rounds of a block-wide (conf desc, pos asc) argmax
@@ -150,9 +186,17 @@ const char* confidence_rows(const float* logits, int rows, int vocab, int ld, in
   return err();
 }
 
-const char* combine_partials(const float* part, int rows, int n_tiles, float* conf, int32_t* tok, cudaStream_t s) {
+const char* combine_partials(const float* part, int rows, int n_tiles, float* conf, int32_t* tok, cudaStream_t s,
+                             const int32_t* rows_idx) {
   if (rows <= 0) return nullptr;
-  combine_kernel<<<(rows + 7) / 8, 256, 0, s>>>(part, rows, n_tiles, conf, tok);
+  combine_kernel<<<(rows + 7) / 8, 256, 0, s>>>(part, rows, n_tiles, conf, tok, rows_idx);
+  return err();
+}
+
+const char* masked_rows(const int32_t* z, int ldz, int batch, int rows, int mask_id, int per_seq, int32_t* idx,
+                        float* conf, cudaStream_t s) {
+  if (batch <= 0 || rows <= 0) return nullptr;
+  masked_rows_kernel<<<batch, 256, 0, s>>>(z, ldz, rows, mask_id, per_seq, idx, conf);
   return err();
 }
 

@@ -116,7 +116,7 @@ struct tadm_handle {
   char* ws = nullptr;
   size_t ws_bytes = 0, ws_need = 0;
   struct Off {
-    size_t status, rope, c, x, h_int, norm, qbuf, kv, attn, glu, f_g, f_hid, f_pre, part, conf, tok, split;
+    size_t status, rope, c, x, h_int, norm, qbuf, kv, attn, glu, f_g, f_hid, f_pre, part, conf, tok, split, idx;
     size_t pa_z, pa_j, pa_mq, pa_mk, pa_mv, pa_mo, pa_r, pa_rb, pa_hid, pa_phi, pa_m, pa_dz, pa_f, pa_g, pa_mb;
   } off{};
   size_t kv_slab = 0;
@@ -253,6 +253,7 @@ void layout(tadm_handle* h) {
   f.split = c.dtype ? take(gemm_tc_split_bytes()) : take(0);
   f.conf = take(M * 4);
   f.tok = take(M * 4);
+  f.idx = take(M * 4);
   h->ws_need = o;
 }
 
@@ -496,23 +497,34 @@ tadm_status run_fusion(tadm_handle* h, int B, int R, const void* cache, cudaStre
   return gemm(h, Mb, Mmax, r, h->fw[9], r, M, d, r, EPI_PA_UP, eu, s);
 }
 
-// D on x, then the output head and the per-row (conf, tok).
-tadm_status run_D_head(tadm_handle* h, int B, int R, float* logits, cudaStream_t s) {
+// D on x, then the output head and the per-row (conf, tok).  With
+// masked_per_seq > 0 (and no logits requested) only the rows that still hold
+// MASK go through the head: the sampler reads nothing else (carry-over), so
+// the result is the same; they are gathered by the final RMSNorm and their
+// (conf, tok) scattered back, the other rows get conf = -inf.
+tadm_status run_D_head(tadm_handle* h, int B, int R, float* logits, cudaStream_t s, const int32_t* z = nullptr,
+                       int ldz = 0, int masked_per_seq = 0) {
   const tadm_config& c = h->cfg;
   const int M = B * R, d = c.d_model;
   const int64_t Mmax = static_cast<int64_t>(h->max_batch) * h->max_rows;
   float* x = h->at<float>(h->off.x);
   TRYS(stack_fwd(h, c.n_shared + c.n_anchor, c.n_denoise, x, B, R, h->ctx, 0, s));
   void* norm = h->at(h->off.norm);
-  TRY(rmsnorm_rows(x, M, d, h->final_norm, c.dtype, c.norm_eps, norm, d, h->act_bf16(), s));
+  const bool compact = masked_per_seq > 0 && !logits && z;
+  const int Mh = compact ? B * masked_per_seq : M;
+  const int32_t* idx = compact ? h->at<int32_t>(h->off.idx) : nullptr;
+  if (compact)
+    TRY(masked_rows(z, ldz, B, R, c.vocab - 1, masked_per_seq, h->at<int32_t>(h->off.idx),
+                    h->at<float>(h->off.conf), s));
+  TRY(rmsnorm_rows(x, Mh, d, h->final_norm, c.dtype, c.norm_eps, norm, d, h->act_bf16(), s, idx));
   EpiParams e{};
   e.part = h->at<float>(h->off.part);
   e.mask_id = c.vocab - 1;
   e.logits = logits;
   e.ld_logits = c.vocab;
-  TRYS(gemm(h, norm, Mmax, d, h->lm_head, d, M, c.vocab, d, EPI_LMHEAD, e, s));
-  TRY(combine_partials(h->at<float>(h->off.part), M, h->n_part_tiles, h->at<float>(h->off.conf),
-                       h->at<int32_t>(h->off.tok), s));
+  TRYS(gemm(h, norm, Mmax, d, h->lm_head, d, Mh, c.vocab, d, EPI_LMHEAD, e, s));
+  TRY(combine_partials(h->at<float>(h->off.part), Mh, h->n_part_tiles, h->at<float>(h->off.conf),
+                       h->at<int32_t>(h->off.tok), s, idx));
   return TADM_OK;
 }
 
@@ -551,7 +563,7 @@ tadm_status check_ready(tadm_handle* h, int B, int R) {
 
 // One reverse step after the (optional) refresh: c is already in the workspace.
 tadm_status step_after_S(tadm_handle* h, int32_t* z, int ldz, int B, int R, int k, const void* cache,
-                         const tadm_step_outputs* out, cudaStream_t s) {
+                         const tadm_step_outputs* out, cudaStream_t s, int masked_per_seq = 0) {
   const tadm_config& c = h->cfg;
   TRYS(run_fusion(h, B, R, cache, s));
   const int M = B * R;
@@ -559,7 +571,7 @@ tadm_status step_after_S(tadm_handle* h, int32_t* z, int ldz, int B, int R, int 
       cudaMemcpyAsync(out->fused, h->at(h->off.x), static_cast<size_t>(M) * c.d_model * 4, cudaMemcpyDeviceToDevice,
                       s) != cudaSuccess)
     return fail(h, TADM_ERR_CUDA, "copy fused latent failed");
-  TRYS(run_D_head(h, B, R, out ? out->logits : nullptr, s));
+  TRYS(run_D_head(h, B, R, out ? out->logits : nullptr, s, z, ldz, masked_per_seq));
   float* conf = h->at<float>(h->off.conf);
   int32_t* tok = h->at<int32_t>(h->off.tok);
   if (out && out->conf && cudaMemcpyAsync(out->conf, conf, M * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess)
@@ -881,11 +893,15 @@ tadm_status tadm_generate(tadm_handle* h, const int32_t* prompt, int batch, int 
         h->counters.anchor_calls += 1;
         have_c = true;
         break;
-      case 2:  // denoising step with the (possibly stale) cache, then the sampler
+      case 2: {  // denoising step with the (possibly stale) cache, then the sampler
         if (!have_c) TRYS(run_S(h, z, total, batch, R, 0, s));
         have_c = false;
-        TRYS(step_after_S(h, z, total, batch, R, e.k, cache, nullptr, s));
+        // positions of the active rows still masked before step n: G_b - floor(n G_b / T)
+        const int Gb = block_len > 0 ? block_len : gen_len;
+        const int masked = Gb - static_cast<int>(static_cast<int64_t>(e.n) * Gb / steps_per_block);
+        TRYS(step_after_S(h, z, total, batch, R, e.k, cache, nullptr, s, masked));
         break;
+      }
       case 3:  // commit the finished block into the KV context
         TRYS(fresh_pass(h, z, total, batch, block_len, s));
         break;
