@@ -192,18 +192,19 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
       const int lim = kv_hi - key0;                                   // visible keys of this tile
       const bool masked = __any_sync(0xffffffffu, lim < TKV);         // warp-uniform path choice
       float v[16];
-      float mx = -INFINITY;
+      float mxa[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};   // independent chains
 #pragma unroll
       for (int c = 0; c < TKV / 16; ++c) {
         tmem_ld16(t_s + lane_off + 16 * c, v);
         if (masked) {
 #pragma unroll
-          for (int i = 0; i < 16; ++i) mx = fmaxf(mx, 16 * c + i < lim ? v[i] : -INFINITY);
+          for (int i = 0; i < 16; ++i) mxa[i & 3] = fmaxf(mxa[i & 3], 16 * c + i < lim ? v[i] : -INFINITY);
         } else {
 #pragma unroll
-          for (int i = 0; i < 16; ++i) mx = fmaxf(mx, v[i]);
+          for (int i = 0; i < 16; ++i) mxa[i & 3] = fmaxf(mxa[i & 3], v[i]);
         }
       }
+      const float mx = fmaxf(fmaxf(mxa[0], mxa[1]), fmaxf(mxa[2], mxa[3]));
       const float m_new = fmaxf(m_run, mx * args.scale_log2);
       const float alpha = (m_run == -INFINITY) ? 0.0f : ex2_approx(m_run - m_new);
       if (j > 0) {
@@ -220,7 +221,7 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
         mbar_arrive(o_free);
       }
       // P = 2^(s * scale - m_new) as bf16 into the swizzled A-operand layout
-      float psum = 0.0f;
+      float ps[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
       for (int c = 0; c < TKV / 16; ++c) {
         tmem_ld16(t_s + lane_off + 16 * c, v);
@@ -233,7 +234,7 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
             p0 = 16 * c + i < lim ? p0 : 0.0f;
             p1 = 16 * c + i + 1 < lim ? p1 : 0.0f;
           }
-          psum += p0 + p1;
+          ps[(i >> 1) & 3] += p0 + p1;
           __nv_bfloat162 t = __floats2bfloat162_rn(p0, p1);
           pk[i / 2] = *reinterpret_cast<uint32_t*>(&t);
         }
@@ -243,6 +244,7 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
         *reinterpret_cast<uint4*>(atom + ((chunk ^ (row & 7)) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
         *reinterpret_cast<uint4*>(atom + (((chunk + 1) ^ (row & 7)) << 4)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
       }
+      const float psum = (ps[0] + ps[1]) + (ps[2] + ps[3]);
       l_run = l_run * alpha + psum;
       m_run = m_new;
       alpha_prev = alpha;
