@@ -191,17 +191,27 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
       const int kv_hi = args.causal ? min(kv_end, qpos + 1) : kv_end;
       const int lim = kv_hi - key0;                                   // visible keys of this tile
       const bool masked = __any_sync(0xffffffffu, lim < TKV);         // warp-uniform path choice
-      float v[16];
+      // pass 1: row max over the tile, 64 columns per TMEM round trip
       float mxa[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};   // independent chains
 #pragma unroll
-      for (int c = 0; c < TKV / 16; ++c) {
-        tmem_ld16(t_s + lane_off + 16 * c, v);
+      for (int c = 0; c < TKV / 64; ++c) {
+        uint32_t ra[32], rb[32];
+        tmem_ld32_nowait(t_s + lane_off + 64 * c, ra);
+        tmem_ld32_nowait(t_s + lane_off + 64 * c + 32, rb);
+        tmem_wait_ld(ra);
+        tmem_bind(rb);
         if (masked) {
 #pragma unroll
-          for (int i = 0; i < 16; ++i) mxa[i & 3] = fmaxf(mxa[i & 3], 16 * c + i < lim ? v[i] : -INFINITY);
+          for (int i = 0; i < 32; ++i) {
+            mxa[i & 3] = fmaxf(mxa[i & 3], 64 * c + i < lim ? __uint_as_float(ra[i]) : -INFINITY);
+            mxa[i & 3] = fmaxf(mxa[i & 3], 64 * c + 32 + i < lim ? __uint_as_float(rb[i]) : -INFINITY);
+          }
         } else {
 #pragma unroll
-          for (int i = 0; i < 16; ++i) mxa[i & 3] = fmaxf(mxa[i & 3], v[i]);
+          for (int i = 0; i < 32; ++i) {
+            mxa[i & 3] = fmaxf(mxa[i & 3], __uint_as_float(ra[i]));
+            mxa[i & 3] = fmaxf(mxa[i & 3], __uint_as_float(rb[i]));
+          }
         }
       }
       const float mx = fmaxf(fmaxf(mxa[0], mxa[1]), fmaxf(mxa[2], mxa[3]));
@@ -212,37 +222,49 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
         if (!warp_wait_bounded(o_full, (j - 1) & 1, abort_flag, args.status)) { ok = false; break; }
         tc_fence_after();
 #pragma unroll
-        for (int c = 0; c < HD / 16; ++c) {
-          tmem_ld16(t_o + lane_off + 16 * c, v);
+        for (int c = 0; c < HD / 64; ++c) {
+          uint32_t ra[32], rb[32];
+          tmem_ld32_nowait(t_o + lane_off + 64 * c, ra);
+          tmem_ld32_nowait(t_o + lane_off + 64 * c + 32, rb);
+          tmem_wait_ld(ra);
+          tmem_bind(rb);
 #pragma unroll
-          for (int i = 0; i < 16; ++i) o_acc[16 * c + i] = fmaf(o_acc[16 * c + i], alpha_prev, v[i]);
+          for (int i = 0; i < 32; ++i) {
+            o_acc[64 * c + i] = fmaf(o_acc[64 * c + i], alpha_prev, __uint_as_float(ra[i]));
+            o_acc[64 * c + 32 + i] = fmaf(o_acc[64 * c + 32 + i], alpha_prev, __uint_as_float(rb[i]));
+          }
         }
         tc_fence_before();
         mbar_arrive(o_free);
       }
-      // P = 2^(s * scale - m_new) as bf16 into the swizzled A-operand layout
+      // pass 2: P = 2^(s * scale - m_new) as bf16 into the swizzled A-operand layout, 32 columns per trip
       float ps[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
-      for (int c = 0; c < TKV / 16; ++c) {
-        tmem_ld16(t_s + lane_off + 16 * c, v);
-        uint32_t pk[8];
+      for (int c = 0; c < TKV / 32; ++c) {
+        uint32_t ra[32];
+        tmem_ld32_nowait(t_s + lane_off + 32 * c, ra);
+        tmem_wait_ld(ra);
+        uint32_t pk[16];
 #pragma unroll
-        for (int i = 0; i < 16; i += 2) {
-          float p0 = ex2_approx(fmaf(v[i], args.scale_log2, -m_new));
-          float p1 = ex2_approx(fmaf(v[i + 1], args.scale_log2, -m_new));
+        for (int i = 0; i < 32; i += 2) {
+          float p0 = ex2_approx(fmaf(__uint_as_float(ra[i]), args.scale_log2, -m_new));
+          float p1 = ex2_approx(fmaf(__uint_as_float(ra[i + 1]), args.scale_log2, -m_new));
           if (masked) {
-            p0 = 16 * c + i < lim ? p0 : 0.0f;
-            p1 = 16 * c + i + 1 < lim ? p1 : 0.0f;
+            p0 = 32 * c + i < lim ? p0 : 0.0f;
+            p1 = 32 * c + i + 1 < lim ? p1 : 0.0f;
           }
           ps[(i >> 1) & 3] += p0 + p1;
           __nv_bfloat162 t = __floats2bfloat162_rn(p0, p1);
           pk[i / 2] = *reinterpret_cast<uint32_t*>(&t);
         }
-        // keys 16c .. 16c+15: atom (16c / 64), 16-byte chunks (16c % 64) / 8 and +1
-        uint8_t* atom = prow0 + (c >> 2) * 16384;
-        const int chunk = (c & 3) * 2;
-        *reinterpret_cast<uint4*>(atom + ((chunk ^ (row & 7)) << 4)) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-        *reinterpret_cast<uint4*>(atom + (((chunk + 1) ^ (row & 7)) << 4)) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+        // keys 32c .. 32c+31: atom (32c / 64), 16-byte chunks (32c % 64) / 8 .. +3
+        uint8_t* atom = prow0 + (c >> 1) * 16384;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int chunk = (c & 1) * 4 + q;
+          *reinterpret_cast<uint4*>(atom + ((chunk ^ (row & 7)) << 4)) =
+              make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+        }
       }
       const float psum = (ps[0] + ps[1]) + (ps[2] + ps[3]);
       l_run = l_run * alpha + psum;
@@ -255,12 +277,13 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
     }
     if (ok && n_tiles > 0 && warp_wait_bounded(o_full, (n_tiles - 1) & 1, abort_flag, args.status)) {
       tc_fence_after();
-      float v[16];
 #pragma unroll
-      for (int c = 0; c < HD / 16; ++c) {
-        tmem_ld16(t_o + lane_off + 16 * c, v);
+      for (int c = 0; c < HD / 32; ++c) {
+        uint32_t ra[32];
+        tmem_ld32_nowait(t_o + lane_off + 32 * c, ra);
+        tmem_wait_ld(ra);
 #pragma unroll
-        for (int i = 0; i < 16; ++i) o_acc[16 * c + i] = fmaf(o_acc[16 * c + i], alpha_prev, v[i]);
+        for (int i = 0; i < 32; ++i) o_acc[32 * c + i] = fmaf(o_acc[32 * c + i], alpha_prev, __uint_as_float(ra[i]));
       }
       const int grow = m0 + row;
       if (grow < args.rows) {
