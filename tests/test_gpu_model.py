@@ -6,6 +6,9 @@ agree; argmax over all positions agrees on >= 95% for bf16 (random-init
 logits have top-1/top-2 gaps of ~0.2 sigma, so bf16 rounding flips a few
 percent of the near-ties; see the reading on token agreement).
 """
+import json
+import os
+
 import numpy as np
 import pytest
 
@@ -326,13 +329,23 @@ def test_committed_token_agreement_teacher_forced(T, case):
     and predicts the tokens at the positions the GPU commits.
 
     small_workload_dims: the 'small' workload's model (d 768, 8 + 4 layers,
-    vocab 32768) on a 256-position canvas, batch 8, 32 steps of 6 commits:
-    confidence-selected commits must agree >= 99.5%.
+    vocab 32768) on a 256-position canvas, batch 8, 32 steps of 6 commits.
+    tests/bf16_floor.py runs this very protocol with the oracle's arithmetic
+    rounded to bf16 at every tensor-core operand and stores the agreement it
+    reaches (tests/golden/bf16_floor_small.json): the GPU must agree on at
+    least as many confidence-selected commits as that ideal bf16 path, less
+    six (rounding-order noise: near-ties flip either way), and on >= 99%.
     test_model: the 4-layer d 256 vocab 4096 test model, batch 16 (>= 99%).
     Forced commits (last step of the block) are reported."""
+    floor = None
     if case == "small_workload_dims":
         m = wl.WORKLOADS["small"].model
-        B, P, G, Tn, K, gate = 8, 64, 192, 32, 4, 0.995
+        B, P, G, Tn, K, gate = 8, 64, 192, 32, 4, 0.99
+        with open(os.path.join(os.path.dirname(__file__), "golden", "bf16_floor_small.json")) as f:
+            floor = json.load(f)
+        fp = floor["protocol"]
+        assert (fp["batch"], fp["prompt_len"], fp["gen_len"], fp["steps"], fp["K"], fp["weight_seed"],
+                fp["prompt_seed"]) == (B, P, G, Tn, K, 7, 17)
     else:
         m = wl.ModelConfig(**SMALL_BF16)
         B, P, G, Tn, K, gate = 16, 32, 96, 16, 4, 0.99
@@ -358,4 +371,8 @@ def test_committed_token_agreement_teacher_forced(T, case):
           f"{agg.masked_ok / agg.masked:.4f}")
     assert agg.committed >= 1000
     assert sel_rate >= gate, sel_rate
+    if floor is not None:
+        print(f"[agreement {case}] ideal bf16 path: {floor['selected_ok']}/{floor['selected']}")
+        assert agg.committed == floor["selected"]
+        assert agg.committed_ok >= floor["selected_ok"] - 6, (agg.committed_ok, floor["selected_ok"])
     assert agg.masked_ok / agg.masked >= 0.95
