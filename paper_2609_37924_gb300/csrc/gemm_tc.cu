@@ -11,11 +11,14 @@
 //               thread; two warps per lane quadrant, each taking half of the
 //               256 columns) and run the fused epilogue of epilogue.cuh, while
 //               the MMA warp fills the other accumulator.
+// GEMMs of more than 128 rows that need no split-K run the CTA-pair variant
+// (gemm_tc2_kernel: 256 x 256 tiles, tcgen05.mma.cta_group::2, six stages).
 // Every mbarrier wait is bounded (mbar_wait_bounded): a role that gives up
 // raises a shared abort flag and the device status word, and the CTA drains
 // its in-flight copies and MMAs, frees TMEM and exits.
 #include <cudaTypedefs.h>
 #include <algorithm>
+#include <cstdlib>
 #include <mutex>
 
 #include "epilogue.cuh"
@@ -285,10 +288,184 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   }
 }
 
+// ------------------------------------------------------- CTA-pair variant
+// One 256 x 256 tile per 2-CTA cluster with tcgen05.mma.cta_group::2 (M=256,
+// N=256, K=16): CTA r holds A rows 128r..128r+127 of the tile and B rows
+// 128r..128r+127 (its half of the N columns) in its own shared memory, and
+// its 128 rows of the accumulator in its own TMEM.  Each SM thus receives
+// 32 KB of operands per 64-deep k-block instead of 48 KB for the same MMA
+// work, and six stages fit in shared memory.  Roles per CTA as above; only
+// the even CTA's MMA thread issues.  Barriers: both producers count their
+// bytes on the even CTA's full[s] (the even producer expects both CTAs'
+// bytes); the MMA thread's commits release empty[s] and signal tfull[a] in
+// both CTAs; every epilogue warp of both CTAs releases an accumulator on the
+// even CTA's tempty[a].
+constexpr int P_STAGES = 6;
+constexpr int P_A_BYTES = BM * BK * 2;            // 16 KB
+constexpr int P_B_BYTES = (BN / 2) * BK * 2;      // 16 KB: this CTA's half of B
+constexpr int P_STAGE_BYTES = P_A_BYTES + P_B_BYTES;
+constexpr size_t P_SMEM_BYTES = 1024 + P_STAGES * P_STAGE_BYTES + EPI_WARPS * STAGE_OUT_BYTES + 256;
+static_assert(P_SMEM_BYTES <= 232448, "pair GEMM shared memory");
+
+template <int EPI>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
+    gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                    const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmC2,
+                    const TcArgs args) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + P_STAGES * P_A_BYTES;
+  uint8_t* sOut = smem + P_STAGES * P_STAGE_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sOut + EPI_WARPS * STAGE_OUT_BYTES);
+  uint64_t* empty = full + P_STAGES;
+  uint64_t* tfull = empty + P_STAGES;
+  uint64_t* tempty = tfull + 2;
+  uint64_t* drain = tempty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < P_STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&tfull[a], 1);
+      mbar_init(&tempty[a], 2 * EPI_WARPS);   // one arrival per epilogue warp of either CTA
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(tmem_slot, TMEM_COLS);   // one warp of each CTA, collectively
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();   // the peer's barriers are initialised (and its TMEM allocated) before any signal
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int num_m2 = (args.M + 2 * BM - 1) / (2 * BM);
+  const int units = num_m2 * args.n_tiles_n;
+  const int u0 = static_cast<int>(blockIdx.x >> 1), ustep = static_cast<int>(gridDim.x >> 1);
+  const int kblocks = (args.K + BK - 1) / BK;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------------------------------------------------------- producer (both CTAs)
+      const uint32_t full_l0 = cluster_addr(full, 0);   // the even CTA's full[0]
+      int stage = 0;
+      uint32_t phase = 0;
+      for (int unit = u0; unit < units && !*abort_flag; unit += ustep) {
+        const int nb = unit % args.n_tiles_n;
+        const int mb = 2 * (unit / args.n_tiles_n) + static_cast<int>(rank);   // this CTA's 128-row block
+        prefetch_epilogue_inputs<EPI>(args, mb, nb);
+        const int brow = args.b_split > 0 ? (rank ? args.b_split : 0) + nb * (BN / 2) : nb * BN + rank * (BN / 2);
+        bool ok = true;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait_bounded(&empty[stage], phase ^ 1, abort_flag, args.status)) { ok = false; break; }
+          if (leader) mbar_arrive_expect_tx(&full[stage], 2 * P_STAGE_BYTES);
+          const uint32_t fb = full_l0 + 8u * stage;
+          tma_load_2d_pair(sA + stage * P_A_BYTES, &tmA, fb, kb * BK, mb * BM);
+          tma_load_2d_pair(sB + stage * P_B_BYTES, &tmB, fb, kb * BK, brow);
+          if (++stage == P_STAGES) { stage = 0; phase ^= 1; }
+        }
+        if (!ok) break;
+      }
+      // the MMA thread's last commits arrive on these barriers (from the even
+      // CTA): wait until every stage is released, which also means every copy
+      // into this CTA's shared memory has landed and been consumed
+      for (int i = 0; i < P_STAGES; ++i) {
+        mbar_wait_bounded(&empty[stage], phase ^ 1, abort_flag, args.status);
+        if (++stage == P_STAGES) { stage = 0; phase ^= 1; }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && leader) {
+      // ---------------------------------------------------------------- MMA issuer (even CTA)
+      constexpr uint32_t idesc = idesc_bf16_f32(2 * BM, BN);
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      for (int unit = u0; unit < units && !*abort_flag; unit += ustep) {
+        if (!mbar_wait_bounded(&tempty[acc], acc_phase ^ 1, abort_flag, args.status)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * BN;
+        bool ok = true;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait_bounded(&full[stage], phase, abort_flag, args.status)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(sA + stage * P_A_BYTES);
+          const uint32_t b0 = smem_u32(sB + stage * P_B_BYTES);
+#pragma unroll
+          for (int k = 0; k < BK / 16; ++k) {
+            umma_bf16_pair(d_tmem, sdesc_kmajor_sw128(a0 + 32 * k), sdesc_kmajor_sw128(b0 + 32 * k), idesc,
+                           (kb != 0) || (k != 0));
+          }
+          umma_commit_pair_mc(&empty[stage], 0x3);
+          if (++stage == P_STAGES) { stage = 0; phase ^= 1; }
+        }
+        if (!ok) break;
+        umma_commit_pair_mc(&tfull[acc], 0x3);
+        if (++acc == 2) { acc = 0; acc_phase ^= 1; }
+      }
+      // every pair MMA is complete (both CTAs' TMEM written) before TMEM is freed
+      umma_commit_pair_mc(drain, 0x1);
+      volatile int never = 0;
+      mbar_wait_bounded(drain, 0, &never, args.status);
+    }
+  } else {
+    // ------------------------------------------------------------------ epilogue (both CTAs)
+    const int quad = warp & 3;
+    const int part = (warp - 2) / 4;
+    constexpr int nsplit = EPI == EPI_PA_GATE ? 1 : 2;
+    const uint32_t tempty_l0 = cluster_addr(tempty, 0);
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int unit = u0; unit < units; unit += ustep) {
+      if (!warp_wait_bounded(&tfull[acc], acc_phase, abort_flag, args.status)) break;
+      tc_fence_after();
+      const int nb = unit % args.n_tiles_n;
+      const int mb = 2 * (unit / args.n_tiles_n) + static_cast<int>(rank);
+      TmemSrc src{tmem_base + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(quad * 32) << 16),
+                  args.staged ? sOut + (warp - 2) * STAGE_OUT_BYTES : nullptr, {&tmC, &tmC2}, mb * BM + quad * 32};
+      const int m = mb * BM + quad * 32 + lane;
+      if (part < nsplit && mb * BM < args.M)   // the odd CTA's rows may lie past M
+        epilogue_row<EPI>(args.ep, m, nb, BN, src, part, nsplit);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_remote(tempty_l0 + 8u * acc);
+      if (++acc == 2) { acc = 0; acc_phase ^= 1; }
+    }
+    if (args.staged && lane == 0) bulk_wait0();
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  // neither CTA frees TMEM or exits while the pair's MMAs, copies or
+  // barrier signals may still reach it
+  cluster_sync();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc_pair(tmem_base, TMEM_COLS);
+  }
+}
+
 // --------------------------------------------------------------------- host
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 std::once_flag g_encode_once;
 int g_num_sms = 0;
+bool g_pair_mma = true;   // CTA-pair kernel for large GEMMs; TADM_GEMM_PAIRS=0 keeps every GEMM on one CTA per tile
 
 bool get_encoder() {
   std::call_once(g_encode_once, [] {
@@ -301,6 +478,8 @@ bool get_encoder() {
     int dev = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
+    const char* env = getenv("TADM_GEMM_PAIRS");
+    if (env && env[0] == '0') g_pair_mma = false;
   });
   return g_encode != nullptr;
 }
@@ -340,6 +519,33 @@ cudaError_t launch_epi(const CUtensorMap& ta, const CUtensorMap& tb, const CUten
     attr_set = true;
   }
   gemm_tc_kernel<EPI><<<grid, NUM_THREADS, SMEM_BYTES, s>>>(ta, tb, tc, tc2, a);
+  return cudaGetLastError();
+}
+
+// CTA-pair kernel: `pairs` = 256-row x 256-column tiles; the grid is capped at
+// the number of 2-CTA clusters that fit on the GPU at once (a persistent grid
+// larger than that would run its last clusters after the others).
+template <int EPI>
+cudaError_t launch_epi_pair(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc,
+                            const CUtensorMap& tc2, const TcArgs& a, int pairs, cudaStream_t s) {
+  static int max_clusters = 0;
+  if (max_clusters == 0) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc2_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(P_SMEM_BYTES));
+    if (e != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3(g_num_sms & ~1);
+    cfg.blockDim = dim3(NUM_THREADS);
+    cfg.dynamicSmemBytes = P_SMEM_BYTES;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc2_kernel<EPI>, &cfg) != cudaSuccess || n <= 0) {
+      cudaGetLastError();
+      n = g_num_sms / 2;
+    }
+    max_clusters = n;
+  }
+  const int clusters = std::min(pairs, max_clusters);
+  gemm_tc2_kernel<EPI><<<2 * clusters, NUM_THREADS, P_SMEM_BYTES, s>>>(ta, tb, tc, tc2, a);
   return cudaGetLastError();
 }
 
@@ -402,6 +608,31 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
       a.part_stride = static_cast<size_t>(g.M) * a.ldp;
       a.staged = 0;
     }
+  }
+  // CTA pairs (256 x 256 tiles, cta_group::2) for every unsplit GEMM of more
+  // than 128 rows: the same SMs as 128 x 256 tiles, less operand traffic each
+  const int pair_units = ((g.M + 2 * BM - 1) / (2 * BM)) * a.n_tiles_n;
+  if (g_pair_mma && a.splits == 1 && g.M > BM) {
+    CUtensorMap tbh;
+    if (!make_map(&tbh, g.B, b_rows, g.K, g.ldb, BN / 2)) return "tensor map (B, half tiles) encode failed";
+    cudaError_t e;
+    switch (g.epi) {
+      case EPI_STORE: e = launch_epi_pair<EPI_STORE>(ta, tbh, tc, tc2, a, pair_units, s); break;
+      case EPI_RESID: e = launch_epi_pair<EPI_RESID>(ta, tbh, tc, tc2, a, pair_units, s); break;
+      case EPI_QKV: e = launch_epi_pair<EPI_QKV>(ta, tbh, tc, tc2, a, pair_units, s); break;
+      case EPI_GLU: e = launch_epi_pair<EPI_GLU>(ta, tbh, tc, tc2, a, pair_units, s); break;
+      case EPI_FUSION1: e = launch_epi_pair<EPI_FUSION1>(ta, tbh, tc, tc2, a, pair_units, s); break;
+      case EPI_FUSION2: e = launch_epi_pair<EPI_FUSION2>(ta, tbh, tc, tc2, a, pair_units, s); break;
+      case EPI_LMHEAD: e = launch_epi_pair<EPI_LMHEAD>(ta, tbh, tc, tc2, a, pair_units, s); break;
+      case EPI_PA_UP: e = launch_epi_pair<EPI_PA_UP>(ta, tbh, tc, tc2, a, pair_units, s); break;
+      case EPI_SILU: e = launch_epi_pair<EPI_SILU>(ta, tbh, tc, tc2, a, pair_units, s); break;
+      case EPI_ADD: e = launch_epi_pair<EPI_ADD>(ta, tbh, tc, tc2, a, pair_units, s); break;
+      case EPI_PA_GATE: e = launch_epi_pair<EPI_PA_GATE>(ta, tbh, tc, tc2, a, pair_units, s); break;
+      default: return "unknown epilogue";
+    }
+    if (e != cudaSuccess) return cudaGetErrorString(e);
+    const_cast<GemmCall&>(g).launched = 1;
+    return nullptr;
   }
   const int units = tiles * a.splits;
   const int grid = units < g_num_sms ? units : g_num_sms;
