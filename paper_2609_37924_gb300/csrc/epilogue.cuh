@@ -29,6 +29,7 @@ struct EpiParams {
   int ldo, out_bf16;        // out element type: bf16 (1) or fp32 (0)
   float* resid;
   int ldr;
+  int resid_tma;            // EPI_RESID on the tensor-core path: resid += acc by TMA reduce-add (map in the source)
   const float* base;        // EPI_ADD base, EPI_FUSION2 h, EPI_PA_UP H0
   int ldb;
   const void* bias;         // [N] weights dtype
@@ -61,11 +62,29 @@ __device__ __forceinline__ float ld_param(const void* p, int bf, int i) {
   return bf ? __bfloat162float(static_cast<const bf16*>(p)[i]) : static_cast<const float*>(p)[i];
 }
 
-__device__ __forceinline__ float silu_f(float x) { return x / (1.0f + expf(-x)); }
-__device__ __forceinline__ float sigmoid_f(float x) { return 1.0f / (1.0f + expf(-x)); }
-__device__ __forceinline__ float gelu_erf_f(float x) { return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f)); }
+// Activations of the epilogues.  Their outputs feed bf16 GEMM operands (or
+// are rounded to bf16), so they use the fast exp2-based exponential and the
+// approximate reciprocal / division, whose errors (a few fp32 ulp) lie far
+// below bf16's rounding step.  At the extremes: exp overflow gives
+// x / inf = -0 for SiLU and 0 for the sigmoid, exp underflow gives x and 1.
+__device__ __forceinline__ float silu_f(float x) { return __fdividef(x, 1.0f + __expf(-x)); }
+__device__ __forceinline__ float sigmoid_f(float x) { return __fdividef(1.0f, 1.0f + __expf(-x)); }
+// erf by the rational approximation of Abramowitz & Stegun, Handbook of
+// Mathematical Functions (1964), formula 7.1.26 (after Hastings):
+//   erf(z) = 1 - (a1 t + a2 t^2 + a3 t^3 + a4 t^4 + a5 t^5) exp(-z^2),
+//   t = 1 / (1 + p z), z >= 0, |error| <= 1.5e-7; erf is odd.
+__device__ __forceinline__ float erf_as7126(float x) {
+  const float z = fabsf(x);
+  const float t = __fdividef(1.0f, fmaf(0.3275911f, z, 1.0f));
+  const float poly =
+      t * fmaf(fmaf(fmaf(fmaf(1.061405429f, t, -1.453152027f), t, 1.421413741f), t, -0.284496736f), t, 0.254829592f);
+  return copysignf(fmaf(-poly, __expf(-z * z), 1.0f), x);
+}
+__device__ __forceinline__ float gelu_erf_f(float x) { return 0.5f * x * (1.0f + erf_as7126(x * 0.70710678118654752f)); }
+// tanh(y) = 1 - 2 / (1 + exp(2y)): +-1 at the extremes, absolute error ~1e-7 near 0
+__device__ __forceinline__ float tanh_fast(float y) { return 1.0f - __fdividef(2.0f, 1.0f + __expf(2.0f * y)); }
 __device__ __forceinline__ float gelu_tanh_f(float x) {
-  return 0.5f * x * (1.0f + tanhf(0.79788456080286536f * (x + 0.044715f * x * x * x)));
+  return 0.5f * x * (1.0f + tanh_fast(0.79788456080286536f * (x + 0.044715f * x * x * x)));
 }
 
 // Stores 32 consecutive values (n0 .. n0+31) of one row; `n_valid` of them.
@@ -168,18 +187,49 @@ __device__ __forceinline__ void epilogue_row(const EpiParams& p, int m, int n_bl
         const int n0 = n_blk * ncols + 32 * c;
         int which = 0, x = n0;
         if constexpr (EPI == EPI_FUSION1) {
-          const bool gate = n0 < p.d_split;     // d_split is a multiple of 64
+          // one bias value per lane, broadcast by shuffles; the activation is
+          // chosen once per 64 columns (d_split is a multiple of 64)
+          const int lane = threadIdx.x & 31;
+          const float bl0 = n0 + lane < p.N ? ld_param(p.bias, p.bias_bf16, n0 + lane) : 0.0f;
+          const float bl1 = n0 + 32 + lane < p.N ? ld_param(p.bias, p.bias_bf16, n0 + 32 + lane) : 0.0f;
+          const bool gate = n0 < p.d_split;
+          if (gate) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const float b0 = n0 + i < p.N ? ld_param(p.bias, p.bias_bf16, n0 + i) : 0.0f;
-            const float b1 = n0 + 32 + i < p.N ? ld_param(p.bias, p.bias_bf16, n0 + 32 + i) : 0.0f;
-            v[i] = gate ? sigmoid_f(v[i] + b0) : gelu_erf_f(v[i] + b0);
-            w[i] = gate ? sigmoid_f(w[i] + b1) : gelu_erf_f(w[i] + b1);
+            for (int i = 0; i < 32; ++i) {
+              v[i] = sigmoid_f(v[i] + __shfl_sync(0xffffffffu, bl0, i));
+              w[i] = sigmoid_f(w[i] + __shfl_sync(0xffffffffu, bl1, i));
+            }
+          } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              v[i] = gelu_erf_f(v[i] + __shfl_sync(0xffffffffu, bl0, i));
+              w[i] = gelu_erf_f(w[i] + __shfl_sync(0xffffffffu, bl1, i));
+            }
           }
           which = gate ? 0 : 1;
           x = gate ? n0 : n0 - p.d_split;
         }
         src.store64(which, x, v, w);
+      }
+      return;
+    }
+  }
+  // residual add on the tensor-core path: the warp's 32 x 32 chunk (+ bias) goes
+  // through its shared-memory box and one TMA reduce-add (resid += chunk at
+  // L2), so the epilogue never waits on a load of the residual stream.  Each
+  // element receives exactly one add per GEMM: the result is deterministic.
+  if constexpr (Src::kStaged && EPI == EPI_RESID) {
+    if (src.has_box() && p.resid_tma) {
+      for (int c = c_lo; c < c_hi; ++c) {
+        src.load(c, v);
+        const int n0 = n_blk * ncols + 32 * c;
+        if (p.bias) {
+          const int lane = threadIdx.x & 31;
+          const float bl = n0 + lane < p.N ? ld_param(p.bias, p.bias_bf16, n0 + lane) : 0.0f;
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] += __shfl_sync(0xffffffffu, bl, i);
+        }
+        if (n0 < p.N && src.row0 < p.M) src.reduce32(n0, v);   // the map clips ragged rows / columns
       }
       return;
     }
@@ -298,12 +348,22 @@ __device__ __forceinline__ void epilogue_row(const EpiParams& p, int m, int n_bl
         for (int c = g_lo; c + 1 < g_hi; c += 2) {
           src.load(c, v);
           src.load(c + half / 32, u);
+          if (p.glu) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) v[i] = (p.glu ? gelu_tanh_f(v[i]) : silu_f(v[i])) * u[i];
+            for (int i = 0; i < 32; ++i) v[i] = gelu_tanh_f(v[i]) * u[i];
+          } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = silu_f(v[i]) * u[i];
+          }
           src.load(c + 1, w);
           src.load(c + 1 + half / 32, u);
+          if (p.glu) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) w[i] = (p.glu ? gelu_tanh_f(w[i]) : silu_f(w[i])) * u[i];
+            for (int i = 0; i < 32; ++i) w[i] = gelu_tanh_f(w[i]) * u[i];
+          } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) w[i] = silu_f(w[i]) * u[i];
+          }
           src.store64(0, n_blk * half + 32 * c, v, w);
         }
         return;

@@ -65,6 +65,19 @@ struct TmemSrc {
     __syncwarp();  // tcgen05.ld is warp-collective: reconverge after divergent stores
     tmem_ld32(taddr + 32 * chunk, v);
   }
+  // this lane's row of a 32 x 32 fp32 chunk into the box, then one TMA
+  // reduce-add of the box into the fp32 output map at column x (resid += box)
+  __device__ __forceinline__ void reduce32(int x, const float (&v)[32]) {
+    const int lane = threadIdx.x & 31;
+    if (lane == 0) bulk_wait_read0();   // the previous reduce has read the box
+    put_row(v);
+    fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+      tma_reduce_add_2d(tm_out[0], stage, x, row0);
+      bulk_commit();
+    }
+  }
   // bf16 of a[0..31] and b[0..31] (output columns x .. x+63 of this lane's row)
   // into the box, then one TMA store of the warp's 32 x 64 block; rows and
   // columns outside the output are clipped by the tensor map.
@@ -497,6 +510,17 @@ bool make_map(CUtensorMap* m, const void* ptr, int64_t rows, int64_t cols, int64
   return r == CUDA_SUCCESS;
 }
 
+// 2-D fp32 map over rows x cols (row stride ld elements), box 32 rows x 32, 128-byte swizzle.
+bool make_f32_map(CUtensorMap* m, const void* ptr, int64_t rows, int64_t cols, int64_t ld) {
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld * 4)};
+  cuuint32_t box[2] = {32, 32};
+  cuuint32_t estr[2] = {1, 1};
+  return g_encode(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // 2-D bf16 output map over rows x cols (row stride ld), box 32 rows x 64, 128-byte swizzle.
 bool make_out_map(CUtensorMap* m, const void* ptr, int64_t rows, int64_t cols, int64_t ld) {
   cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
@@ -580,8 +604,12 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
   CUtensorMap tc{}, tc2{};
   a.staged = 0;
   auto aligned = [](const void* p, int ld) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0 && ld % 8 == 0; };
+  a.ep.resid_tma = 0;
   if (g.epi == EPI_RESID || g.epi == EPI_FUSION2) {
-    a.staged = 1;   // the boxes serve as transpose scratch; no output map
+    a.staged = 1;   // the boxes serve as transpose scratch, or as the source of TMA reduce-adds
+    if (g.epi == EPI_RESID && (reinterpret_cast<uintptr_t>(g.ep.resid) & 15) == 0 && g.ep.ldr % 4 == 0 &&
+        make_f32_map(&tc, g.ep.resid, g.M, g.N, g.ep.ldr))
+      a.ep.resid_tma = 1;
   } else if (g.ep.out_bf16 && (g.epi == EPI_STORE || g.epi == EPI_GLU)) {
     if (aligned(g.ep.out, g.ep.ldo) && make_out_map(&tc, g.ep.out, g.M, g.N, g.ep.ldo)) a.staged = 1;
   } else if (g.ep.out_bf16 && g.epi == EPI_FUSION1 && g.ep.d_split % 64 == 0) {
