@@ -12,9 +12,9 @@
 //   one (batch, head).  Warp 0 streams Q once and K / V^T tiles of 128 keys
 //   (2-stage ring) with TMA; warp 1 issues S = Q K^T into TMEM and, once the
 //   probabilities are in shared memory, O_tile = P V into TMEM; warps 2..5
-//   own one query row per thread: masked online softmax on the S row, P as
-//   bf16 into the 128-byte-swizzled operand layout, and O accumulated in
-//   registers with the running-max correction.
+//   own one query row per thread: masked softmax on the S row, P as bf16
+//   into the 128-byte-swizzled operand layout; O accumulates in TMEM across
+//   key tiles, rescaled only when a row's running max grows by more than 2^8.
 // bf16, short rows (attn_bf16_kernel): mma.sync m16n8k16 flash attention.
 // fp32: one warp per query row on the CUDA cores.
 #include <cudaTypedefs.h>
@@ -77,7 +77,6 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
   uint64_t* s_free = bars + 6;
   uint64_t* p_full = bars + 7;
   uint64_t* o_full = bars + 8;
-  uint64_t* o_free = bars + 9;
   uint64_t* drain = bars + 10;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 11);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
@@ -98,7 +97,6 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
     mbar_init(s_free, 128);
     mbar_init(p_full, 128);
     mbar_init(o_full, 1);
-    mbar_init(o_free, 128);
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
@@ -157,13 +155,14 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
           umma_bf16(t_s, sdesc_kmajor_sw128(q0 + (kk >> 2) * 16384 + (kk & 3) * 32),
                     sdesc_kmajor_sw128(k0 + (kk >> 2) * 16384 + (kk & 3) * 32), idesc_s, kk != 0);
         umma_commit(s_full);
+        // P of tile j is in shared memory and any rescale of O by the softmax
+        // threads is complete: O += P V
         if (!mbar_wait_bounded(p_full, j & 1, abort_flag, args.status)) break;
-        if (j > 0 && !mbar_wait_bounded(o_free, (j - 1) & 1, abort_flag, args.status)) break;
         tc_fence_after();
 #pragma unroll
         for (int kk = 0; kk < TKV / 16; ++kk)
           umma_bf16(t_o, sdesc_kmajor_sw128(p0 + (kk >> 2) * 16384 + (kk & 3) * 32),
-                    sdesc_kmajor_sw128(v0 + (kk >> 2) * (HD * 128) + (kk & 3) * 32), idesc_o, kk != 0);
+                    sdesc_kmajor_sw128(v0 + (kk >> 2) * (HD * 128) + (kk & 3) * 32), idesc_o, (j != 0) || (kk != 0));
         umma_commit(o_full);
         umma_commit(&kv_empty[st]);
       }
@@ -173,16 +172,21 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
     }
   } else {
     // --------------------------------------------------------------- softmax
+    // One query row per thread (row = TMEM lane).  O is accumulated in TMEM
+    // by the P V MMAs of all key tiles.  The exponentials of every tile use a
+    // per-row reference max m_ref (log2 units); m_ref moves only when a tile's
+    // max exceeds it by more than 8, and then this thread rescales its row of
+    // O (and l) by 2^(m_ref_old - m_ref_new) before the next P V.  Softmax is
+    // invariant to the reference, and P <= 2^8 keeps bf16 P and fp32 O exact
+    // in range.  The passes use 3-input max and packed fp32-pair arithmetic.
     const int quad = warp & 3;
     const int row = quad * 32 + lane;                 // row within the tile = TMEM lane
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
     const int qpos = args.ctx + m0 + row;
-    float o_acc[HD];
-#pragma unroll
-    for (int i = 0; i < HD; ++i) o_acc[i] = 0.0f;
-    float m_run = -INFINITY, l_run = 0.0f, alpha_prev = 0.0f;
+    float m_ref = -INFINITY, l_run = 0.0f;
     bool ok = true;
     uint8_t* prow0 = sP + row * 128;
+    const uint64_t sc2 = f2_pack(args.scale_log2, args.scale_log2);
     for (int j = 0; j < n_tiles; ++j) {
       if (!warp_wait_bounded(s_full, j & 1, abort_flag, args.status)) { ok = false; break; }
       tc_fence_after();
@@ -202,43 +206,41 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
         tmem_bind(rb);
         if (masked) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            mxa[i & 3] = fmaxf(mxa[i & 3], 64 * c + i < lim ? __uint_as_float(ra[i]) : -INFINITY);
-            mxa[i & 3] = fmaxf(mxa[i & 3], 64 * c + 32 + i < lim ? __uint_as_float(rb[i]) : -INFINITY);
-          }
+          for (int i = 0; i < 32; ++i)
+            mxa[i & 3] = fmax3(mxa[i & 3], 64 * c + i < lim ? __uint_as_float(ra[i]) : -INFINITY,
+                               64 * c + 32 + i < lim ? __uint_as_float(rb[i]) : -INFINITY);
         } else {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            mxa[i & 3] = fmaxf(mxa[i & 3], __uint_as_float(ra[i]));
-            mxa[i & 3] = fmaxf(mxa[i & 3], __uint_as_float(rb[i]));
-          }
+          for (int i = 0; i < 32; ++i) mxa[i & 3] = fmax3(mxa[i & 3], __uint_as_float(ra[i]), __uint_as_float(rb[i]));
         }
       }
-      const float mx = fmaxf(fmaxf(mxa[0], mxa[1]), fmaxf(mxa[2], mxa[3]));
-      const float m_new = fmaxf(m_run, mx * args.scale_log2);
-      const float alpha = (m_run == -INFINITY) ? 0.0f : ex2_approx(m_run - m_new);
-      if (j > 0) {
-        // O of the previous tile is ready: fold it in with its correction
+      const float m_tile = fmax3(fmaxf(mxa[0], mxa[1]), mxa[2], mxa[3]) * args.scale_log2;
+      float m_new = m_ref, factor = 1.0f;
+      if (m_ref == -INFINITY) {
+        m_new = m_tile;                          // every earlier exponential was 0: nothing to rescale
+      } else if (m_tile > m_ref + 8.0f) {
+        m_new = m_tile;
+        factor = ex2_approx(m_ref - m_tile);     // < 2^-8
+      }
+      if (__any_sync(0xffffffffu, factor != 1.0f)) {
+        // O holds tiles 0 .. j-1 once the P V of tile j-1 is done (j >= 1 here)
         if (!warp_wait_bounded(o_full, (j - 1) & 1, abort_flag, args.status)) { ok = false; break; }
         tc_fence_after();
 #pragma unroll
-        for (int c = 0; c < HD / 64; ++c) {
-          uint32_t ra[32], rb[32];
-          tmem_ld32_nowait(t_o + lane_off + 64 * c, ra);
-          tmem_ld32_nowait(t_o + lane_off + 64 * c + 32, rb);
+        for (int c = 0; c < HD / 32; ++c) {
+          uint32_t ra[32];
+          tmem_ld32_nowait(t_o + lane_off + 32 * c, ra);
           tmem_wait_ld(ra);
-          tmem_bind(rb);
 #pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            o_acc[64 * c + i] = fmaf(o_acc[64 * c + i], alpha_prev, __uint_as_float(ra[i]));
-            o_acc[64 * c + 32 + i] = fmaf(o_acc[64 * c + 32 + i], alpha_prev, __uint_as_float(rb[i]));
-          }
+          for (int i = 0; i < 32; ++i) ra[i] = __float_as_uint(__uint_as_float(ra[i]) * factor);
+          tmem_st32(t_o + lane_off + 32 * c, ra);
         }
-        tc_fence_before();
-        mbar_arrive(o_free);
+        tmem_wait_st();
+        l_run *= factor;
       }
       // pass 2: P = 2^(s * scale - m_new) as bf16 into the swizzled A-operand layout, 32 columns per trip
-      float ps[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+      const uint64_t negm2 = f2_pack(-m_new, -m_new);
+      uint64_t ps2[2] = {0, 0};                  // packed partial sums, two chains
 #pragma unroll
       for (int c = 0; c < TKV / 32; ++c) {
         uint32_t ra[32];
@@ -247,13 +249,14 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
         uint32_t pk[16];
 #pragma unroll
         for (int i = 0; i < 32; i += 2) {
-          float p0 = ex2_approx(fmaf(__uint_as_float(ra[i]), args.scale_log2, -m_new));
-          float p1 = ex2_approx(fmaf(__uint_as_float(ra[i + 1]), args.scale_log2, -m_new));
+          float x0, x1;
+          f2_unpack(f2_fma(f2_pack(__uint_as_float(ra[i]), __uint_as_float(ra[i + 1])), sc2, negm2), x0, x1);
+          float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
           if (masked) {
             p0 = 32 * c + i < lim ? p0 : 0.0f;
             p1 = 32 * c + i + 1 < lim ? p1 : 0.0f;
           }
-          ps[(i >> 1) & 3] += p0 + p1;
+          ps2[(i >> 1) & 1] = f2_add(ps2[(i >> 1) & 1], f2_pack(p0, p1));
           __nv_bfloat162 t = __floats2bfloat162_rn(p0, p1);
           pk[i / 2] = *reinterpret_cast<uint32_t*>(&t);
         }
@@ -266,10 +269,11 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
               make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
         }
       }
-      const float psum = (ps[0] + ps[1]) + (ps[2] + ps[3]);
-      l_run = l_run * alpha + psum;
-      m_run = m_new;
-      alpha_prev = alpha;
+      float a0, a1, b0, b1;
+      f2_unpack(ps2[0], a0, a1);
+      f2_unpack(ps2[1], b0, b1);
+      l_run += (a0 + a1) + (b0 + b1);
+      m_ref = m_new;
       tc_fence_before();
       fence_proxy_async_smem();
       mbar_arrive(s_free);
@@ -277,28 +281,25 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
     }
     if (ok && n_tiles > 0 && warp_wait_bounded(o_full, (n_tiles - 1) & 1, abort_flag, args.status)) {
       tc_fence_after();
+      const int grow = m0 + row;
+      const float inv = l_run > 0.0f ? 1.0f / l_run : 0.0f;
+      bf16* orow = args.o + (static_cast<size_t>(b) * args.rows + grow) * args.n_heads * HD + static_cast<size_t>(h) * HD;
 #pragma unroll
       for (int c = 0; c < HD / 32; ++c) {
         uint32_t ra[32];
         tmem_ld32_nowait(t_o + lane_off + 32 * c, ra);
         tmem_wait_ld(ra);
+        if (grow < args.rows) {
 #pragma unroll
-        for (int i = 0; i < 32; ++i) o_acc[32 * c + i] = fmaf(o_acc[32 * c + i], alpha_prev, __uint_as_float(ra[i]));
-      }
-      const int grow = m0 + row;
-      if (grow < args.rows) {
-        const float inv = l_run > 0.0f ? 1.0f / l_run : 0.0f;
-        bf16* orow = args.o + (static_cast<size_t>(b) * args.rows + grow) * args.n_heads * HD +
-                     static_cast<size_t>(h) * HD;
-#pragma unroll
-        for (int i = 0; i < HD; i += 8) {
-          __nv_bfloat162 t0 = __floats2bfloat162_rn(o_acc[i] * inv, o_acc[i + 1] * inv);
-          __nv_bfloat162 t1 = __floats2bfloat162_rn(o_acc[i + 2] * inv, o_acc[i + 3] * inv);
-          __nv_bfloat162 t2 = __floats2bfloat162_rn(o_acc[i + 4] * inv, o_acc[i + 5] * inv);
-          __nv_bfloat162 t3 = __floats2bfloat162_rn(o_acc[i + 6] * inv, o_acc[i + 7] * inv);
-          *reinterpret_cast<uint4*>(orow + i) =
-              make_uint4(*reinterpret_cast<uint32_t*>(&t0), *reinterpret_cast<uint32_t*>(&t1),
-                         *reinterpret_cast<uint32_t*>(&t2), *reinterpret_cast<uint32_t*>(&t3));
+          for (int i = 0; i < 32; i += 8) {
+            __nv_bfloat162 t0 = __floats2bfloat162_rn(__uint_as_float(ra[i]) * inv, __uint_as_float(ra[i + 1]) * inv);
+            __nv_bfloat162 t1 = __floats2bfloat162_rn(__uint_as_float(ra[i + 2]) * inv, __uint_as_float(ra[i + 3]) * inv);
+            __nv_bfloat162 t2 = __floats2bfloat162_rn(__uint_as_float(ra[i + 4]) * inv, __uint_as_float(ra[i + 5]) * inv);
+            __nv_bfloat162 t3 = __floats2bfloat162_rn(__uint_as_float(ra[i + 6]) * inv, __uint_as_float(ra[i + 7]) * inv);
+            *reinterpret_cast<uint4*>(orow + 32 * c + i) =
+                make_uint4(*reinterpret_cast<uint32_t*>(&t0), *reinterpret_cast<uint32_t*>(&t1),
+                           *reinterpret_cast<uint32_t*>(&t2), *reinterpret_cast<uint32_t*>(&t3));
+          }
         }
       }
     }
