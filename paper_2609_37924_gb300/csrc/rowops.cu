@@ -105,6 +105,50 @@ __global__ void rmsnorm_kernel(const float* __restrict__ x, int M, int d, const 
   }
 }
 
+// out = x / sqrt(mean(x^2) + eps) * gain for d = 256 * NCH: one warp per row,
+// the row held in registers (8 consecutive elements per lane and chunk), one
+// 16-byte load of 8 gains and one 16-byte store of 8 bf16 outputs per chunk.
+// Needs 16-byte aligned x, out (ldo % 8 == 0) and bf16 gains.
+template <int NCH>
+__global__ void __launch_bounds__(WPB * 32) rmsnorm_reg_kernel(const float* __restrict__ x, int M,
+                                                               const bf16* __restrict__ gain, float eps,
+                                                               bf16* __restrict__ out, int ldo,
+                                                               const int32_t* __restrict__ rows_idx) {
+  constexpr int d = 256 * NCH;
+  const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (m >= M) return;
+  const float* xr = x + static_cast<size_t>(rows_idx ? rows_idx[m] : m) * d;
+  float v[NCH][8];
+  float ss = 0.0f;
+#pragma unroll
+  for (int c = 0; c < NCH; ++c) {
+    const int j = (c * 32 + lane) * 8;
+    const float4 a = *reinterpret_cast<const float4*>(xr + j);
+    const float4 b = *reinterpret_cast<const float4*>(xr + j + 4);
+    v[c][0] = a.x; v[c][1] = a.y; v[c][2] = a.z; v[c][3] = a.w;
+    v[c][4] = b.x; v[c][5] = b.y; v[c][6] = b.z; v[c][7] = b.w;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) ss = fmaf(v[c][i], v[c][i], ss);
+  }
+  ss = warp_sum(ss);
+  const float inv = rsqrtf(ss / static_cast<float>(d) + eps);
+  bf16* orow = out + static_cast<size_t>(m) * ldo;
+#pragma unroll
+  for (int c = 0; c < NCH; ++c) {
+    const int j = (c * 32 + lane) * 8;
+    const uint4 graw = *reinterpret_cast<const uint4*>(gain + j);
+    const __nv_bfloat162* g2 = reinterpret_cast<const __nv_bfloat162*>(&graw);
+    uint32_t packed[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float2 g = __bfloat1622float2(g2[q]);
+      __nv_bfloat162 t = __floats2bfloat162_rn(v[c][2 * q] * inv * g.x, v[c][2 * q + 1] * inv * g.y);
+      packed[q] = *reinterpret_cast<uint32_t*>(&t);
+    }
+    *reinterpret_cast<uint4*>(orow + j) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+  }
+}
+
 __device__ __forceinline__ void row_mean_var(const float* xr, int d, int lane, float& mean, float& rstd, float eps) {
   float s = 0.0f;
   for (int j = lane * 4; j < d; j += 128) {
@@ -245,6 +289,20 @@ const char* rmsnorm_rows(const float* x, int M, int d, const void* gain, int w_b
     else
       rmsnorm_block_kernel<float><<<M, 256, 0, s>>>(x, d, gain, w_bf16, eps, out, ldo, rows_idx);
     return err();
+  }
+  const bool vec = act_bf16 && w_bf16 && ldo % 8 == 0 &&
+                   ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(out) | reinterpret_cast<uintptr_t>(gain)) & 15) == 0;
+  if (vec) {
+    const bf16* g = static_cast<const bf16*>(gain);
+    bf16* o = static_cast<bf16*>(out);
+    switch (d) {
+      case 256: rmsnorm_reg_kernel<1><<<rows_grid(M), WPB * 32, 0, s>>>(x, M, g, eps, o, ldo, rows_idx); return err();
+      case 512: rmsnorm_reg_kernel<2><<<rows_grid(M), WPB * 32, 0, s>>>(x, M, g, eps, o, ldo, rows_idx); return err();
+      case 768: rmsnorm_reg_kernel<3><<<rows_grid(M), WPB * 32, 0, s>>>(x, M, g, eps, o, ldo, rows_idx); return err();
+      case 1024: rmsnorm_reg_kernel<4><<<rows_grid(M), WPB * 32, 0, s>>>(x, M, g, eps, o, ldo, rows_idx); return err();
+      case 2048: rmsnorm_reg_kernel<8><<<rows_grid(M), WPB * 32, 0, s>>>(x, M, g, eps, o, ldo, rows_idx); return err();
+      default: break;
+    }
   }
   if (act_bf16)
     rmsnorm_kernel<bf16><<<rows_grid(M), WPB * 32, 0, s>>>(x, M, d, gain, w_bf16, eps, out, ldo, rows_idx);
