@@ -46,6 +46,8 @@ def parse():
                     help="override reverse steps per block (short runs for launch-list profiles)")
     ap.add_argument("--G", type=int, default=None, help="override the generation length (short profiling runs)")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
+    ap.add_argument("--fusion-off", action="store_true",
+                    help="with --sweep-workloads: run the workloads with the fusion disabled (App. D naive reuse)")
     ap.add_argument("--sweep-workloads", default=None,
                     help="comma list of workloads: print one JSON line per (workload, batch, K) instead")
     ap.add_argument("--sweep-batches", default="", help="batches for the 'sweep' workload (default 1,8,32,128)")
@@ -384,8 +386,12 @@ def workload_sweep(args):
     from paper_2609_37924_gb300 import TadmModel, upload_weights
 
     torch.cuda.set_device(0)
+    peaks = load_peaks()
+    peak = peaks["bf16_tflops_sustained"] if peaks else 1700.0
     for name in args.sweep_workloads.split(","):
-        base = wl.get_workload(name)
+        # --fusion-off: the same workload with the fusion disabled (the naive
+        # stale-anchor reuse baseline of App. D), for the fusion-cost ablation
+        base = wl.get_workload(name, **({"model_fusion": "none"} if args.fusion_off else {}))
         batches = [base.batch]
         if name == "sweep":
             batches = [int(b) for b in (args.sweep_batches or "1,8,32,128").split(",")]
@@ -394,7 +400,7 @@ def workload_sweep(args):
         dev_w = upload_weights(m, wl.make_weights(m, seed=base.seed))
         t_w = time.perf_counter() - t0
         for B in batches:
-            w = wl.get_workload(name, batch=B)
+            w = wl.get_workload(name, batch=B, **({"model_fusion": "none"} if args.fusion_off else {}))
             bl = w.block_len
             tm = TadmModel(m, dev_w, max_batch=B, max_rows=max(w.prompt_len, bl) if bl else w.total_len,
                            max_ctx=w.total_len if bl else 0)
@@ -415,10 +421,20 @@ def workload_sweep(args):
                 ms = e0.elapsed_time(e1) / args.steps
                 c = tm.tadm_get_counters()
                 res[K] = B * w.gen_len / (ms / 1000.0)
-                print(json.dumps({"workload": name, "batch": B, "K": K, "tokens_per_s": res[K], "ms_per_generation": ms,
+                # one more generation with every GEMM launch bracketed by events (up to 60000 launches)
+                tm.tadm_probe_enable(60000)
+                tm.tadm_generate(p, out, w.gen_len, w.steps_per_block, K, bl)
+                n_l, g_ms, g_fl = tm.tadm_probe_read()
+                tm.tadm_probe_enable(0)
+                tm.tadm_sync_status()
+                g_tf = g_fl / (g_ms / 1000.0) / 1e12 if g_ms > 0 else None
+                print(json.dumps({"workload": name, "fusion": m.fusion, "batch": B, "K": K, "tokens_per_s": res[K],
+                                  "ms_per_generation": ms,
                                   "vs_K1": res[K] / res[1] if 1 in res else None, "anchor_calls": c["anchor_calls"],
                                   "denoise_steps": c["denoise_steps"], "commit_passes": c["commit_passes"],
-                                  "gpu_launches": c["kernel_launches"], "weights_s": round(t_w, 1)}), flush=True)
+                                  "gpu_launches": c["kernel_launches"], "weights_s": round(t_w, 1),
+                                  "gemm": {"tflops": g_tf, "frac_of_sustained": (g_tf / peak) if g_tf else None,
+                                           "launches_probed": n_l, "ms_probed": g_ms}}), flush=True)
             tm.close()
             del tm
             torch.cuda.empty_cache()

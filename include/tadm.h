@@ -65,7 +65,10 @@ typedef enum {
  *              u = [LN(c); LN(h)], g = sigmoid(W_g u + b_g),
  *              Delta = W_2 GELU(W_1 u + b_1) + b_2, h~ = LN(h + g * Delta);
  *           1 = paired attention with cached shallow state (App. C.1,
- *              Eqs. paired-attention-difference, stale-anchor-fusion-app).
+ *              Eqs. paired-attention-difference, stale-anchor-fusion-app);
+ *           2 = off: the denoiser reads the cached anchor output itself,
+ *              h~ = h' (the naive stale-anchor reuse baseline of App. D,
+ *              Table naive-vs-tadm-posttrain); no fusion weights.
  *  fusion_rank, fusion_heads: r and the mixer heads of fusion 1.
  *  dtype:   0 = fp32 weights and activations, 1 = bf16 weights and GEMM
  *           operands (fp32 accumulation, fp32 residual stream).
@@ -128,7 +131,7 @@ TADM_API tadm_status tadm_workspace_size(const tadm_handle* h, size_t* bytes);
 TADM_API tadm_status tadm_bind_workspace(tadm_handle* h, void* dev_ptr, size_t bytes);
 
 /* Bytes of one anchor cache for `batch` sequences of `rows` canvas rows
- * (fusion 0: h, fp32 [batch*rows, d]; fusion 1: H0, s_C, s_H, Z0, U and
+ * (fusion 0 and 2: h, fp32 [batch*rows, d]; fusion 1: H0, s_C, s_H, Z0, U and
  * phi(Z0, U)).  Caller-allocated, device, 256-byte aligned. */
 TADM_API tadm_status tadm_cache_size(const tadm_handle* h, int batch, int rows, size_t* bytes);
 

@@ -13,6 +13,9 @@ What it computes (paper section / equation it follows):
     - gated residual MLP (TADM:Pretraining): App. C.2;
     - paired attention with cached shallow state (TADM:Post-train): App. C.1,
       Eqs. (paired-attention-difference) and (stale-anchor-fusion-app).
+  Fusion off ("none"): the naive stale-anchor reuse baseline of App. D
+  (Table naive-vs-tadm-posttrain): Alg. 1 with the fusion disabled, so the
+  denoiser receives the cached anchor output itself, h~ = h'.
 * Anchor-cache inference loop: Alg. 1 (Anchor-Cache Inference), §3.3;
   transformer-layer cost: Eq. (anchor-cache-compute).
 * Masked-diffusion reverse step with zero-masking and carry-over unmasking:
@@ -350,6 +353,8 @@ class Oracle:
     def fuse(self, c: np.ndarray, cache) -> np.ndarray:
         if self.m.fusion == "paired_attn":
             return self.fusion_paired_attn(c, cache)
+        if self.m.fusion == "none":              # App. D naive reuse: D reads the stale h' as is
+            return cache["h"].copy()
         return self.fusion_gated_mlp(c, cache["h"])
 
     # -- sessions (block mode context) ----------------------------------------

@@ -39,7 +39,7 @@ bool valid_config(const tadm_config* c, std::string* why) {
   if (c->head_dim % 2) return fail("head_dim must be even");
   if (c->glu != 0 && c->glu != 1) return fail("glu must be 0 or 1");
   if (c->n_shared < 0 || c->n_anchor < 0 || c->n_denoise < 0) return fail("layer counts must be >= 0");
-  if (c->fusion != 0 && c->fusion != 1) return fail("fusion must be 0 or 1");
+  if (c->fusion < 0 || c->fusion > 2) return fail("fusion must be 0, 1 or 2");
   if (c->fusion == 1 && (c->fusion_rank <= 0 || c->fusion_heads <= 0 || c->fusion_rank % c->fusion_heads))
     return fail("fusion_rank must be a positive multiple of fusion_heads");
   if (c->dtype != 0 && c->dtype != 1) return fail("dtype must be 0 (fp32) or 1 (bf16)");
@@ -79,7 +79,7 @@ Inventory inventory(const tadm_config* c) {
     add("fusion.b2", d, 1);
     add("fusion.ln_out.w", d, 1);
     add("fusion.ln_out.b", d, 1);
-  } else {
+  } else if (c->fusion == 1) {
     const int64_t r = c->fusion_rank;
     add("fusion.wc", r, d);
     add("fusion.wh", r, d);
@@ -170,7 +170,7 @@ tadm_status fail(tadm_handle* h, tadm_status s, const char* fmt, ...) {
 
 size_t cache_bytes(const tadm_config& c, int batch, int rows) {
   const size_t M = static_cast<size_t>(batch) * rows;
-  if (c.fusion == 0) return align_up(M * c.d_model * 4, 256);
+  if (c.fusion != 1) return align_up(M * c.d_model * 4, 256);   // h only (fusion 0 and 2)
   const size_t r = c.fusion_rank;
   // H0 [M,d] | sC [M] | sH [M] | Z0 [M,r] | U [M,r] | phi0 [M,r]   (fp32)
   return align_up(M * c.d_model * 4, 256) + 2 * align_up(M * 4, 256) + 3 * align_up(M * r * 4, 256);
@@ -184,7 +184,7 @@ CacheView cache_view(const tadm_config& c, void* base, int batch, int rows) {
   const size_t M = static_cast<size_t>(batch) * rows;
   char* p = static_cast<char*>(base);
   v.h = reinterpret_cast<float*>(p);
-  if (c.fusion == 0) return v;
+  if (c.fusion != 1) return v;
   const size_t r = c.fusion_rank;
   p += align_up(M * c.d_model * 4, 256);
   v.sC = reinterpret_cast<float*>(p);
@@ -231,7 +231,7 @@ void layout(tadm_handle* h) {
     f.f_g = take(M * d * es);
     f.f_hid = take(M * 4 * d * es);
     f.f_pre = take(M * d * 4);
-  } else {
+  } else if (c.fusion == 1) {
     const size_t r = c.fusion_rank;
     f.pa_z = take(M * r * 4);
     f.pa_j = take(M * 4 * r * es);
@@ -437,6 +437,12 @@ tadm_status run_fusion(tadm_handle* h, int B, int R, const void* cache, cudaStre
   CacheView cv = cache_view(c, const_cast<void*>(cache), B, R);
   const float* cbuf = h->at<float>(h->off.c);
   float* x = h->at<float>(h->off.x);
+  if (c.fusion == 2) {
+    // fusion off (the naive stale-anchor reuse of App. D): D reads h' itself
+    if (cudaMemcpyAsync(x, cv.h, static_cast<size_t>(M) * d * 4, cudaMemcpyDeviceToDevice, s) != cudaSuccess)
+      return fail(h, TADM_ERR_CUDA, "copy h -> x failed");
+    return TADM_OK;
+  }
   if (c.fusion == 0) {
     // u = [LN(c); LN(h)];  [g | a] = [sigmoid(W_g u + b_g) | GELU(W_1 u + b_1)];
     // pre = h + g * (W_2 a + b_2);  h~ = LN(pre)                        (App. C.2)
@@ -696,9 +702,19 @@ tadm_status tadm_create(const tadm_config* cfg, const void* const* weights, int 
     L.wdown = weights[i++];
     h->layers.push_back(L);
   }
-  for (int f = 0; f < 10; ++f) h->fw[f] = weights[i++];
+  // fusion tensors (10 for fusion 0 and 1, none for fusion 2), in inventory order
+  const int n_fusion = static_cast<int>(inv.names.size()) - i - (c.tied_lm_head ? 1 : 2);
+  if (n_fusion < 0 || n_fusion > static_cast<int>(sizeof(h->fw) / sizeof(h->fw[0]))) {
+    delete h;
+    return TADM_ERR_INVALID_ARG;
+  }
+  for (int f = 0; f < n_fusion; ++f) h->fw[f] = weights[i++];
   h->final_norm = weights[i++];
   h->lm_head = c.tied_lm_head ? h->embed : weights[i++];
+  if (i != static_cast<int>(inv.names.size())) {
+    delete h;
+    return TADM_ERR_INVALID_ARG;
+  }
   layout(h);
   *out = h;
   return TADM_OK;

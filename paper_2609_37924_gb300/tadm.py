@@ -120,7 +120,7 @@ def make_config(model) -> tadm_config:
     return tadm_config(
         vocab=model.vocab, d_model=model.d_model, n_heads=model.n_heads, n_kv_heads=model.n_kv_heads,
         head_dim=model.head_dim, ffn=model.ffn, glu=1 if model.glu == "geglu" else 0, n_shared=model.n_shared,
-        n_anchor=model.n_anchor, n_denoise=model.n_denoise, fusion=1 if model.fusion == "paired_attn" else 0,
+        n_anchor=model.n_anchor, n_denoise=model.n_denoise, fusion={"gated_mlp": 0, "paired_attn": 1, "none": 2}[model.fusion],
         fusion_rank=model.fusion_rank, fusion_heads=model.fusion_heads, dtype=1 if model.dtype == "bf16" else 0,
         tied_lm_head=int(bool(model.tied_lm_head)), norm_eps=model.norm_eps, rope_theta=model.rope_theta)
 

@@ -78,9 +78,12 @@ def test_layer_cost_matches_paper_tables(lib):
             assert lib.tadm_layer_cost(2, 20, 8, T, K) == O.layer_cost(2, 20, 8, T, K)
 
 
-@pytest.mark.parametrize("name", list(wl.WORKLOADS))
+@pytest.mark.parametrize("name", list(wl.WORKLOADS) + ["small+fusion_off"])
 def test_weight_inventory_matches_the_generator(lib, name):
-    m = wl.WORKLOADS[name].model
+    if name.endswith("+fusion_off"):
+        m = wl.ModelConfig(**{**wl.WORKLOADS[name.split("+")[0]].model.__dict__, "fusion": "none"})
+    else:
+        m = wl.WORKLOADS[name].model
     inv = lib.tadm_weight_inventory(lib.make_config(m))
     specs = wl.weight_specs(m)
     assert [n for n, _ in inv] == [s.name for s in specs]
@@ -99,6 +102,9 @@ def test_invalid_configs_are_rejected(lib):
         if over.get("glu"):
             cfg.glu = 7
         assert so.tadm_weight_count(ctypes.byref(cfg)) == -1
+    cfg = lib.make_config(base)
+    cfg.fusion = 3                                  # 0, 1, 2 are the only fusion modes
+    assert so.tadm_weight_count(ctypes.byref(cfg)) == -1
     h = ctypes.c_void_p()
     cfg = lib.make_config(base)
     assert so.tadm_create(ctypes.byref(cfg), None, 0, 1, 1, 0, ctypes.byref(h)) == 1   # no weights

@@ -163,6 +163,39 @@ def test_bf16_teacher_forced_step_stale_cache(T, glu):
     agg.check()
 
 
+def test_fusion_off_stale_reuse_parity(T):
+    """Fusion off (App. D naive stale reuse): the denoiser reads the cached h'
+    itself.  bf16 teacher-forced step on a stale cache; fp32 full generations
+    (single block and block mode) against the oracle."""
+    m = wl.ModelConfig(**SMALL_BF16, fusion="none")
+    w = wl.Workload("t", m, batch=2, prompt_len=40, gen_len=160, steps_per_block=16, K=4)
+    B, R = 2, 200
+    tm, o = setup(T, m, B, R)
+    z0 = wl.random_canvas(w, B, R, 0.8, seed=7, start=40)
+    z1 = wl.random_canvas(w, B, R, 0.5, seed=8, start=40)
+    cache = tm.new_cache(B, R)
+    tm.tadm_reset(B)
+    tm.tadm_anchor_forward(torch.from_numpy(z0).cuda(), 16, cache)
+    sess = o.new_session(B)
+    cache_o = o.anchor_forward(sess, z0)
+    g = gpu_step(tm, z1, 14, 16, 160, cache, want_fused=True)
+    assert rel_l2(g["fused"], np.stack([c["h"] for c in cache_o])) < 1e-2
+    agg = Agreement()
+    check_step(o, sess, z1, cache_o, g, 2, 16, 160, tol=2e-2, min_agree=0.95, agg=agg)
+    agg.check()
+    tiny = wl.WORKLOADS["tiny"]
+    mf = wl.ModelConfig(**{**tiny.model.__dict__, "fusion": "none"})
+    prompts = wl.make_prompts(tiny)
+    for bl in (0, 32):
+        tm2, o2 = setup(T, mf, 1, tiny.prompt_len if bl else tiny.total_len, max_ctx=tiny.total_len if bl else 0,
+                        affine_std=0.0)
+        got = tm2.generate(torch.from_numpy(prompts).cuda(), tiny.gen_len, 8 if bl else tiny.steps_per_block, 2,
+                           bl).cpu().numpy()
+        ref = o2.generate(prompts, tiny.gen_len, 8 if bl else tiny.steps_per_block, 2, block_len=bl)
+        assert float(np.mean(got == ref)) >= 0.99, bl
+        tm2.close()
+
+
 def test_generate_k1_equals_step_loop_and_counts(T):
     m = wl.ModelConfig(**SMALL_BF16)
     w = wl.Workload("t", m, batch=2, prompt_len=16, gen_len=48, steps_per_block=8, K=1)

@@ -445,3 +445,45 @@ def test_tied_head_reads_the_embedding():
     E = o.W("embed")
     logits = o.lm_head(E[:127])
     assert np.array_equal(np.argmax(logits, -1), np.arange(127))
+
+
+# --------------------------------------------------------------------- fusion off (App. D)
+def test_fusion_off_is_one_backbone_at_a_refresh():
+    """Fusion off (the naive stale-reuse baseline of App. D): at a refresh step
+    D reads A's output unchanged, so anchor (a layers) + denoiser (b layers)
+    is one stack of a + b layers.  Rebuild it as a model with no anchor layers
+    whose denoiser holds the same a + b layers, and compare logits exactly."""
+    o = tiny_oracle(fusion="none", n_anchor=2, n_denoise=2)
+    m2 = tiny_model(fusion="none", n_anchor=0, n_denoise=4)
+    w2 = {}
+    for k, v in o._raw.items():
+        if k.startswith("anchor."):
+            w2["denoise." + k[len("anchor."):]] = v
+        elif k.startswith("denoise."):
+            i, rest = k[len("denoise."):].split(".", 1)
+            w2[f"denoise.{int(i) + 2}.{rest}"] = v
+        else:
+            w2[k] = v
+    assert set(w2) == {s.name for s in wl.weight_specs(m2)}
+    o2 = O.Oracle(m2, w2)
+    z = rng.integers(0, o.m.vocab - 1, (2, 7)).astype(np.int32)
+    z[:, 3:] = o.mask_id
+    l1 = o.denoise_logits(o.new_session(2), z, o.anchor_forward(o.new_session(2), z))
+    l2 = o2.denoise_logits(o2.new_session(2), z, o2.anchor_forward(o2.new_session(2), z))
+    np.testing.assert_array_equal(l1, l2)
+
+
+def test_fusion_off_ignores_the_current_canvas():
+    """With fusion off the denoiser sees only the cached h': logits between
+    refreshes do not depend on the current canvas; with the gated-MLP fusion
+    they do (the current state enters through c)."""
+    for fusion, same in (("none", True), ("gated_mlp", False)):
+        o = tiny_oracle(fusion=fusion)
+        z0 = rng.integers(0, o.m.vocab - 1, (2, 6)).astype(np.int32)
+        z0[:, 2:] = o.mask_id
+        z1 = z0.copy()
+        z1[:, 2:4] = rng.integers(0, o.m.vocab - 1, (2, 2))
+        cache = o.anchor_forward(o.new_session(2), z0)
+        l0 = o.denoise_logits(o.new_session(2), z0, cache)
+        l1 = o.denoise_logits(o.new_session(2), z1, cache)
+        assert np.array_equal(l0, l1) == same

@@ -117,7 +117,7 @@ class ModelConfig:
     n_shared: int = 0            # L_S: transformer layers inside S (embedding always)
     n_anchor: int = 4            # L_A
     n_denoise: int = 2           # L_D
-    fusion: str = "gated_mlp"    # "gated_mlp" (Pretraining) | "paired_attn" (Post-train)
+    fusion: str = "gated_mlp"    # "gated_mlp" (Pretraining) | "paired_attn" (Post-train) | "none" (stale reuse, no fusion)
     fusion_rank: int = 256       # r of the paired-attention fusion
     fusion_heads: int = 4
     dtype: str = "bf16"          # "f32" | "bf16"
@@ -239,7 +239,7 @@ def weight_specs(m: ModelConfig) -> List[TensorSpec]:
             TensorSpec("fusion.bg", (1,), "bias"),
             TensorSpec("fusion.wup", (d, r), "matrix"),
         ]
-    else:
+    elif m.fusion != "none":
         raise ValueError(m.fusion)
     specs.append(TensorSpec("final_norm", (d,), "gain"))
     if not m.tied_lm_head:
