@@ -15,7 +15,8 @@
 //   own one query row per thread: masked softmax on the S row, P as bf16
 //   into the 128-byte-swizzled operand layout; O accumulates in TMEM across
 //   key tiles, rescaled only when a row's running max grows by more than 2^8.
-// bf16, short rows (attn_bf16_kernel): mma.sync m16n8k16 flash attention.
+// bf16, short rows (attn_bf16_kernel): mma.sync m16n8k16 flash attention;
+//   a CTA takes 64 rows of all query heads of one KV group (one K/V read).
 // fp32: one warp per query row on the CUDA cores.
 #include <cudaTypedefs.h>
 #include <mutex>
@@ -409,21 +410,30 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const bf16* __restrict__
   bf16* sK = sQ + AM * LD;          // [2][AN][LD]
   bf16* sV = sK + 2 * AN * LD;      // [2][HD][LDV]
 
+  // One CTA serves AM "virtual rows" v = (query head within the KV group) *
+  // rows + row of one (batch, KV head): the group's query heads share every
+  // K / V tile, which is read once for all of them.
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int m0 = blockIdx.x * AM, h = blockIdx.y, b = blockIdx.z;
-  const int hk = h / (n_heads / n_kv_heads);
-  const bf16* qb = q + (static_cast<size_t>(b) * n_heads + h) * rows * HD;
+  const int m0 = blockIdx.x * AM, hk = blockIdx.y, b = blockIdx.z;
+  const int group = n_heads / n_kv_heads, n_virt = group * rows;
   const bf16* kb = k + (static_cast<size_t>(b) * n_kv_heads + hk) * kv_stride * HD;
   const bf16* vb = vt + (static_cast<size_t>(b) * n_kv_heads + hk) * HD * kv_stride;
   const int kv_len = ctx + rows;
-  const int kv_end = causal ? min(kv_len, ctx + min(m0 + AM, rows)) : kv_len;
+  // causal: the last key any of this CTA's rows may see
+  const int v_last = min(m0 + AM, n_virt) - 1;
+  const int r_max = (m0 / rows != v_last / rows) ? rows - 1 : v_last % rows;
+  const int kv_end = causal ? min(kv_len, ctx + r_max + 1) : kv_len;
   const int n_tiles = (kv_end + AN - 1) / AN;
+  // global row of virtual row v in q [B, Hq, rows, hd]
+  auto q_row = [&](int v) {
+    return (static_cast<size_t>(b) * n_heads + hk * group + v / rows) * rows + v % rows;
+  };
 
   constexpr int CPR = HD / 8;  // 16-byte chunks per Q / K row
   for (int i = tid; i < AM * CPR; i += 128) {
     const int r = i / CPR, c = i % CPR;
-    const bool ok = m0 + r < rows;
-    cp_async16(sQ + r * LD + c * 8, qb + static_cast<size_t>(ok ? m0 + r : 0) * HD + c * 8, ok);
+    const bool ok = m0 + r < n_virt;
+    cp_async16(sQ + r * LD + c * 8, q + (ok ? q_row(m0 + r) : 0) * HD + c * 8, ok);
   }
   auto load_kv = [&](int t, int buf) {
     const int n0 = t * AN;
@@ -456,7 +466,9 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const bf16* __restrict__
   for (int j = 0; j < HD / 8; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.0f;
   float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.0f, 0.0f};
   const int g = lane >> 2, t4 = lane & 3;
-  const int qpos0 = ctx + m0 + warp * 16 + g;
+  // query positions of this lane's two fragment rows (virtual rows v and v + 8)
+  const int v0 = m0 + warp * 16 + g;
+  const int qpos_r[2] = {ctx + v0 % rows, ctx + (v0 + 8) % rows};
   uint32_t qf[HD / 16][4];
 
   for (int t = 0; t < n_tiles; ++t) {
@@ -494,7 +506,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const bf16* __restrict__
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         const int key = n0 + j * 8 + 2 * t4 + (e & 1);
-        const int qp = qpos0 + (e >> 1) * 8;
+        const int qp = qpos_r[e >> 1];
         const bool ok = key < kv_end && (!causal || key < ctx || key <= qp);
         s[j][e] = ok ? s[j][e] * scale_log2 : -INFINITY;
         tmax[e >> 1] = fmaxf(tmax[e >> 1], s[j][e]);
@@ -556,8 +568,9 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const bf16* __restrict__
   const size_t ldo = static_cast<size_t>(n_heads) * HD;
 #pragma unroll
   for (int r = 0; r < 2; ++r) {
-    const int row = m0 + warp * 16 + g + r * 8;
-    if (row >= rows) continue;
+    const int v = v0 + r * 8;
+    if (v >= n_virt) continue;
+    const int row = v % rows, h = hk * group + v / rows;
     const float inv = lrow[r] > 0.0f ? 1.0f / lrow[r] : 0.0f;
     bf16* orow = o + (static_cast<size_t>(b) * rows + row) * ldo + static_cast<size_t>(h) * HD;
 #pragma unroll
@@ -617,7 +630,8 @@ cudaError_t launch_bf16(const AttnCall& a, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     attr = true;
   }
-  dim3 grid((a.rows + AM - 1) / AM, a.n_heads, a.batch);
+  const int n_virt = (a.n_heads / a.n_kv_heads) * a.rows;
+  dim3 grid((n_virt + AM - 1) / AM, a.n_kv_heads, a.batch);
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(HD));
   attn_bf16_kernel<HD><<<grid, 128, smem, s>>>(static_cast<const bf16*>(a.q), static_cast<const bf16*>(a.k),
                                                static_cast<const bf16*>(a.v), static_cast<bf16*>(a.o), a.n_heads,

@@ -625,7 +625,12 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
   a.splits = 1;
   a.kb_per_split = kblocks;
   a.ldp = a.n_tiles_n * BN;
-  if (g.split_buf && tiles * 3 < g_num_sms * 2 && kblocks >= 8) {
+  // CTA-pair tiles that keep >= 40% of the SMs busy beat split-K: no fp32
+  // partials, no reduction launches
+  const int pair_units = ((g.M + 2 * BM - 1) / (2 * BM)) * a.n_tiles_n;
+  const bool pair_ok = g_pair_mma && g.M > BM;
+  const bool pairs_fill = pair_ok && 2 * pair_units * 5 >= g_num_sms * 2;
+  if (g.split_buf && !pairs_fill && tiles * 3 < g_num_sms * 2 && kblocks >= 8) {
     int sp = std::min(std::min(g_num_sms / tiles, kblocks / 4), 16);
     const size_t per = static_cast<size_t>(g.M) * a.ldp * sizeof(float);
     while (sp > 1 && sp * per > g.split_bytes) --sp;
@@ -639,8 +644,7 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
   }
   // CTA pairs (256 x 256 tiles, cta_group::2) for every unsplit GEMM of more
   // than 128 rows: the same SMs as 128 x 256 tiles, less operand traffic each
-  const int pair_units = ((g.M + 2 * BM - 1) / (2 * BM)) * a.n_tiles_n;
-  if (g_pair_mma && a.splits == 1 && g.M > BM) {
+  if (pair_ok && a.splits == 1) {
     CUtensorMap tbh;
     if (!make_map(&tbh, g.B, b_rows, g.K, g.ldb, BN / 2)) return "tensor map (B, half tiles) encode failed";
     cudaError_t e;
