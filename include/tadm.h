@@ -213,18 +213,20 @@ typedef struct {
 } tadm_counters;
 TADM_API tadm_status tadm_get_counters(const tadm_handle* h, tadm_counters* out);
 
-/* GEMM timing probe.  While enabled, every GEMM launch of the handle is
- * bracketed by two CUDA events recorded on its stream (a pool of up to
- * `max_launches` pairs, created here), and its algorithmic work 2*M*N*K is
- * noted.  tadm_probe_read waits for the last event and returns the number
- * of bracketed launches, their summed duration (ms) and summed FLOPs, then
- * clears the records.  tadm_probe_enable(h, 0) frees the events. */
+/* Timing probe.  While enabled, every GEMM, attention and normalisation
+ * launch of the handle is bracketed by two CUDA events recorded on its
+ * stream (a pool of up to `max_launches` pairs, created here), and the
+ * algorithmic work of GEMMs (2*M*N*K) and attention (4*rows*keys*hd per
+ * head) is noted.  tadm_probe_read waits for the last event and returns the
+ * number of bracketed GEMM launches, their summed duration (ms) and summed
+ * FLOPs, then clears the records.  tadm_probe_enable(h, 0) frees the events. */
 TADM_API tadm_status tadm_probe_enable(tadm_handle* h, int max_launches);
 TADM_API tadm_status tadm_probe_read(tadm_handle* h, int64_t* launches, double* total_ms, double* total_flops);
-/* The same records split by GEMM epilogue kind (0 plain, 1 residual, 2 QKV +
+/* The records split by kind: GEMM epilogues 0 plain, 1 residual, 2 QKV +
  * RoPE, 3 GLU, 4 fusion gate/hidden, 5 fusion output, 6 output head,
- * 7..10 paired-attention fusion): arrays of n_kinds entries.  Call before
- * tadm_probe_read, which clears the records. */
+ * 7..10 paired-attention fusion; 11 attention; 12 RMSNorm / LayerNorm
+ * launches.  Arrays of n_kinds entries.  Call before tadm_probe_read, which
+ * clears the records. */
 TADM_API tadm_status tadm_probe_breakdown(tadm_handle* h, int n_kinds, int64_t* launches, double* ms,
                                           double* flops);
 

@@ -19,6 +19,7 @@
 //   a CTA takes 64 rows of all query heads of one KV group (one K/V read).
 // fp32: one warp per query row on the CUDA cores.
 #include <cudaTypedefs.h>
+#include <algorithm>
 #include <mutex>
 
 #include "kernels.h"
@@ -27,36 +28,49 @@ namespace tadm {
 namespace {
 
 // =============================================================== tcgen05 path
-constexpr int TQ = 128;      // query rows per CTA
-constexpr int TKV = 128;     // keys per tile
+constexpr int TQ = 128;      // virtual query rows per CTA (see AttnTcArgs)
 
-template <int HD>
+// TKV keys per tile: 128, or 64 for hd 128 with few rows, which lets two CTAs
+// share an SM.
+template <int HD, int TKV>
 struct AttnTcCfg {
-  static constexpr int Q_BYTES = HD / 64 * 16384;       // HD/64 swizzle atoms of 128 x 64
-  static constexpr int K_BYTES = HD / 64 * 16384;
-  static constexpr int V_BYTES = 2 * HD * 128;           // two 64-key atoms of HD rows
-  static constexpr int P_BYTES = 2 * 16384;              // two 64-key atoms of 128 rows
+  static constexpr int Q_BYTES = HD / 64 * 16384;       // HD/64 swizzle atoms of 128 rows x 64
+  static constexpr int K_BYTES = HD / 64 * TKV * 128;   // HD/64 atoms of TKV keys x 64
+  static constexpr int V_BYTES = TKV / 64 * HD * 128;   // TKV/64 atoms of HD rows x 64 keys
+  static constexpr int P_BYTES = TKV / 64 * 16384;      // TKV/64 atoms of 128 rows x 64 keys
   static constexpr int STAGES = 2;
-  // hd 64 runs two CTAs per SM, which leaves no room for re-alignment slack:
-  // the kernel then requires (and checks) a 1024-byte aligned dynamic base.
-  static constexpr int SLACK = HD == 64 ? 0 : 1024;
+  static constexpr int MIN_BLOCKS = (HD == 64 || TKV == 64) ? 2 : 1;
+  // two CTAs per SM leave no room for re-alignment slack: the kernel then
+  // requires (and checks) a 1024-byte aligned dynamic base
+  static constexpr int SLACK = MIN_BLOCKS == 2 ? 0 : 1024;
   static constexpr int SMEM = SLACK + Q_BYTES + STAGES * (K_BYTES + V_BYTES) + P_BYTES + 256;
-  static constexpr int TMEM_COLS = 256;                  // S: [0,128), O tile: [128, 128+HD)
-  static constexpr int MIN_BLOCKS = HD == 64 ? 2 : 1;
+  static constexpr int TMEM_COLS = 256;                  // S: [0, TKV), O: [TKV, TKV + HD)
+  static_assert(TKV + HD <= TMEM_COLS, "TMEM columns");
 };
 
+// Virtual rows: the CTA at blockIdx = (tile + n_vtiles * split, kv head hk,
+// batch b) serves virtual rows v = 128 * tile + 0..127, where v = (query head
+// within hk's group) * rows + row, so that all query heads of a KV group read
+// each K / V tile once, and short canvases fill the 128-row MMA.  With
+// `splits` > 1 the keys are cut into splits ranges of tiles_per_split tiles;
+// each CTA writes its unnormalised O (fp32), reference max and sum for its
+// range to part_o / part_ml, and attn_combine_kernel merges them.
 struct AttnTcArgs {
+  const bf16* q;
   int rows, ctx, kv_len, n_heads, n_kv_heads, causal;
   float scale_log2;
   bf16* o;
+  int n_vtiles, splits, tiles_per_split;
+  float* part_o;     // [splits][B*Hkv][group*rows][HD]
+  float2* part_ml;   // [splits][B*Hkv][group*rows]: (reference max in log2 units, sum)
   int* status;
 };
 
-template <int HD>
-__global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
-    attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
-                   const __grid_constant__ CUtensorMap tmV, const AttnTcArgs args) {
-  using C = AttnTcCfg<HD>;
+template <int HD, int TKV>
+__global__ void __launch_bounds__(192, AttnTcCfg<HD, TKV>::MIN_BLOCKS)
+    attn_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                   const AttnTcArgs args) {
+  using C = AttnTcCfg<HD, TKV>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = smem_raw;
   if (C::SLACK) {
@@ -83,13 +97,18 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m0 = blockIdx.x * TQ, h = blockIdx.y, b = blockIdx.z;
-  const int hk = h / (args.n_heads / args.n_kv_heads);
-  const int kv_end = args.causal ? min(args.kv_len, args.ctx + min(m0 + TQ, args.rows)) : args.kv_len;
-  const int n_tiles = (kv_end + TKV - 1) / TKV;
+  const int tile = blockIdx.x % args.n_vtiles, split = blockIdx.x / args.n_vtiles;
+  const int m0 = tile * TQ, hk = blockIdx.y, b = blockIdx.z;
+  const int group = args.n_heads / args.n_kv_heads, n_virt = group * args.rows;
+  // causal: the last key any of this CTA's rows may see
+  const int v_last = min(m0 + TQ, n_virt) - 1;
+  const int r_max = (m0 / args.rows != v_last / args.rows) ? args.rows - 1 : v_last % args.rows;
+  const int kv_end = args.causal ? min(args.kv_len, args.ctx + r_max + 1) : args.kv_len;
+  const int t0 = split * args.tiles_per_split;
+  const int n_tiles = max(0, min((kv_end + TKV - 1) / TKV, t0 + args.tiles_per_split) - t0);
 
   if (threadIdx.x == 0) {
-    mbar_init(q_full, 1);
+    mbar_init(q_full, 128);            // the softmax threads stage Q
     for (int s = 0; s < 2; ++s) {
       mbar_init(&kv_full[s], 1);
       mbar_init(&kv_empty[s], 1);
@@ -101,7 +120,6 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
-    tma_prefetch_desc(&tmQ);
     tma_prefetch_desc(&tmK);
     tma_prefetch_desc(&tmV);
   }
@@ -113,28 +131,25 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t t_s = tmem, t_o = tmem + 128;
+  const uint32_t t_s = tmem, t_o = tmem + TKV;
 
   if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------------------- producer
       int issued0 = 0, issued1 = 0;
-      mbar_arrive_expect_tx(q_full, C::Q_BYTES);
-      for (int s = 0; s < HD / 64; ++s) tma_load_3d(sQ + s * 16384, &tmQ, q_full, 64 * s, m0, b * args.n_heads + h);
-      for (int j = 0; j < n_tiles; ++j) {
-        const int st = j & 1;
-        if (!mbar_wait_bounded(&kv_empty[st], ((j >> 1) & 1) ^ 1, abort_flag, args.status)) break;
+      const int z = b * args.n_kv_heads + hk;
+      for (int i = 0; i < n_tiles; ++i) {
+        const int st = i & 1, j = t0 + i;
+        if (!mbar_wait_bounded(&kv_empty[st], ((i >> 1) & 1) ^ 1, abort_flag, args.status)) break;
         mbar_arrive_expect_tx(&kv_full[st], C::K_BYTES + C::V_BYTES);
-        const int z = b * args.n_kv_heads + hk;
         for (int s = 0; s < HD / 64; ++s)
-          tma_load_3d(sK + st * C::K_BYTES + s * 16384, &tmK, &kv_full[st], 64 * s, j * TKV, z);
-        for (int s = 0; s < 2; ++s)
+          tma_load_3d(sK + st * C::K_BYTES + s * (TKV * 128), &tmK, &kv_full[st], 64 * s, j * TKV, z);
+        for (int s = 0; s < TKV / 64; ++s)
           tma_load_3d(sV + st * C::V_BYTES + s * HD * 128, &tmV, &kv_full[st], j * TKV + 64 * s, 0, z);
         if (st) ++issued1; else ++issued0;
       }
       // every copy started here has landed before the CTA may exit
       volatile int never = 0;
-      mbar_wait_bounded(q_full, 0, &never, args.status);
       if (issued0 > 0) mbar_wait_bounded(&kv_full[0], (issued0 - 1) & 1, &never, args.status);
       if (issued1 > 0) mbar_wait_bounded(&kv_full[1], (issued1 - 1) & 1, &never, args.status);
     }
@@ -143,27 +158,27 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
       // ------------------------------------------------------------- MMA issuer
       constexpr uint32_t idesc_s = idesc_bf16_f32(TQ, TKV);
       constexpr uint32_t idesc_o = idesc_bf16_f32(TQ, HD);
-      bool ok = mbar_wait_bounded(q_full, 0, abort_flag, args.status);
+      bool ok = n_tiles > 0 && mbar_wait_bounded(q_full, 0, abort_flag, args.status);
       const uint32_t q0 = smem_u32(sQ), p0 = smem_u32(sP);
-      for (int j = 0; ok && j < n_tiles; ++j) {
-        const int st = j & 1;
-        if (!mbar_wait_bounded(&kv_full[st], (j >> 1) & 1, abort_flag, args.status)) break;
-        if (j > 0 && !mbar_wait_bounded(s_free, (j - 1) & 1, abort_flag, args.status)) break;
+      for (int i = 0; ok && i < n_tiles; ++i) {
+        const int st = i & 1;
+        if (!mbar_wait_bounded(&kv_full[st], (i >> 1) & 1, abort_flag, args.status)) break;
+        if (i > 0 && !mbar_wait_bounded(s_free, (i - 1) & 1, abort_flag, args.status)) break;
         tc_fence_after();
         const uint32_t k0 = smem_u32(sK + st * C::K_BYTES), v0 = smem_u32(sV + st * C::V_BYTES);
 #pragma unroll
         for (int kk = 0; kk < HD / 16; ++kk)
           umma_bf16(t_s, sdesc_kmajor_sw128(q0 + (kk >> 2) * 16384 + (kk & 3) * 32),
-                    sdesc_kmajor_sw128(k0 + (kk >> 2) * 16384 + (kk & 3) * 32), idesc_s, kk != 0);
+                    sdesc_kmajor_sw128(k0 + (kk >> 2) * (TKV * 128) + (kk & 3) * 32), idesc_s, kk != 0);
         umma_commit(s_full);
-        // P of tile j is in shared memory and any rescale of O by the softmax
+        // P of tile i is in shared memory and any rescale of O by the softmax
         // threads is complete: O += P V
-        if (!mbar_wait_bounded(p_full, j & 1, abort_flag, args.status)) break;
+        if (!mbar_wait_bounded(p_full, i & 1, abort_flag, args.status)) break;
         tc_fence_after();
 #pragma unroll
         for (int kk = 0; kk < TKV / 16; ++kk)
           umma_bf16(t_o, sdesc_kmajor_sw128(p0 + (kk >> 2) * 16384 + (kk & 3) * 32),
-                    sdesc_kmajor_sw128(v0 + (kk >> 2) * (HD * 128) + (kk & 3) * 32), idesc_o, (j != 0) || (kk != 0));
+                    sdesc_kmajor_sw128(v0 + (kk >> 2) * (HD * 128) + (kk & 3) * 32), idesc_o, (i != 0) || (kk != 0));
         umma_commit(o_full);
         umma_commit(&kv_empty[st]);
       }
@@ -173,25 +188,46 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
     }
   } else {
     // --------------------------------------------------------------- softmax
-    // One query row per thread (row = TMEM lane).  O is accumulated in TMEM
-    // by the P V MMAs of all key tiles.  The exponentials of every tile use a
-    // per-row reference max m_ref (log2 units); m_ref moves only when a tile's
-    // max exceeds it by more than 8, and then this thread rescales its row of
-    // O (and l) by 2^(m_ref_old - m_ref_new) before the next P V.  Softmax is
-    // invariant to the reference, and P <= 2^8 keeps bf16 P and fp32 O exact
-    // in range.  The passes use 3-input max and packed fp32-pair arithmetic.
+    // One virtual query row per thread (row = TMEM lane).  O is accumulated
+    // in TMEM by the P V MMAs of all key tiles.  The exponentials of every
+    // tile use a per-row reference max m_ref (log2 units); m_ref moves only
+    // when a tile's max exceeds it by more than 8, and then this thread
+    // rescales its row of O (and l) by 2^(m_ref_old - m_ref_new) before the
+    // next P V.  Softmax is invariant to the reference, and P <= 2^8 keeps
+    // bf16 P and fp32 O exact in range.  The passes use 3-input max and
+    // packed fp32-pair arithmetic.
     const int quad = warp & 3;
     const int row = quad * 32 + lane;                 // row within the tile = TMEM lane
     const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
-    const int qpos = args.ctx + m0 + row;
+    const int v = m0 + row;
+    const bool v_ok = v < n_virt;
+    const int qh = hk * group + (v_ok ? v / args.rows : 0);   // query head
+    const int qr = v_ok ? v % args.rows : 0;                                         // row of the canvas
+    const int qpos = args.ctx + qr;
+    // stage this row of Q (zeros past the virtual rows) in the swizzled operand layout
+    {
+      const uint4* src = reinterpret_cast<const uint4*>(
+          args.q + ((static_cast<size_t>(b) * args.n_heads + qh) * args.rows + qr) * HD);
+#pragma unroll
+      for (int s = 0; s < HD / 64; ++s) {
+        uint8_t* dst = sQ + s * 16384 + row * 128;
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          const uint4 val = v_ok ? src[s * 8 + c] : make_uint4(0, 0, 0, 0);
+          *reinterpret_cast<uint4*>(dst + ((c ^ (row & 7)) << 4)) = val;
+        }
+      }
+      fence_proxy_async_smem();
+      mbar_arrive(q_full);
+    }
     float m_ref = -INFINITY, l_run = 0.0f;
     bool ok = true;
     uint8_t* prow0 = sP + row * 128;
     const uint64_t sc2 = f2_pack(args.scale_log2, args.scale_log2);
-    for (int j = 0; j < n_tiles; ++j) {
-      if (!warp_wait_bounded(s_full, j & 1, abort_flag, args.status)) { ok = false; break; }
+    for (int i = 0; i < n_tiles; ++i) {
+      if (!warp_wait_bounded(s_full, i & 1, abort_flag, args.status)) { ok = false; break; }
       tc_fence_after();
-      const int key0 = j * TKV;
+      const int key0 = (t0 + i) * TKV;
       // keys visible to this row: key < kv_hi (kv_end, or the causal bound)
       const int kv_hi = args.causal ? min(kv_end, qpos + 1) : kv_end;
       const int lim = kv_hi - key0;                                   // visible keys of this tile
@@ -207,12 +243,12 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
         tmem_bind(rb);
         if (masked) {
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
-            mxa[i & 3] = fmax3(mxa[i & 3], 64 * c + i < lim ? __uint_as_float(ra[i]) : -INFINITY,
-                               64 * c + 32 + i < lim ? __uint_as_float(rb[i]) : -INFINITY);
+          for (int k = 0; k < 32; ++k)
+            mxa[k & 3] = fmax3(mxa[k & 3], 64 * c + k < lim ? __uint_as_float(ra[k]) : -INFINITY,
+                               64 * c + 32 + k < lim ? __uint_as_float(rb[k]) : -INFINITY);
         } else {
 #pragma unroll
-          for (int i = 0; i < 32; ++i) mxa[i & 3] = fmax3(mxa[i & 3], __uint_as_float(ra[i]), __uint_as_float(rb[i]));
+          for (int k = 0; k < 32; ++k) mxa[k & 3] = fmax3(mxa[k & 3], __uint_as_float(ra[k]), __uint_as_float(rb[k]));
         }
       }
       const float m_tile = fmax3(fmaxf(mxa[0], mxa[1]), mxa[2], mxa[3]) * args.scale_log2;
@@ -224,8 +260,8 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
         factor = ex2_approx(m_ref - m_tile);     // < 2^-8
       }
       if (__any_sync(0xffffffffu, factor != 1.0f)) {
-        // O holds tiles 0 .. j-1 once the P V of tile j-1 is done (j >= 1 here)
-        if (!warp_wait_bounded(o_full, (j - 1) & 1, abort_flag, args.status)) { ok = false; break; }
+        // O holds tiles 0 .. i-1 once the P V of tile i-1 is done (i >= 1 here)
+        if (!warp_wait_bounded(o_full, (i - 1) & 1, abort_flag, args.status)) { ok = false; break; }
         tc_fence_after();
 #pragma unroll
         for (int c = 0; c < HD / 32; ++c) {
@@ -233,7 +269,7 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
           tmem_ld32_nowait(t_o + lane_off + 32 * c, ra);
           tmem_wait_ld(ra);
 #pragma unroll
-          for (int i = 0; i < 32; ++i) ra[i] = __float_as_uint(__uint_as_float(ra[i]) * factor);
+          for (int k = 0; k < 32; ++k) ra[k] = __float_as_uint(__uint_as_float(ra[k]) * factor);
           tmem_st32(t_o + lane_off + 32 * c, ra);
         }
         tmem_wait_st();
@@ -249,17 +285,17 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
         tmem_wait_ld(ra);
         uint32_t pk[16];
 #pragma unroll
-        for (int i = 0; i < 32; i += 2) {
+        for (int k = 0; k < 32; k += 2) {
           float x0, x1;
-          f2_unpack(f2_fma(f2_pack(__uint_as_float(ra[i]), __uint_as_float(ra[i + 1])), sc2, negm2), x0, x1);
+          f2_unpack(f2_fma(f2_pack(__uint_as_float(ra[k]), __uint_as_float(ra[k + 1])), sc2, negm2), x0, x1);
           float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
           if (masked) {
-            p0 = 32 * c + i < lim ? p0 : 0.0f;
-            p1 = 32 * c + i + 1 < lim ? p1 : 0.0f;
+            p0 = 32 * c + k < lim ? p0 : 0.0f;
+            p1 = 32 * c + k + 1 < lim ? p1 : 0.0f;
           }
-          ps2[(i >> 1) & 1] = f2_add(ps2[(i >> 1) & 1], f2_pack(p0, p1));
+          ps2[(k >> 1) & 1] = f2_add(ps2[(k >> 1) & 1], f2_pack(p0, p1));
           __nv_bfloat162 t = __floats2bfloat162_rn(p0, p1);
-          pk[i / 2] = *reinterpret_cast<uint32_t*>(&t);
+          pk[k / 2] = *reinterpret_cast<uint32_t*>(&t);
         }
         // keys 32c .. 32c+31: atom (32c / 64), 16-byte chunks (32c % 64) / 8 .. +3
         uint8_t* atom = prow0 + (c >> 1) * 16384;
@@ -280,26 +316,52 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
       mbar_arrive(s_free);
       mbar_arrive(p_full);
     }
-    if (ok && n_tiles > 0 && warp_wait_bounded(o_full, (n_tiles - 1) & 1, abort_flag, args.status)) {
+    const size_t bk = static_cast<size_t>(b) * args.n_kv_heads + hk;
+    if (args.splits > 1 && ok && n_tiles == 0) {
+      // no key of this split: an empty partial
+      if (v_ok) {
+        const size_t pr = (static_cast<size_t>(split) * args.n_kv_heads * gridDim.z + bk) * n_virt + v;
+        float4* po = reinterpret_cast<float4*>(args.part_o + pr * HD);
+        for (int k = 0; k < HD / 4; ++k) po[k] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+        args.part_ml[pr] = make_float2(-INFINITY, 0.0f);
+      }
+    } else if (ok && n_tiles > 0 && warp_wait_bounded(o_full, (n_tiles - 1) & 1, abort_flag, args.status)) {
       tc_fence_after();
-      const int grow = m0 + row;
-      const float inv = l_run > 0.0f ? 1.0f / l_run : 0.0f;
-      bf16* orow = args.o + (static_cast<size_t>(b) * args.rows + grow) * args.n_heads * HD + static_cast<size_t>(h) * HD;
+      if (args.splits > 1) {
+        const size_t pr = (static_cast<size_t>(split) * args.n_kv_heads * gridDim.z + bk) * n_virt + v;
+        float4* po = reinterpret_cast<float4*>(args.part_o + pr * HD);
 #pragma unroll
-      for (int c = 0; c < HD / 32; ++c) {
-        uint32_t ra[32];
-        tmem_ld32_nowait(t_o + lane_off + 32 * c, ra);
-        tmem_wait_ld(ra);
-        if (grow < args.rows) {
+        for (int c = 0; c < HD / 32; ++c) {
+          uint32_t ra[32];
+          tmem_ld32_nowait(t_o + lane_off + 32 * c, ra);
+          tmem_wait_ld(ra);
+          if (v_ok) {
 #pragma unroll
-          for (int i = 0; i < 32; i += 8) {
-            __nv_bfloat162 t0 = __floats2bfloat162_rn(__uint_as_float(ra[i]) * inv, __uint_as_float(ra[i + 1]) * inv);
-            __nv_bfloat162 t1 = __floats2bfloat162_rn(__uint_as_float(ra[i + 2]) * inv, __uint_as_float(ra[i + 3]) * inv);
-            __nv_bfloat162 t2 = __floats2bfloat162_rn(__uint_as_float(ra[i + 4]) * inv, __uint_as_float(ra[i + 5]) * inv);
-            __nv_bfloat162 t3 = __floats2bfloat162_rn(__uint_as_float(ra[i + 6]) * inv, __uint_as_float(ra[i + 7]) * inv);
-            *reinterpret_cast<uint4*>(orow + 32 * c + i) =
-                make_uint4(*reinterpret_cast<uint32_t*>(&t0), *reinterpret_cast<uint32_t*>(&t1),
-                           *reinterpret_cast<uint32_t*>(&t2), *reinterpret_cast<uint32_t*>(&t3));
+            for (int k = 0; k < 32; k += 4)
+              po[(32 * c + k) / 4] = make_float4(__uint_as_float(ra[k]), __uint_as_float(ra[k + 1]),
+                                                 __uint_as_float(ra[k + 2]), __uint_as_float(ra[k + 3]));
+          }
+        }
+        if (v_ok) args.part_ml[pr] = make_float2(m_ref, l_run);
+      } else {
+        const float inv = l_run > 0.0f ? 1.0f / l_run : 0.0f;
+        bf16* orow = args.o + (static_cast<size_t>(b) * args.rows + qr) * args.n_heads * HD + static_cast<size_t>(qh) * HD;
+#pragma unroll
+        for (int c = 0; c < HD / 32; ++c) {
+          uint32_t ra[32];
+          tmem_ld32_nowait(t_o + lane_off + 32 * c, ra);
+          tmem_wait_ld(ra);
+          if (v_ok) {
+#pragma unroll
+            for (int k = 0; k < 32; k += 8) {
+              __nv_bfloat162 w0 = __floats2bfloat162_rn(__uint_as_float(ra[k]) * inv, __uint_as_float(ra[k + 1]) * inv);
+              __nv_bfloat162 w1 = __floats2bfloat162_rn(__uint_as_float(ra[k + 2]) * inv, __uint_as_float(ra[k + 3]) * inv);
+              __nv_bfloat162 w2 = __floats2bfloat162_rn(__uint_as_float(ra[k + 4]) * inv, __uint_as_float(ra[k + 5]) * inv);
+              __nv_bfloat162 w3 = __floats2bfloat162_rn(__uint_as_float(ra[k + 6]) * inv, __uint_as_float(ra[k + 7]) * inv);
+              *reinterpret_cast<uint4*>(orow + 32 * c + k) =
+                  make_uint4(*reinterpret_cast<uint32_t*>(&w0), *reinterpret_cast<uint32_t*>(&w1),
+                             *reinterpret_cast<uint32_t*>(&w2), *reinterpret_cast<uint32_t*>(&w3));
+            }
           }
         }
       }
@@ -312,6 +374,45 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD>::MIN_BLOCKS)
     tc_fence_after();
     tmem_dealloc(tmem, C::TMEM_COLS);
   }
+}
+
+// Merges the split partials of one virtual row per warp, in split order:
+// m* = max m_s, O = sum 2^(m_s - m*) O_s / sum 2^(m_s - m*) l_s.
+template <int HD>
+__global__ void __launch_bounds__(256) attn_combine_kernel(const float* __restrict__ part_o,
+                                                           const float2* __restrict__ part_ml, int splits,
+                                                           int n_bk, int n_virt, int rows, int n_heads,
+                                                           int n_kv_heads, bf16* __restrict__ o) {
+  constexpr int PL = HD / 32;   // dims per lane
+  const int lane = threadIdx.x & 31;
+  const int g = blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (g >= n_bk * n_virt) return;
+  const size_t stride = static_cast<size_t>(n_bk) * n_virt;
+  float mx = -INFINITY;
+  for (int s = 0; s < splits; ++s) mx = fmaxf(mx, part_ml[s * stride + g].x);
+  float acc[PL];
+#pragma unroll
+  for (int k = 0; k < PL; ++k) acc[k] = 0.0f;
+  float L = 0.0f;
+  if (mx != -INFINITY) {
+    for (int s = 0; s < splits; ++s) {
+      const float2 ml = part_ml[s * stride + g];
+      const float w = ml.x == -INFINITY ? 0.0f : ex2_approx(ml.x - mx);
+      L = fmaf(w, ml.y, L);
+      const float* src = part_o + (s * stride + g) * HD + lane * PL;
+#pragma unroll
+      for (int k = 0; k < PL; ++k) acc[k] = fmaf(w, src[k], acc[k]);
+    }
+  }
+  const float inv = L > 0.0f ? 1.0f / L : 0.0f;
+  const int bk = g / n_virt, v = g - bk * n_virt;
+  const int group = n_heads / n_kv_heads;
+  const int b = bk / n_kv_heads, hk = bk - b * n_kv_heads;
+  const int h = hk * group + v / rows, r = v % rows;
+  bf16* orow = o + (static_cast<size_t>(b) * rows + r) * n_heads * HD + static_cast<size_t>(h) * HD + lane * PL;
+#pragma unroll
+  for (int k = 0; k < PL; k += 2)
+    *reinterpret_cast<__nv_bfloat162*>(orow + k) = __floats2bfloat162_rn(acc[k] * inv, acc[k + 1] * inv);
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 g_enc = nullptr;
@@ -341,33 +442,62 @@ bool map3d(CUtensorMap* m, const void* ptr, uint64_t d0, uint64_t d1, uint64_t d
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int HD>
-const char* launch_tc(const AttnCall& a, int* status, cudaStream_t s) {
-  using C = AttnTcCfg<HD>;
+template <int HD, int TKV>
+const char* launch_tc(const AttnCall& a, cudaStream_t s) {
+  using C = AttnTcCfg<HD, TKV>;
   if (!encoder()) return "cuTensorMapEncodeTiled is unavailable";
   const int kv_len = a.ctx + a.rows;
-  CUtensorMap mq, mk, mv;
-  // Q: {hd, rows, B*Hq}; K: {hd, kv_len, B*Hkv}; V^T: {kv_len, hd, B*Hkv} -- positions past kv_len read zeros
-  if (!map3d(&mq, a.q, HD, a.rows, static_cast<uint64_t>(a.batch) * a.n_heads, HD * 2ull,
-             static_cast<uint64_t>(a.rows) * HD * 2, TQ) ||
-      !map3d(&mk, a.k, HD, kv_len, static_cast<uint64_t>(a.batch) * a.n_kv_heads, HD * 2ull,
+  CUtensorMap mk, mv;
+  // K: {hd, kv_len, B*Hkv}; V^T: {kv_len, hd, B*Hkv} -- positions past kv_len read zeros
+  if (!map3d(&mk, a.k, HD, kv_len, static_cast<uint64_t>(a.batch) * a.n_kv_heads, HD * 2ull,
              static_cast<uint64_t>(a.kv_stride) * HD * 2, TKV) ||
       !map3d(&mv, a.v, kv_len, HD, static_cast<uint64_t>(a.batch) * a.n_kv_heads, a.kv_stride * 2ull,
              static_cast<uint64_t>(a.kv_stride) * HD * 2, HD))
     return "attention tensor map encode failed";
-  static bool attr = false;
-  if (!attr) {
-    if (cudaFuncSetAttribute(attn_tc_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM) !=
+  static int n_sms = 0;
+  if (n_sms == 0) {
+    if (cudaFuncSetAttribute(attn_tc_kernel<HD, TKV>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM) !=
         cudaSuccess)
       return "attention smem attribute failed";
-    attr = true;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&n_sms, cudaDevAttrMultiProcessorCount, dev);
+    if (n_sms <= 0) n_sms = 1;
   }
-  AttnTcArgs args{a.rows, a.ctx, kv_len, a.n_heads, a.n_kv_heads, a.causal,
-                  1.4426950408889634f / sqrtf(static_cast<float>(HD)), static_cast<bf16*>(a.o), status};
-  dim3 grid((a.rows + TQ - 1) / TQ, a.n_heads, a.batch);
-  attn_tc_kernel<HD><<<grid, 192, C::SMEM, s>>>(mq, mk, mv, args);
+  const int group = a.n_heads / a.n_kv_heads, n_virt = group * a.rows;
+  const int n_vtiles = (n_virt + TQ - 1) / TQ;
+  const int base = n_vtiles * a.n_kv_heads * a.batch;
+  const int kv_tiles = (kv_len + TKV - 1) / TKV;
+  // split the keys when the CTAs would not fill two waves: every split keeps
+  // >= 3 tiles and its fp32 partials fit the caller's scratch
+  int splits = 1;
+  if (a.part && a.part_bytes > 0) {
+    const int slots = C::MIN_BLOCKS * n_sms;
+    const size_t per_split = static_cast<size_t>(a.batch) * a.n_kv_heads * n_virt * (HD + 2) * sizeof(float);
+    splits = std::min(std::min((2 * slots + base - 1) / base, kv_tiles / 3), 8);
+    while (splits > 1 && static_cast<size_t>(splits) * per_split > a.part_bytes) --splits;
+    if (splits < 1) splits = 1;
+  }
+  const int tps = (kv_tiles + splits - 1) / splits;
+  splits = (kv_tiles + tps - 1) / tps;
+  float* part_o = static_cast<float*>(a.part);
+  float2* part_ml = reinterpret_cast<float2*>(part_o + static_cast<size_t>(splits) * a.batch * a.n_kv_heads * n_virt * HD);
+  AttnTcArgs args{static_cast<const bf16*>(a.q), a.rows, a.ctx, kv_len, a.n_heads, a.n_kv_heads, a.causal,
+                  1.4426950408889634f / sqrtf(static_cast<float>(HD)), static_cast<bf16*>(a.o),
+                  n_vtiles, splits, tps, part_o, part_ml, a.status};
+  dim3 grid(n_vtiles * splits, a.n_kv_heads, a.batch);
+  attn_tc_kernel<HD, TKV><<<grid, 192, C::SMEM, s>>>(mk, mv, args);
   cudaError_t e = cudaGetLastError();
-  return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
+  if (e != cudaSuccess) return cudaGetErrorString(e);
+  if (splits > 1) {
+    const int n_bk = a.batch * a.n_kv_heads;
+    const int rows_total = n_bk * n_virt;
+    attn_combine_kernel<HD><<<(rows_total + 7) / 8, 256, 0, s>>>(part_o, part_ml, splits, n_bk, n_virt, a.rows,
+                                                               a.n_heads, a.n_kv_heads, static_cast<bf16*>(a.o));
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return cudaGetErrorString(e);
+  }
+  return nullptr;
 }
 
 // ============================================================= mma.sync path
@@ -655,9 +785,14 @@ const char* attention(const AttnCall& a, cudaStream_t s) {
   if (a.n_kv_heads <= 0 || a.n_heads % a.n_kv_heads) return "n_heads must be a multiple of n_kv_heads";
   if (a.kv_stride < a.ctx + a.rows) return "kv_stride smaller than ctx + rows";
   if (a.bf16) {
-    const bool tc = a.rows >= TQ && a.kv_stride % 8 == 0;
-    if (a.head_dim == 64) return tc ? launch_tc<64>(a, a.status, s) : (launch_bf16<64>(a, s) == cudaSuccess ? nullptr : "attention launch failed");
-    if (a.head_dim == 128) return tc ? launch_tc<128>(a, a.status, s) : (launch_bf16<128>(a, s) == cudaSuccess ? nullptr : "attention launch failed");
+    // tcgen05 whenever the V^T rows are 16-byte aligned for TMA (the library's
+    // KV buffers always are); 64-key tiles for hd 128 with few query rows
+    const bool tc = a.kv_stride % 8 == 0 && (reinterpret_cast<uintptr_t>(a.q) & 15) == 0;
+    if (a.head_dim == 64) return tc ? launch_tc<64, 128>(a, s) : (launch_bf16<64>(a, s) == cudaSuccess ? nullptr : "attention launch failed");
+    if (a.head_dim == 128) {
+      if (!tc) return launch_bf16<128>(a, s) == cudaSuccess ? nullptr : "attention launch failed";
+      return (a.n_heads / a.n_kv_heads) * a.rows < 2 * TQ ? launch_tc<128, 64>(a, s) : launch_tc<128, 128>(a, s);
+    }
     return "bf16 attention supports head_dim 64 and 128";
   }
   cudaError_t e;

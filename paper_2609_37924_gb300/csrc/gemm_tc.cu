@@ -125,14 +125,14 @@ struct TcArgs {
 // epilogue will read (residual stream, h, gate), so the epilogue does not wait
 // on DRAM latency.
 template <int EPI>
-__device__ __forceinline__ void prefetch_epilogue_inputs(const TcArgs& a, int mb, int nb) {
+__device__ __forceinline__ void prefetch_epilogue_inputs(const TcArgs& a, int mb, int nb, int ncols = BN) {
   const EpiParams& p = a.ep;
   const float* src = nullptr;
   int ld = 0;
   if constexpr (EPI == EPI_RESID) { src = p.resid; ld = p.ldr; }
   else if constexpr (EPI == EPI_FUSION2 || EPI == EPI_ADD || EPI == EPI_PA_UP) { src = p.base; ld = p.ldb; }
   if (!src) return;
-  const int n0 = nb * BN, ncol = min(BN, p.N - n0);
+  const int n0 = nb * ncols, ncol = min(ncols, p.N - n0);
   if (ncol <= 0 || (ld & 3) || (n0 & 3)) return;
   const uint32_t bytes = static_cast<uint32_t>(ncol) * 4u & ~15u;
   for (int r = mb * BM; r < min(mb * BM + BM, p.M); ++r) prefetch_l2(src + static_cast<size_t>(r) * ld + n0, bytes);
@@ -313,18 +313,26 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 // bytes); the MMA thread's commits release empty[s] and signal tfull[a] in
 // both CTAs; every epilogue warp of both CTAs releases an accumulator on the
 // even CTA's tempty[a].
-constexpr int P_STAGES = 6;
-constexpr int P_A_BYTES = BM * BK * 2;            // 16 KB
-constexpr int P_B_BYTES = (BN / 2) * BK * 2;      // 16 KB: this CTA's half of B
-constexpr int P_STAGE_BYTES = P_A_BYTES + P_B_BYTES;
-constexpr size_t P_SMEM_BYTES = 1024 + P_STAGES * P_STAGE_BYTES + EPI_WARPS * STAGE_OUT_BYTES + 256;
-static_assert(P_SMEM_BYTES <= 232448, "pair GEMM shared memory");
+// PBN: columns of the pair tile (256, or 128 for GEMMs whose 256-wide pair
+// tiles would leave most SMs idle).
+template <int PBN>
+struct PairCfg {
+  static constexpr int STAGES = PBN == 256 ? 6 : 8;
+  static constexpr int A_BYTES = BM * BK * 2;            // 16 KB
+  static constexpr int B_BYTES = (PBN / 2) * BK * 2;     // this CTA's half of B: 16 KB / 8 KB
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr size_t SMEM = 1024 + STAGES * STAGE_BYTES + EPI_WARPS * STAGE_OUT_BYTES + 256;
+  static_assert(SMEM <= 232448, "pair GEMM shared memory");
+};
 
-template <int EPI>
+template <int EPI, int PBN>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmC2,
                     const TcArgs args) {
+  using PC = PairCfg<PBN>;
+  constexpr int P_STAGES = PC::STAGES, P_A_BYTES = PC::A_BYTES, P_B_BYTES = PC::B_BYTES;
+  constexpr int P_STAGE_BYTES = PC::STAGE_BYTES;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
@@ -380,8 +388,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       for (int unit = u0; unit < units && !*abort_flag; unit += ustep) {
         const int nb = unit % args.n_tiles_n;
         const int mb = 2 * (unit / args.n_tiles_n) + static_cast<int>(rank);   // this CTA's 128-row block
-        prefetch_epilogue_inputs<EPI>(args, mb, nb);
-        const int brow = args.b_split > 0 ? (rank ? args.b_split : 0) + nb * (BN / 2) : nb * BN + rank * (BN / 2);
+        prefetch_epilogue_inputs<EPI>(args, mb, nb, PBN);
+        const int brow = args.b_split > 0 ? (rank ? args.b_split : 0) + nb * (PBN / 2) : nb * PBN + rank * (PBN / 2);
         bool ok = true;
         for (int kb = 0; kb < kblocks; ++kb) {
           if (!mbar_wait_bounded(&empty[stage], phase ^ 1, abort_flag, args.status)) { ok = false; break; }
@@ -404,7 +412,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
   } else if (warp == 1) {
     if (lane == 0 && leader) {
       // ---------------------------------------------------------------- MMA issuer (even CTA)
-      constexpr uint32_t idesc = idesc_bf16_f32(2 * BM, BN);
+      constexpr uint32_t idesc = idesc_bf16_f32(2 * BM, PBN);
       int stage = 0;
       uint32_t phase = 0;
       int acc = 0;
@@ -412,7 +420,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       for (int unit = u0; unit < units && !*abort_flag; unit += ustep) {
         if (!mbar_wait_bounded(&tempty[acc], acc_phase ^ 1, abort_flag, args.status)) break;
         tc_fence_after();
-        const uint32_t d_tmem = tmem_base + acc * BN;
+        const uint32_t d_tmem = tmem_base + acc * PBN;
         bool ok = true;
         for (int kb = 0; kb < kblocks; ++kb) {
           if (!mbar_wait_bounded(&full[stage], phase, abort_flag, args.status)) { ok = false; break; }
@@ -449,11 +457,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       tc_fence_after();
       const int nb = unit % args.n_tiles_n;
       const int mb = 2 * (unit / args.n_tiles_n) + static_cast<int>(rank);
-      TmemSrc src{tmem_base + static_cast<uint32_t>(acc * BN) + (static_cast<uint32_t>(quad * 32) << 16),
+      TmemSrc src{tmem_base + static_cast<uint32_t>(acc * PBN) + (static_cast<uint32_t>(quad * 32) << 16),
                   args.staged ? sOut + (warp - 2) * STAGE_OUT_BYTES : nullptr, {&tmC, &tmC2}, mb * BM + quad * 32};
       const int m = mb * BM + quad * 32 + lane;
       if (part < nsplit && mb * BM < args.M)   // the odd CTA's rows may lie past M
-        epilogue_row<EPI>(args.ep, m, nb, BN, src, part, nsplit);
+        epilogue_row<EPI>(args.ep, m, nb, PBN, src, part, nsplit);
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_remote(tempty_l0 + 8u * acc);
@@ -549,27 +557,28 @@ cudaError_t launch_epi(const CUtensorMap& ta, const CUtensorMap& tb, const CUten
 // CTA-pair kernel: `pairs` = 256-row x 256-column tiles; the grid is capped at
 // the number of 2-CTA clusters that fit on the GPU at once (a persistent grid
 // larger than that would run its last clusters after the others).
-template <int EPI>
+template <int EPI, int PBN = 256>
 cudaError_t launch_epi_pair(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc,
                             const CUtensorMap& tc2, const TcArgs& a, int pairs, cudaStream_t s) {
+  constexpr size_t smem = PairCfg<PBN>::SMEM;
   static int max_clusters = 0;
   if (max_clusters == 0) {
-    cudaError_t e = cudaFuncSetAttribute(gemm_tc2_kernel<EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(P_SMEM_BYTES));
+    cudaError_t e = cudaFuncSetAttribute(gemm_tc2_kernel<EPI, PBN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = dim3(g_num_sms & ~1);
     cfg.blockDim = dim3(NUM_THREADS);
-    cfg.dynamicSmemBytes = P_SMEM_BYTES;
+    cfg.dynamicSmemBytes = smem;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc2_kernel<EPI>, &cfg) != cudaSuccess || n <= 0) {
+    if (cudaOccupancyMaxActiveClusters(&n, gemm_tc2_kernel<EPI, PBN>, &cfg) != cudaSuccess || n <= 0) {
       cudaGetLastError();
       n = g_num_sms / 2;
     }
     max_clusters = n;
   }
   const int clusters = std::min(pairs, max_clusters);
-  gemm_tc2_kernel<EPI><<<2 * clusters, NUM_THREADS, P_SMEM_BYTES, s>>>(ta, tb, tc, tc2, a);
+  gemm_tc2_kernel<EPI, PBN><<<2 * clusters, NUM_THREADS, smem, s>>>(ta, tb, tc, tc2, a);
   return cudaGetLastError();
 }
 
@@ -626,9 +635,14 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
   a.kb_per_split = kblocks;
   a.ldp = a.n_tiles_n * BN;
   // CTA-pair tiles that keep >= 40% of the SMs busy beat split-K: no fp32
-  // partials, no reduction launches
-  const int pair_units = ((g.M + 2 * BM - 1) / (2 * BM)) * a.n_tiles_n;
+  // partials, no reduction launches.  Residual and fusion-output GEMMs (N =
+  // d) whose 256-wide pair tiles would occupy at most half the SMs use
+  // 256 x 128 pair tiles instead.
+  const int m_pairs = (g.M + 2 * BM - 1) / (2 * BM);
   const bool pair_ok = g_pair_mma && g.M > BM;
+  const bool narrow = pair_ok && (g.epi == EPI_RESID || g.epi == EPI_FUSION2) &&
+                      m_pairs * a.n_tiles_n * 4 <= g_num_sms;
+  const int pair_units = narrow ? m_pairs * ((g.N + 127) / 128) : m_pairs * a.n_tiles_n;
   const bool pairs_fill = pair_ok && 2 * pair_units * 5 >= g_num_sms * 2;
   if (g.split_buf && !pairs_fill && tiles * 3 < g_num_sms * 2 && kblocks >= 8) {
     int sp = std::min(std::min(g_num_sms / tiles, kblocks / 4), 16);
@@ -644,6 +658,17 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
   }
   // CTA pairs (256 x 256 tiles, cta_group::2) for every unsplit GEMM of more
   // than 128 rows: the same SMs as 128 x 256 tiles, less operand traffic each
+  if (pair_ok && a.splits == 1 && narrow) {
+    CUtensorMap tbh;
+    if (!make_map(&tbh, g.B, b_rows, g.K, g.ldb, 64)) return "tensor map (B, quarter tiles) encode failed";
+    TcArgs a2 = a;
+    a2.n_tiles_n = (g.N + 127) / 128;
+    cudaError_t e = g.epi == EPI_RESID ? launch_epi_pair<EPI_RESID, 128>(ta, tbh, tc, tc2, a2, pair_units, s)
+                                       : launch_epi_pair<EPI_FUSION2, 128>(ta, tbh, tc, tc2, a2, pair_units, s);
+    if (e != cudaSuccess) return cudaGetErrorString(e);
+    const_cast<GemmCall&>(g).launched = 1;
+    return nullptr;
+  }
   if (pair_ok && a.splits == 1) {
     CUtensorMap tbh;
     if (!make_map(&tbh, g.B, b_rows, g.K, g.ldb, BN / 2)) return "tensor map (B, half tiles) encode failed";

@@ -41,6 +41,8 @@ struct AttnCall {
   int batch, n_heads, n_kv_heads, head_dim, rows, ctx, kv_stride, causal;
   int bf16;
   int* status;   // device status word (may be null)
+  void* part = nullptr;      // optional fp32 scratch for split-key partials (16-byte aligned)
+  size_t part_bytes = 0;
 };
 const char* attention(const AttnCall& a, cudaStream_t s);
 

@@ -117,6 +117,7 @@ struct tadm_handle {
   size_t ws_bytes = 0, ws_need = 0;
   struct Off {
     size_t status, rope, c, x, h_int, norm, qbuf, kv, attn, glu, f_g, f_hid, f_pre, part, conf, tok, split, idx;
+    size_t attn_part;
     size_t pa_z, pa_j, pa_mq, pa_mk, pa_mv, pa_mo, pa_r, pa_rb, pa_hid, pa_phi, pa_m, pa_dz, pa_f, pa_g, pa_mb;
   } off{};
   size_t kv_slab = 0;
@@ -167,6 +168,9 @@ tadm_status fail(tadm_handle* h, tadm_status s, const char* fmt, ...) {
     tadm_status _s = (expr);               \
     if (_s != TADM_OK) return _s;          \
   } while (0)
+
+// fp32 scratch for the split-key partials of attention (bf16 models)
+constexpr size_t kAttnPartBytes = size_t(64) << 20;
 
 size_t cache_bytes(const tadm_config& c, int batch, int rows) {
   const size_t M = static_cast<size_t>(batch) * rows;
@@ -251,6 +255,7 @@ void layout(tadm_handle* h) {
   }
   f.part = take(M * h->n_part_tiles * 3 * 4);
   f.split = c.dtype ? take(gemm_tc_split_bytes()) : take(0);
+  f.attn_part = c.dtype ? take(kAttnPartBytes) : take(0);
   f.conf = take(M * 4);
   f.tok = take(M * 4);
   f.idx = take(M * 4);
@@ -258,6 +263,21 @@ void layout(tadm_handle* h) {
 }
 
 // --------------------------------------------------------------------------- kernels wrappers
+// probe kinds beyond the GEMM epilogues (0..10)
+constexpr int kProbeAttention = 11, kProbeNorm = 12;
+// Opens a probe record (start event) when the probe is on and has room: returns its index, else -1.
+int probe_begin(tadm_handle* h, cudaStream_t s) {
+  if (h->probe_next >= static_cast<int>(h->probe_flops.size())) return -1;
+  cudaEventRecord(h->probe_ev[2 * h->probe_next], s);
+  return h->probe_next++;
+}
+void probe_end(tadm_handle* h, cudaStream_t s, int idx, int kind, double flops) {
+  if (idx < 0) return;
+  cudaEventRecord(h->probe_ev[2 * idx + 1], s);
+  h->probe_kind[idx] = kind;
+  h->probe_flops[idx] = flops;
+}
+
 tadm_status gemm(tadm_handle* h, const void* A, int64_t a_rows, int lda, const void* B, int ldb, int M, int N, int K,
                  int epi, const EpiParams& ep, cudaStream_t s, bool out_f32 = false) {
   GemmCall g{};
@@ -278,17 +298,12 @@ tadm_status gemm(tadm_handle* h, const void* A, int64_t a_rows, int lda, const v
   }
   g.ep.out_bf16 = out_f32 ? 0 : h->act_bf16();
   g.ep.bias_bf16 = h->cfg.dtype;
-  const bool probe = h->probe_next < static_cast<int>(h->probe_flops.size());
-  if (probe) cudaEventRecord(h->probe_ev[2 * h->probe_next], s);
+  const int pi = probe_begin(h, s);
   const char* e = h->cfg.dtype ? gemm_tc(g, s) : gemm_simt(g, s);
   if (e) return fail(h, TADM_ERR_CUDA, "GEMM (M=%d N=%d K=%d epi=%d): %s", M, N, K, epi, e);
   h->counters.kernel_launches += h->cfg.dtype ? g.launched : 1;
-  if (probe) {
-    cudaEventRecord(h->probe_ev[2 * h->probe_next + 1], s);
-    const double n_acc = epi == EPI_GLU ? 2.0 * N : static_cast<double>(N);
-    h->probe_kind[h->probe_next] = epi;
-    h->probe_flops[h->probe_next++] = 2.0 * M * n_acc * K;
-  }
+  const double n_acc = epi == EPI_GLU ? 2.0 * N : static_cast<double>(N);
+  probe_end(h, s, pi, epi, 2.0 * M * n_acc * K);
   return TADM_OK;
 }
 
@@ -306,7 +321,9 @@ tadm_status layer_fwd(tadm_handle* h, int li, float* x, int B, int R, int ctx, i
   const int q = c.n_heads * hd, nqkv = (c.n_heads + 2 * c.n_kv_heads) * hd;
   const int64_t Mmax = static_cast<int64_t>(h->max_batch) * h->max_rows;
   void* norm = h->at(h->off.norm);
+  int pi = probe_begin(h, s);
   TRY(rmsnorm_rows(x, M, d, L.attn_norm, c.dtype, c.norm_eps, norm, d, h->act_bf16(), s));
+  probe_end(h, s, pi, kProbeNorm, 0.0);
   EpiParams ep{};
   ep.q = h->at(h->off.qbuf);
   ep.k = kv_ptr(h, li, 0);
@@ -323,12 +340,22 @@ tadm_status layer_fwd(tadm_handle* h, int li, float* x, int B, int R, int ctx, i
   TRYS(gemm(h, norm, Mmax, d, L.wqkv, d, M, nqkv, d, EPI_QKV, ep, s));
   AttnCall a{ep.q, ep.k, ep.v, h->at(h->off.attn), B, c.n_heads, c.n_kv_heads, hd, R, ctx, h->kv_stride, causal,
              h->act_bf16(), h->status()};
+  if (c.dtype) {
+    a.part = h->at(h->off.attn_part);
+    a.part_bytes = kAttnPartBytes;
+  }
+  pi = probe_begin(h, s);
   TRY(attention(a, s));
+  // keys seen per query row: all of them, or the causal average
+  const double keys = causal ? ctx + 0.5 * (R + 1) : static_cast<double>(ctx + R);
+  probe_end(h, s, pi, kProbeAttention, 4.0 * M * c.n_heads * keys * hd);
   EpiParams er{};
   er.resid = x;
   er.ldr = d;
   TRYS(gemm(h, h->at(h->off.attn), Mmax, q, L.wo, q, M, d, q, EPI_RESID, er, s));
+  pi = probe_begin(h, s);
   TRY(rmsnorm_rows(x, M, d, L.ffn_norm, c.dtype, c.norm_eps, norm, d, h->act_bf16(), s));
+  probe_end(h, s, pi, kProbeNorm, 0.0);
   EpiParams eg{};
   eg.out = h->at(h->off.glu);
   eg.ldo = c.ffn;
@@ -447,8 +474,10 @@ tadm_status run_fusion(tadm_handle* h, int B, int R, const void* cache, cudaStre
     // u = [LN(c); LN(h)];  [g | a] = [sigmoid(W_g u + b_g) | GELU(W_1 u + b_1)];
     // pre = h + g * (W_2 a + b_2);  h~ = LN(pre)                        (App. C.2)
     void* u = h->at(h->off.norm);
+    int pi = probe_begin(h, s);
     TRY(ln_pair_rows(cbuf, cv.h, M, d, h->fw[0], h->fw[1], h->fw[2], h->fw[3], c.dtype, c.norm_eps, u,
                      h->act_bf16(), s));
+    probe_end(h, s, pi, kProbeNorm, 0.0);
     EpiParams e1{};
     e1.bias = h->fw[5];
     e1.d_split = d;
@@ -466,7 +495,9 @@ tadm_status run_fusion(tadm_handle* h, int B, int R, const void* cache, cudaStre
     e2.out = h->at(h->off.f_pre);
     e2.ldo = d;
     TRYS(gemm(h, h->at(h->off.f_hid), Mmax, 4 * d, h->fw[6], 4 * d, M, d, 4 * d, EPI_FUSION2, e2, s));
+    pi = probe_begin(h, s);
     TRY(layernorm_rows(h->at<float>(h->off.f_pre), M, d, h->fw[8], h->fw[9], c.dtype, c.norm_eps, x, s));
+    probe_end(h, s, pi, kProbeNorm, 0.0);
     return TADM_OK;
   }
   // paired attention (App. C.1): Z = (C/s_C) W_C; M = phi(Z, U) - phi(Z0, U);
@@ -766,14 +797,17 @@ tadm_status tadm_probe_read(tadm_handle* h, int64_t* launches, double* total_ms,
   double ms = 0.0, fl = 0.0;
   if (h->probe_next > 0 && cudaEventSynchronize(h->probe_ev[2 * h->probe_next - 1]) != cudaSuccess)
     return fail(h, TADM_ERR_CUDA, "probe event sync failed");
+  int64_t n_gemm = 0;
   for (int i = 0; i < h->probe_next; ++i) {
+    if (h->probe_kind[i] >= kProbeAttention) continue;   // GEMM launches only
     float t = 0.0f;
     if (cudaEventElapsedTime(&t, h->probe_ev[2 * i], h->probe_ev[2 * i + 1]) != cudaSuccess)
       return fail(h, TADM_ERR_CUDA, "probe elapsed time failed");
     ms += t;
     fl += h->probe_flops[i];
+    ++n_gemm;
   }
-  if (launches) *launches = h->probe_next;
+  if (launches) *launches = n_gemm;
   if (total_ms) *total_ms = ms;
   if (total_flops) *total_flops = fl;
   h->probe_next = 0;

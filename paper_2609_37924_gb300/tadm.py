@@ -305,7 +305,8 @@ class TadmModel:
         _check(self.lib.tadm_probe_enable(self.h, max_launches), self.h)
 
     EPI_NAMES = ["plain", "residual", "qkv_rope", "glu", "fusion_gate_hidden", "fusion_out", "output_head",
-                 "pa_up", "pa_silu", "pa_add", "pa_gate"]
+                 "pa_up", "pa_silu", "pa_add", "pa_gate", "attention", "norms"]
+    N_GEMM_KINDS = 11
 
     def tadm_probe_breakdown(self) -> dict:
         n = len(self.EPI_NAMES)

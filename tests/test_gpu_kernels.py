@@ -63,11 +63,16 @@ def test_gemm_f32_cuda_cores(T, M, N, K):
 
 
 # -------------------------------------------------------------------------- attention
-# rows >= 128 with kv_stride % 8 == 0 run the tcgen05 kernel, the others mma.sync
+# kv_stride % 8 == 0 runs the tcgen05 kernel (128 virtual rows = query heads of
+# a KV group x rows per CTA; 64-key tiles for hd 128 with < 256 virtual rows),
+# the other strides the mma.sync kernel
 @pytest.mark.parametrize("hd,Hq,Hkv,rows,ctx,causal,pad", [
     (64, 4, 4, 70, 0, False, 5), (64, 4, 2, 64, 0, True, 5), (128, 4, 2, 32, 37, False, 5),
     (128, 2, 1, 100, 130, True, 5), (64, 12, 12, 1024, 0, False, 0), (64, 4, 2, 300, 77, True, 3),
-    (128, 4, 2, 260, 0, False, 4), (128, 2, 2, 512, 200, True, 0), (64, 2, 1, 200, 0, False, 1)])
+    (128, 4, 2, 260, 0, False, 4), (128, 2, 2, 512, 200, True, 0), (64, 2, 1, 200, 0, False, 1),
+    # short rows on tcgen05: GQA group packing, heads straddling a 128-row tile, causal
+    (128, 4, 2, 32, 37, False, 3), (128, 16, 8, 32, 200, True, 0), (64, 4, 2, 48, 40, True, 0),
+    (128, 2, 1, 100, 130, True, 2), (64, 8, 2, 20, 300, False, 0)])
 def test_attention_bf16(T, hd, Hq, Hkv, rows, ctx, causal, pad):
     B, stride = 2, ctx + rows + pad
     q, qd = bf16_tensor((B, Hq, rows, hd), 5)
@@ -159,3 +164,35 @@ def test_head_confidence_fused(T, rows, d, V, dtype):
     assert np.max(np.abs(conf.cpu().numpy() - rc) / rc) < 4e-6
     lf = xd @ wd.T                                   # fp64 from the same inputs
     assert np.linalg.norm(logits.cpu().numpy() - lf) / np.linalg.norm(lf) < 1e-5
+
+
+@pytest.mark.parametrize("hd,Hq,Hkv,rows,ctx,causal", [(128, 4, 2, 32, 40, False), (128, 4, 2, 32, 72, True),
+                                                      (64, 4, 2, 32, 40, False)])
+def test_attention_short_rows_tcgen05_as_accurate_as_mma_sync(T, hd, Hq, Hkv, rows, ctx, causal):
+    """The same Q, K, V through the tcgen05 kernel (KV stride a multiple of 8)
+    and the mma.sync kernel (stride one more): both within the bf16-P bound of
+    the fp64 reference, and the tcgen05 error no larger than 1.5x the other's."""
+    B = 2
+    L = ctx + rows
+    q, qd = bf16_tensor((B, Hq, rows, hd), 15)
+    k8, kd = bf16_tensor((B, Hkv, L, hd), 16)
+    vt8, vtd = bf16_tensor((B, Hkv, hd, L), 17)
+    errs = []
+    for stride in (L + (-L) % 8, L + (-L) % 8 + 1):
+        k = torch.zeros((B, Hkv, stride, hd), dtype=torch.bfloat16, device="cuda")
+        vt = torch.zeros((B, Hkv, hd, stride), dtype=torch.bfloat16, device="cuda")
+        k[:, :, :L] = k8
+        vt[..., :L] = vt8
+        o = torch.empty((B * rows, Hq * hd), dtype=torch.bfloat16, device="cuda")
+        T.tadm_attention(q, k, vt, o, Hq, Hkv, rows, ctx, causal, dtype=1)
+        torch.cuda.synchronize()
+        got = o.float().cpu().numpy().astype(np.float64).reshape(B, rows, Hq, hd)
+        e = 0.0
+        for b in range(B):
+            ref = O.attention(qd[b], kd[b], vtd[b].transpose(0, 2, 1), ctx + np.arange(rows), np.arange(L),
+                              causal).transpose(1, 0, 2)
+            e = max(e, np.linalg.norm(got[b] - ref) / np.linalg.norm(ref))
+        errs.append(e)
+    print(f"[short-row attention hd {hd}] rel-L2 tcgen05 {errs[0]:.2e}  mma.sync {errs[1]:.2e}")
+    assert errs[0] < 1e-2 and errs[1] < 1e-2
+    assert errs[0] <= 1.5 * errs[1], errs
