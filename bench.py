@@ -316,12 +316,12 @@ def gpu_arm(args):
                 "probe": "one extra generation with events around every GEMM / attention / norm launch",
                 "by_epilogue": {k: {"ms_per_step": v["ms"], "tflops": round(v["tflops"], 1),
                                     "launches_per_step": v["launches"]}
-                                for k, v in gemm_kinds.items() if k not in ("attention", "norms")},
+                                for k, v in gemm_kinds.items() if k not in ("attention", "norms", "attention_short_rows")},
                 # the other probed launches of the step: attention (FLOP/s) and the norms
                 "others": {k: {"ms_per_step": v["ms"], "share_of_step": v["ms"] / (ms / args.steps) if ms else None,
-                               "tflops": round(v["tflops"], 1) if k == "attention" else None,
+                               "tflops": round(v["tflops"], 1) if k.startswith("attention") else None,
                                "launches_per_step": v["launches"]}
-                           for k, v in gemm_kinds.items() if k in ("attention", "norms")}}
+                           for k, v in gemm_kinds.items() if k in ("attention", "norms", "attention_short_rows")}}
 
     line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
@@ -358,7 +358,17 @@ def kernel_bench(args):
     from paper_2609_37924_gb300 import tadm
     kind, shape = args.kernel_bench.split(":")
     g = torch.Generator(device="cuda").manual_seed(0)
-    if kind == "attn":
+    if kind == "attnctx":
+        # attnctx:B,H,Hkv,R,ctx,hd  R canvas rows over ctx committed keys + themselves (block-step shape), bf16
+        B, H, Hkv, R, ctx, hd = (int(x) for x in shape.split(","))
+        stride = (ctx + R + 7) // 8 * 8
+        q = torch.randn((B, H, R, hd), device="cuda", generator=g).to(torch.bfloat16)
+        k = torch.randn((B, Hkv, stride, hd), device="cuda", generator=g).to(torch.bfloat16)
+        v = torch.randn((B, Hkv, hd, stride), device="cuda", generator=g).to(torch.bfloat16)
+        o = torch.empty((B * R, H * hd), device="cuda", dtype=torch.bfloat16)
+        run = lambda: tadm.tadm_attention(q, k, v, o, H, Hkv, R, ctx, False, dtype=1)  # noqa: E731
+        flops = 4.0 * B * H * R * (ctx + R) * hd
+    elif kind == "attn":
         # attn:B,H,Hkv,R,hd  bidirectional attention of R rows (no context), bf16
         B, H, Hkv, R, hd = (int(x) for x in shape.split(","))
         q = torch.randn((B, H, R, hd), device="cuda", generator=g).to(torch.bfloat16)
@@ -384,7 +394,10 @@ def kernel_bench(args):
     e1.record()
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1) / args.steps
-    print(json.dumps({"kernel": kind, "shape": shape, "ms": ms, "tflops": flops / (ms / 1000.0) / 1e12}), flush=True)
+    line = {"kernel": kind, "shape": shape, "ms": ms, "tflops": flops / (ms / 1000.0) / 1e12}
+    if kind == "attnctx":   # K and V bytes read once per launch
+        line["kv_gbs"] = 2 * k.numel() * (ctx + R) / stride * 2 / (ms / 1000.0) / 1e9
+    print(json.dumps(line), flush=True)
 
 
 def workload_sweep(args):

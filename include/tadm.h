@@ -225,7 +225,7 @@ TADM_API tadm_status tadm_probe_read(tadm_handle* h, int64_t* launches, double* 
 /* The records split by kind: GEMM epilogues 0 plain, 1 residual, 2 QKV +
  * RoPE, 3 GLU, 4 fusion gate/hidden, 5 fusion output, 6 output head,
  * 7..10 paired-attention fusion; 11 attention; 12 RMSNorm / LayerNorm
- * launches.  Arrays of n_kinds entries.  Call before tadm_probe_read, which
+ * launches; 13 attention over fewer than 128 canvas rows (block steps).  Arrays of n_kinds entries.  Call before tadm_probe_read, which
  * clears the records. */
 TADM_API tadm_status tadm_probe_breakdown(tadm_handle* h, int n_kinds, int64_t* launches, double* ms,
                                           double* flops);

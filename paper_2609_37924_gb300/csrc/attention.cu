@@ -70,6 +70,7 @@ template <int HD, int TKV>
 __global__ void __launch_bounds__(192, AttnTcCfg<HD, TKV>::MIN_BLOCKS)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
                    const AttnTcArgs args) {
+  pdl_enter();
   using C = AttnTcCfg<HD, TKV>;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = smem_raw;
@@ -147,6 +148,11 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD, TKV>::MIN_BLOCKS)
         for (int s = 0; s < TKV / 64; ++s)
           tma_load_3d(sV + st * C::V_BYTES + s * HD * 128, &tmV, &kv_full[st], j * TKV + 64 * s, 0, z);
         if (st) ++issued1; else ++issued0;
+        // two stages hold tiles i and i+1; L2 fetches tile i+2 meanwhile
+        if (i + 2 < n_tiles) {
+          for (int s = 0; s < HD / 64; ++s) tma_prefetch_3d(&tmK, 64 * s, (j + 2) * TKV, z);
+          for (int s = 0; s < TKV / 64; ++s) tma_prefetch_3d(&tmV, (j + 2) * TKV + 64 * s, 0, z);
+        }
       }
       // every copy started here has landed before the CTA may exit
       volatile int never = 0;
@@ -383,6 +389,7 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(const float* __restri
                                                            const float2* __restrict__ part_ml, int splits,
                                                            int n_bk, int n_virt, int rows, int n_heads,
                                                            int n_kv_heads, bf16* __restrict__ o) {
+  pdl_enter();
   constexpr int PL = HD / 32;   // dims per lane
   const int lane = threadIdx.x & 31;
   const int g = blockIdx.x * 8 + (threadIdx.x >> 5);
@@ -468,13 +475,15 @@ const char* launch_tc(const AttnCall& a, cudaStream_t s) {
   const int n_vtiles = (n_virt + TQ - 1) / TQ;
   const int base = n_vtiles * a.n_kv_heads * a.batch;
   const int kv_tiles = (kv_len + TKV - 1) / TKV;
-  // split the keys when the CTAs would not fill two waves: every split keeps
-  // >= 3 tiles and its fp32 partials fit the caller's scratch
+  // split the keys only into as many ranges as the resident CTA slots leave
+  // room for (splitting adds partial traffic and a merge, it only pays for
+  // idle SMs): every split keeps >= 3 tiles and its fp32 partials fit the
+  // caller's scratch
   int splits = 1;
   if (a.part && a.part_bytes > 0) {
     const int slots = C::MIN_BLOCKS * n_sms;
     const size_t per_split = static_cast<size_t>(a.batch) * a.n_kv_heads * n_virt * (HD + 2) * sizeof(float);
-    splits = std::min(std::min((2 * slots + base - 1) / base, kv_tiles / 3), 8);
+    splits = std::min(std::min(slots / base, kv_tiles / 3), 8);
     while (splits > 1 && static_cast<size_t>(splits) * per_split > a.part_bytes) --splits;
     if (splits < 1) splits = 1;
   }
@@ -486,13 +495,13 @@ const char* launch_tc(const AttnCall& a, cudaStream_t s) {
                   1.4426950408889634f / sqrtf(static_cast<float>(HD)), static_cast<bf16*>(a.o),
                   n_vtiles, splits, tps, part_o, part_ml, a.status};
   dim3 grid(n_vtiles * splits, a.n_kv_heads, a.batch);
-  attn_tc_kernel<HD, TKV><<<grid, 192, C::SMEM, s>>>(mk, mv, args);
+  launch_pdl(attn_tc_kernel<HD, TKV>, grid, 192, C::SMEM, s, mk, mv, args);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cudaGetErrorString(e);
   if (splits > 1) {
     const int n_bk = a.batch * a.n_kv_heads;
     const int rows_total = n_bk * n_virt;
-    attn_combine_kernel<HD><<<(rows_total + 7) / 8, 256, 0, s>>>(part_o, part_ml, splits, n_bk, n_virt, a.rows,
+    launch_pdl(attn_combine_kernel<HD>, (rows_total + 7) / 8, 256, 0, s, part_o, part_ml, splits, n_bk, n_virt, a.rows,
                                                                a.n_heads, a.n_kv_heads, static_cast<bf16*>(a.o));
     e = cudaGetLastError();
     if (e != cudaSuccess) return cudaGetErrorString(e);
@@ -533,6 +542,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const bf16* __restrict__
                                                         const bf16* __restrict__ vt, bf16* __restrict__ o,
                                                         int n_heads, int n_kv_heads, int rows, int ctx,
                                                         int kv_stride, int causal, float scale_log2) {
+  pdl_enter();
   constexpr int LD = HD + 8;   // padded smem row of Q / K (bf16)
   constexpr int LDV = AN + 8;  // padded smem row of V^T (one head dim, AN keys)
   extern __shared__ __align__(16) uint8_t smem_raw[];
@@ -717,6 +727,7 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const float* __restrict__
                                                        const float* __restrict__ vt, float* __restrict__ o,
                                                        int n_heads, int n_kv_heads, int rows, int ctx,
                                                        int kv_stride, int causal, float scale) {
+  pdl_enter();
   constexpr int PL = HD / 32;
   const int lane = threadIdx.x & 31;
   const int row = blockIdx.x * 4 + (threadIdx.x >> 5);
@@ -763,7 +774,7 @@ cudaError_t launch_bf16(const AttnCall& a, cudaStream_t s) {
   const int n_virt = (a.n_heads / a.n_kv_heads) * a.rows;
   dim3 grid((n_virt + AM - 1) / AM, a.n_kv_heads, a.batch);
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(HD));
-  attn_bf16_kernel<HD><<<grid, 128, smem, s>>>(static_cast<const bf16*>(a.q), static_cast<const bf16*>(a.k),
+  launch_pdl(attn_bf16_kernel<HD>, grid, 128, smem, s, static_cast<const bf16*>(a.q), static_cast<const bf16*>(a.k),
                                                static_cast<const bf16*>(a.v), static_cast<bf16*>(a.o), a.n_heads,
                                                a.n_kv_heads, a.rows, a.ctx, a.kv_stride, a.causal, scale_log2);
   return cudaGetLastError();
@@ -772,7 +783,7 @@ cudaError_t launch_bf16(const AttnCall& a, cudaStream_t s) {
 template <int HD>
 cudaError_t launch_f32(const AttnCall& a, cudaStream_t s) {
   dim3 grid((a.rows + 3) / 4, a.n_heads, a.batch);
-  attn_f32_kernel<HD><<<grid, 128, 0, s>>>(static_cast<const float*>(a.q), static_cast<const float*>(a.k),
+  launch_pdl(attn_f32_kernel<HD>, grid, 128, 0, s, static_cast<const float*>(a.q), static_cast<const float*>(a.k),
                                            static_cast<const float*>(a.v), static_cast<float*>(a.o), a.n_heads,
                                            a.n_kv_heads, a.rows, a.ctx, a.kv_stride, a.causal,
                                            1.0f / sqrtf(static_cast<float>(HD)));

@@ -119,6 +119,13 @@ __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, u
       "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y), "r"(z)
       : "memory");
 }
+// Asks L2 for a 3-D box of a tensor map (no shared memory, no completion).
+__device__ __forceinline__ void tma_prefetch_3d(const CUtensorMap* map, int x, int y, int z) {
+  asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];" ::"l"(
+                   reinterpret_cast<uint64_t>(map)),
+               "r"(x), "r"(y), "r"(z)
+               : "memory");
+}
 // TMA tensor store of a 2-D box from shared memory (bulk-group completion).
 __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* src, int x, int y) {
   asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
@@ -180,6 +187,17 @@ __device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t a_desc, uint
       : "memory");
 }
 // Arrive once on `bar` when every tcgen05 op issued so far by this thread is done.
+// -------------------------------------------- programmatic dependent launch
+// Every kernel of the library calls this before its first global-memory
+// access: it waits until the previous kernel of the stream has completed and
+// its writes are visible (a no-op when there is no programmatic dependency),
+// then lets the next kernel start launching; that kernel's CTAs wait in this
+// same call before they touch memory, so only launch latency overlaps.
+__device__ __forceinline__ void pdl_enter() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ------------------------------------------------- CTA pairs (cluster of 2)
 // A pair of CTAs in one 2-CTA cluster runs one tcgen05.mma.cta_group::2: the
 // even CTA (rank 0) issues it; each CTA holds half of A (its rows of D) and

@@ -24,6 +24,7 @@ template <int EPI>
 __global__ void __launch_bounds__(256) gemm_simt_kernel(const float* __restrict__ A, const float* __restrict__ B,
                                                         int M, int K, int lda, int ldb, int n_rows_b,
                                                         int b_split, EpiParams ep) {
+  pdl_enter();
   __shared__ float sA[TK][TM + 4];
   __shared__ float sB[TK][TN + 4];
   __shared__ float sC[TM][TN + 1];
@@ -68,7 +69,7 @@ __global__ void __launch_bounds__(256) gemm_simt_kernel(const float* __restrict_
 template <int EPI>
 cudaError_t launch(const GemmCall& g, int tiles_n, int b_split, int n_rows_b, const EpiParams& ep, cudaStream_t s) {
   dim3 grid(tiles_n, (g.M + TM - 1) / TM);
-  gemm_simt_kernel<EPI><<<grid, 256, 0, s>>>(static_cast<const float*>(g.A), static_cast<const float*>(g.B), g.M,
+  launch_pdl(gemm_simt_kernel<EPI>, grid, 256, 0, s, static_cast<const float*>(g.A), static_cast<const float*>(g.B), g.M,
                                              g.K, g.lda, g.ldb, n_rows_b, b_split, ep);
   return cudaGetLastError();
 }

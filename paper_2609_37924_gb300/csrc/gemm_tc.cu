@@ -143,6 +143,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmC2,
                    const TcArgs args) {
+  pdl_enter();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sA = smem;
@@ -330,6 +331,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmC2,
                     const TcArgs args) {
+  pdl_enter();
   using PC = PairCfg<PBN>;
   constexpr int P_STAGES = PC::STAGES, P_A_BYTES = PC::A_BYTES, P_B_BYTES = PC::B_BYTES;
   constexpr int P_STAGE_BYTES = PC::STAGE_BYTES;
@@ -550,7 +552,7 @@ cudaError_t launch_epi(const CUtensorMap& ta, const CUtensorMap& tb, const CUten
     if (e != cudaSuccess) return e;
     attr_set = true;
   }
-  gemm_tc_kernel<EPI><<<grid, NUM_THREADS, SMEM_BYTES, s>>>(ta, tb, tc, tc2, a);
+  launch_pdl(gemm_tc_kernel<EPI>, grid, NUM_THREADS, SMEM_BYTES, s, ta, tb, tc, tc2, a);
   return cudaGetLastError();
 }
 
@@ -578,7 +580,7 @@ cudaError_t launch_epi_pair(const CUtensorMap& ta, const CUtensorMap& tb, const 
     max_clusters = n;
   }
   const int clusters = std::min(pairs, max_clusters);
-  gemm_tc2_kernel<EPI, PBN><<<2 * clusters, NUM_THREADS, smem, s>>>(ta, tb, tc, tc2, a);
+  launch_pdl(gemm_tc2_kernel<EPI, PBN>, 2 * clusters, NUM_THREADS, smem, s, ta, tb, tc, tc2, a);
   return cudaGetLastError();
 }
 

@@ -4,9 +4,20 @@
 // LayerNorm of the gated-MLP fusion (App. C.2), the RMS scales and feature
 // concatenations of the paired-attention fusion (App. C.1), the RoPE table,
 // and canvas set-up.
+#include <cstdlib>
+
 #include "kernels.h"
 
 namespace tadm {
+
+bool pdl_enabled() {
+  static const bool on = [] {
+    const char* e = getenv("TADM_PDL");
+    return !(e && e[0] == '0');
+  }();
+  return on;
+}
+
 namespace {
 
 constexpr int WPB = 8;  // warps (rows) per block
@@ -26,6 +37,7 @@ __device__ __forceinline__ float ldw(const void* w, int bf, int i) {
 
 __global__ void embed_kernel(const int32_t* __restrict__ z, int ldz, int rows, int M, const void* __restrict__ E,
                              int e_bf16, int d, int vocab, float* __restrict__ out, float* __restrict__ out2) {
+  pdl_enter();
   const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (m >= M) return;
   const int b = m / rows, r = m - b * rows;
@@ -56,6 +68,7 @@ __global__ void __launch_bounds__(256) rmsnorm_block_kernel(const float* __restr
                                                             const void* __restrict__ gain, int w_bf16, float eps,
                                                             void* __restrict__ out, int ldo,
                                                             const int32_t* __restrict__ rows_idx) {
+  pdl_enter();
   __shared__ float red[8];
   const int m = blockIdx.x;
   const float* xr = x + static_cast<size_t>(rows_idx ? rows_idx[m] : m) * d;
@@ -85,6 +98,7 @@ __global__ void __launch_bounds__(256) rmsnorm_block_kernel(const float* __restr
 template <class T>
 __global__ void rmsnorm_kernel(const float* __restrict__ x, int M, int d, const void* __restrict__ gain, int w_bf16,
                                float eps, void* __restrict__ out, int ldo, const int32_t* __restrict__ rows_idx) {
+  pdl_enter();
   const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (m >= M) return;
   const float* xr = x + static_cast<size_t>(rows_idx ? rows_idx[m] : m) * d;
@@ -114,6 +128,7 @@ __global__ void __launch_bounds__(WPB * 32) rmsnorm_reg_kernel(const float* __re
                                                                const bf16* __restrict__ gain, float eps,
                                                                bf16* __restrict__ out, int ldo,
                                                                const int32_t* __restrict__ rows_idx) {
+  pdl_enter();
   constexpr int d = 256 * NCH;
   const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (m >= M) return;
@@ -170,6 +185,7 @@ template <class T>
 __global__ void ln_pair_kernel(const float* __restrict__ c, const float* __restrict__ h, int M, int d,
                                const void* wc, const void* bc, const void* wh, const void* bh, int w_bf16, float eps,
                                void* __restrict__ u) {
+  pdl_enter();
   const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (m >= M) return;
   for (int part = 0; part < 2; ++part) {
@@ -186,6 +202,7 @@ __global__ void ln_pair_kernel(const float* __restrict__ c, const float* __restr
 
 __global__ void layernorm_kernel(const float* __restrict__ x, int M, int d, const void* w, const void* b, int w_bf16,
                                  float eps, float* __restrict__ out) {
+  pdl_enter();
   const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (m >= M) return;
   const float* xr = x + static_cast<size_t>(m) * d;
@@ -196,6 +213,7 @@ __global__ void layernorm_kernel(const float* __restrict__ x, int M, int d, cons
 }
 
 __global__ void rms_scale_kernel(const float* __restrict__ x, int M, int d, float eps, float* __restrict__ s) {
+  pdl_enter();
   const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (m >= M) return;
   const float* xr = x + static_cast<size_t>(m) * d;
@@ -208,6 +226,7 @@ __global__ void rms_scale_kernel(const float* __restrict__ x, int M, int d, floa
 template <class T>
 __global__ void scale_rows_kernel(const float* __restrict__ x, const float* __restrict__ sc, int M, int d,
                                   void* __restrict__ out) {
+  pdl_enter();
   const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (m >= M) return;
   const float s = sc[m];
@@ -223,6 +242,7 @@ struct Parts {
 
 template <class T>
 __global__ void concat_kernel(Parts parts, int M, int width, void* __restrict__ out) {
+  pdl_enter();
   const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (m >= M) return;
   int col = 0;
@@ -234,6 +254,7 @@ __global__ void concat_kernel(Parts parts, int M, int width, void* __restrict__ 
 }
 
 __global__ void sub_kernel(const float* __restrict__ a, const float* __restrict__ b, size_t n, float* __restrict__ o) {
+  pdl_enter();
   for (size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x; i < n;
        i += static_cast<size_t>(gridDim.x) * blockDim.x)
     o[i] = a[i] - b[i];
@@ -241,6 +262,7 @@ __global__ void sub_kernel(const float* __restrict__ a, const float* __restrict_
 
 // tab[j][pos] = (cos, sin)(pos * theta^(-2j/hd)), angles evaluated in double
 __global__ void rope_table_kernel(float2* tab, int n_pos, int half, int hd, double theta) {
+  pdl_enter();
   const size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x;
   if (i >= static_cast<size_t>(n_pos) * half) return;
   const int j = static_cast<int>(i / n_pos), pos = static_cast<int>(i % n_pos);
@@ -251,6 +273,7 @@ __global__ void rope_table_kernel(float2* tab, int n_pos, int half, int hd, doub
 
 __global__ void fill_canvas_kernel(int32_t* z, int ldz, const int32_t* prompt, int batch, int P, int total,
                                    int mask_id) {
+  pdl_enter();
   const size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x;
   if (i >= static_cast<size_t>(batch) * total) return;
   const int b = static_cast<int>(i / total), p = static_cast<int>(i % total);
@@ -258,6 +281,7 @@ __global__ void fill_canvas_kernel(int32_t* z, int ldz, const int32_t* prompt, i
 }
 
 __global__ void copy_i32_kernel(const int32_t* src, int lds, int32_t* dst, int ldd, int batch, int cols) {
+  pdl_enter();
   const size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x;
   if (i >= static_cast<size_t>(batch) * cols) return;
   const int b = static_cast<int>(i / cols), c = static_cast<int>(i % cols);
@@ -276,7 +300,7 @@ const char* embed_rows(const int32_t* z, int ldz, int batch, int rows, const voi
   const int M = batch * rows;
   if (M <= 0) return nullptr;
   if (d % 4) return "d_model must be a multiple of 4";
-  embed_kernel<<<rows_grid(M), WPB * 32, 0, s>>>(z, ldz, rows, M, E, e_bf16, d, vocab, out, out2);
+  launch_pdl(embed_kernel, rows_grid(M), WPB * 32, 0, s, z, ldz, rows, M, E, e_bf16, d, vocab, out, out2);
   return err();
 }
 
@@ -285,9 +309,9 @@ const char* rmsnorm_rows(const float* x, int M, int d, const void* gain, int w_b
   if (M <= 0) return nullptr;
   if (M < 1024) {   // few rows: a block per row keeps enough SMs busy
     if (act_bf16)
-      rmsnorm_block_kernel<bf16><<<M, 256, 0, s>>>(x, d, gain, w_bf16, eps, out, ldo, rows_idx);
+      launch_pdl(rmsnorm_block_kernel<bf16>, M, 256, 0, s, x, d, gain, w_bf16, eps, out, ldo, rows_idx);
     else
-      rmsnorm_block_kernel<float><<<M, 256, 0, s>>>(x, d, gain, w_bf16, eps, out, ldo, rows_idx);
+      launch_pdl(rmsnorm_block_kernel<float>, M, 256, 0, s, x, d, gain, w_bf16, eps, out, ldo, rows_idx);
     return err();
   }
   const bool vec = act_bf16 && w_bf16 && ldo % 8 == 0 &&
@@ -296,18 +320,18 @@ const char* rmsnorm_rows(const float* x, int M, int d, const void* gain, int w_b
     const bf16* g = static_cast<const bf16*>(gain);
     bf16* o = static_cast<bf16*>(out);
     switch (d) {
-      case 256: rmsnorm_reg_kernel<1><<<rows_grid(M), WPB * 32, 0, s>>>(x, M, g, eps, o, ldo, rows_idx); return err();
-      case 512: rmsnorm_reg_kernel<2><<<rows_grid(M), WPB * 32, 0, s>>>(x, M, g, eps, o, ldo, rows_idx); return err();
-      case 768: rmsnorm_reg_kernel<3><<<rows_grid(M), WPB * 32, 0, s>>>(x, M, g, eps, o, ldo, rows_idx); return err();
-      case 1024: rmsnorm_reg_kernel<4><<<rows_grid(M), WPB * 32, 0, s>>>(x, M, g, eps, o, ldo, rows_idx); return err();
-      case 2048: rmsnorm_reg_kernel<8><<<rows_grid(M), WPB * 32, 0, s>>>(x, M, g, eps, o, ldo, rows_idx); return err();
+      case 256: launch_pdl(rmsnorm_reg_kernel<1>, rows_grid(M), WPB * 32, 0, s, x, M, g, eps, o, ldo, rows_idx); return err();
+      case 512: launch_pdl(rmsnorm_reg_kernel<2>, rows_grid(M), WPB * 32, 0, s, x, M, g, eps, o, ldo, rows_idx); return err();
+      case 768: launch_pdl(rmsnorm_reg_kernel<3>, rows_grid(M), WPB * 32, 0, s, x, M, g, eps, o, ldo, rows_idx); return err();
+      case 1024: launch_pdl(rmsnorm_reg_kernel<4>, rows_grid(M), WPB * 32, 0, s, x, M, g, eps, o, ldo, rows_idx); return err();
+      case 2048: launch_pdl(rmsnorm_reg_kernel<8>, rows_grid(M), WPB * 32, 0, s, x, M, g, eps, o, ldo, rows_idx); return err();
       default: break;
     }
   }
   if (act_bf16)
-    rmsnorm_kernel<bf16><<<rows_grid(M), WPB * 32, 0, s>>>(x, M, d, gain, w_bf16, eps, out, ldo, rows_idx);
+    launch_pdl(rmsnorm_kernel<bf16>, rows_grid(M), WPB * 32, 0, s, x, M, d, gain, w_bf16, eps, out, ldo, rows_idx);
   else
-    rmsnorm_kernel<float><<<rows_grid(M), WPB * 32, 0, s>>>(x, M, d, gain, w_bf16, eps, out, ldo, rows_idx);
+    launch_pdl(rmsnorm_kernel<float>, rows_grid(M), WPB * 32, 0, s, x, M, d, gain, w_bf16, eps, out, ldo, rows_idx);
   return err();
 }
 
@@ -315,31 +339,31 @@ const char* ln_pair_rows(const float* c, const float* h, int M, int d, const voi
                          const void* bh, int w_bf16, float eps, void* u, int act_bf16, cudaStream_t s) {
   if (M <= 0) return nullptr;
   if (act_bf16)
-    ln_pair_kernel<bf16><<<rows_grid(M), WPB * 32, 0, s>>>(c, h, M, d, wc, bc, wh, bh, w_bf16, eps, u);
+    launch_pdl(ln_pair_kernel<bf16>, rows_grid(M), WPB * 32, 0, s, c, h, M, d, wc, bc, wh, bh, w_bf16, eps, u);
   else
-    ln_pair_kernel<float><<<rows_grid(M), WPB * 32, 0, s>>>(c, h, M, d, wc, bc, wh, bh, w_bf16, eps, u);
+    launch_pdl(ln_pair_kernel<float>, rows_grid(M), WPB * 32, 0, s, c, h, M, d, wc, bc, wh, bh, w_bf16, eps, u);
   return err();
 }
 
 const char* layernorm_rows(const float* x, int M, int d, const void* w, const void* b, int w_bf16, float eps,
                            float* out, cudaStream_t s) {
   if (M <= 0) return nullptr;
-  layernorm_kernel<<<rows_grid(M), WPB * 32, 0, s>>>(x, M, d, w, b, w_bf16, eps, out);
+  launch_pdl(layernorm_kernel, rows_grid(M), WPB * 32, 0, s, x, M, d, w, b, w_bf16, eps, out);
   return err();
 }
 
 const char* rms_scale_rows(const float* x, int M, int d, float eps, float* s_out, cudaStream_t st) {
   if (M <= 0) return nullptr;
-  rms_scale_kernel<<<rows_grid(M), WPB * 32, 0, st>>>(x, M, d, eps, s_out);
+  launch_pdl(rms_scale_kernel, rows_grid(M), WPB * 32, 0, st, x, M, d, eps, s_out);
   return err();
 }
 
 const char* scale_rows(const float* x, const float* sc, int M, int d, void* out, int act_bf16, cudaStream_t s) {
   if (M <= 0) return nullptr;
   if (act_bf16)
-    scale_rows_kernel<bf16><<<rows_grid(M), WPB * 32, 0, s>>>(x, sc, M, d, out);
+    launch_pdl(scale_rows_kernel<bf16>, rows_grid(M), WPB * 32, 0, s, x, sc, M, d, out);
   else
-    scale_rows_kernel<float><<<rows_grid(M), WPB * 32, 0, s>>>(x, sc, M, d, out);
+    launch_pdl(scale_rows_kernel<float>, rows_grid(M), WPB * 32, 0, s, x, sc, M, d, out);
   return err();
 }
 
@@ -356,9 +380,9 @@ const char* concat_rows(const float* const* parts, const int* widths, int n_part
   }
   p.n = n_parts;
   if (act_bf16)
-    concat_kernel<bf16><<<rows_grid(M), WPB * 32, 0, s>>>(p, M, width, out);
+    launch_pdl(concat_kernel<bf16>, rows_grid(M), WPB * 32, 0, s, p, M, width, out);
   else
-    concat_kernel<float><<<rows_grid(M), WPB * 32, 0, s>>>(p, M, width, out);
+    launch_pdl(concat_kernel<float>, rows_grid(M), WPB * 32, 0, s, p, M, width, out);
   return err();
 }
 
@@ -366,14 +390,14 @@ const char* sub_rows(const float* a, const float* b, int M, int d, float* out, c
   const size_t n = static_cast<size_t>(M) * d;
   if (n == 0) return nullptr;
   const int blocks = static_cast<int>((n + 255) / 256 < 65535 ? (n + 255) / 256 : 65535);
-  sub_kernel<<<blocks, 256, 0, s>>>(a, b, n, out);
+  launch_pdl(sub_kernel, blocks, 256, 0, s, a, b, n, out);
   return err();
 }
 
 const char* rope_table(float2* tab, int n_pos, int head_dim, float theta, cudaStream_t s) {
   const size_t n = static_cast<size_t>(n_pos) * (head_dim / 2);
   if (n == 0) return nullptr;
-  rope_table_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, s>>>(tab, n_pos, head_dim / 2, head_dim,
+  launch_pdl(rope_table_kernel, static_cast<unsigned>((n + 255) / 256), 256, 0, s, tab, n_pos, head_dim / 2, head_dim,
                                                                             static_cast<double>(theta));
   return err();
 }
@@ -382,7 +406,7 @@ const char* fill_canvas(int32_t* z, int ldz, const int32_t* prompt, int batch, i
                         int mask_id, cudaStream_t s) {
   const size_t n = static_cast<size_t>(batch) * total;
   if (n == 0) return nullptr;
-  fill_canvas_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, s>>>(z, ldz, prompt, batch, prompt_len,
+  launch_pdl(fill_canvas_kernel, static_cast<unsigned>((n + 255) / 256), 256, 0, s, z, ldz, prompt, batch, prompt_len,
                                                                              total, mask_id);
   return err();
 }
@@ -390,7 +414,7 @@ const char* fill_canvas(int32_t* z, int ldz, const int32_t* prompt, int batch, i
 const char* copy_rows_i32(const int32_t* src, int lds, int32_t* dst, int ldd, int batch, int cols, cudaStream_t s) {
   const size_t n = static_cast<size_t>(batch) * cols;
   if (n == 0) return nullptr;
-  copy_i32_kernel<<<static_cast<unsigned>((n + 255) / 256), 256, 0, s>>>(src, lds, dst, ldd, batch, cols);
+  launch_pdl(copy_i32_kernel, static_cast<unsigned>((n + 255) / 256), 256, 0, s, src, lds, dst, ldd, batch, cols);
   return err();
 }
 

@@ -48,6 +48,7 @@ __device__ __forceinline__ void block_argmax(float& v, int& i, float* sv, int* s
 __global__ void __launch_bounds__(256) confidence_kernel(const float* __restrict__ logits, int vocab, int ld,
                                                          int mask_id, float* __restrict__ conf,
                                                          int32_t* __restrict__ tok) {
+  pdl_enter();
   __shared__ float sv[32];
   __shared__ int si[32];
   const float* l = logits + static_cast<size_t>(blockIdx.x) * ld;
@@ -77,6 +78,7 @@ __global__ void __launch_bounds__(256) confidence_kernel(const float* __restrict
 // written by the output-head GEMM epilogue.
 __global__ void combine_kernel(const float* __restrict__ part, int rows, int n_tiles, float* __restrict__ conf,
                                int32_t* __restrict__ tok, const int32_t* __restrict__ rows_idx) {
+  pdl_enter();
   const int r = blockIdx.x * 8 + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (r >= rows) return;
   const float* p = part + static_cast<size_t>(r) * n_tiles * 3;
@@ -110,6 +112,7 @@ __global__ void combine_kernel(const float* __restrict__ part, int rows, int n_t
 __global__ void __launch_bounds__(256) masked_rows_kernel(const int32_t* __restrict__ z, int ldz, int rows,
                                                           int mask_id, int per_seq, int32_t* __restrict__ idx,
                                                           float* __restrict__ conf) {
+  pdl_enter();
   __shared__ int base;
   __shared__ int wsum[8];
   const int b = blockIdx.x;
@@ -147,6 +150,7 @@ __global__ void __launch_bounds__(256) masked_rows_kernel(const int32_t* __restr
 __global__ void __launch_bounds__(256) topk_kernel(int32_t* __restrict__ z, int ldz, const float* __restrict__ conf,
                                                    const int32_t* __restrict__ tok, int rows, int k, int mask_id,
                                                    int32_t* __restrict__ selected) {
+  pdl_enter();
   __shared__ float sv[32];
   __shared__ int si[32];
   const int b = blockIdx.x;
@@ -182,28 +186,28 @@ inline const char* err() {
 const char* confidence_rows(const float* logits, int rows, int vocab, int ld, int mask_id, float* conf, int32_t* tok,
                             cudaStream_t s) {
   if (rows <= 0) return nullptr;
-  confidence_kernel<<<rows, 256, 0, s>>>(logits, vocab, ld, mask_id, conf, tok);
+  launch_pdl(confidence_kernel, rows, 256, 0, s, logits, vocab, ld, mask_id, conf, tok);
   return err();
 }
 
 const char* combine_partials(const float* part, int rows, int n_tiles, float* conf, int32_t* tok, cudaStream_t s,
                              const int32_t* rows_idx) {
   if (rows <= 0) return nullptr;
-  combine_kernel<<<(rows + 7) / 8, 256, 0, s>>>(part, rows, n_tiles, conf, tok, rows_idx);
+  launch_pdl(combine_kernel, (rows + 7) / 8, 256, 0, s, part, rows, n_tiles, conf, tok, rows_idx);
   return err();
 }
 
 const char* masked_rows(const int32_t* z, int ldz, int batch, int rows, int mask_id, int per_seq, int32_t* idx,
                         float* conf, cudaStream_t s) {
   if (batch <= 0 || rows <= 0) return nullptr;
-  masked_rows_kernel<<<batch, 256, 0, s>>>(z, ldz, rows, mask_id, per_seq, idx, conf);
+  launch_pdl(masked_rows_kernel, batch, 256, 0, s, z, ldz, rows, mask_id, per_seq, idx, conf);
   return err();
 }
 
 const char* topk_unmask(int32_t* z, int ldz, const float* conf, const int32_t* tok, int batch, int rows, int k,
                         int mask_id, int32_t* selected, cudaStream_t s) {
   if (batch <= 0 || rows <= 0 || k <= 0) return nullptr;
-  topk_kernel<<<batch, 256, 0, s>>>(z, ldz, conf, tok, rows, k, mask_id, selected);
+  launch_pdl(topk_kernel, batch, 256, 0, s, z, ldz, conf, tok, rows, k, mask_id, selected);
   return err();
 }
 

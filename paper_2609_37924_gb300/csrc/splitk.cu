@@ -43,6 +43,7 @@ __device__ __forceinline__ int reduce_groups(const EpiParams& ep) {
 template <int EPI>
 __global__ void __launch_bounds__(256) splitk_reduce_kernel(EpiParams ep, const float* __restrict__ part,
                                                             size_t stride, int ldp, int splits) {
+  pdl_enter();
   const int m = blockIdx.x * 32 + (threadIdx.x & 31), slot = threadIdx.x >> 5, nb = blockIdx.y;
   const int groups = reduce_groups<EPI>(ep);
   if (m >= ep.M || slot >= groups) return;
@@ -53,6 +54,7 @@ __global__ void __launch_bounds__(256) splitk_reduce_kernel(EpiParams ep, const 
 // Phase 1: slice 0 <- sum of all slices in slice order, one float4 per thread.
 __global__ void __launch_bounds__(256) splitk_sum_kernel(float* __restrict__ part, size_t stride, size_t n4,
                                                          int splits) {
+  pdl_enter();
   const size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x;
   if (i >= n4) return;
   float4* p = reinterpret_cast<float4*>(part);
@@ -69,10 +71,10 @@ template <int EPI>
 cudaError_t launch(const EpiParams& ep, const float* part, size_t stride, int ldp, int splits, int n_tiles_n,
                    cudaStream_t s) {
   const size_t n4 = static_cast<size_t>(ep.M) * ldp / 4;
-  splitk_sum_kernel<<<static_cast<unsigned>((n4 + 255) / 256), 256, 0, s>>>(const_cast<float*>(part), stride, n4,
+  launch_pdl(splitk_sum_kernel, static_cast<unsigned>((n4 + 255) / 256), 256, 0, s, const_cast<float*>(part), stride, n4,
                                                                             splits);
   dim3 grid((ep.M + 31) / 32, n_tiles_n);
-  splitk_reduce_kernel<EPI><<<grid, 256, 0, s>>>(ep, part, stride, ldp, 1);
+  launch_pdl(splitk_reduce_kernel<EPI>, grid, 256, 0, s, ep, part, stride, ldp, 1);
   return cudaGetLastError();
 }
 }  // namespace

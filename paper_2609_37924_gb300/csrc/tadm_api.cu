@@ -264,7 +264,7 @@ void layout(tadm_handle* h) {
 
 // --------------------------------------------------------------------------- kernels wrappers
 // probe kinds beyond the GEMM epilogues (0..10)
-constexpr int kProbeAttention = 11, kProbeNorm = 12;
+constexpr int kProbeAttention = 11, kProbeNorm = 12, kProbeAttentionShort = 13;   // 13: attention of < 128 rows
 // Opens a probe record (start event) when the probe is on and has room: returns its index, else -1.
 int probe_begin(tadm_handle* h, cudaStream_t s) {
   if (h->probe_next >= static_cast<int>(h->probe_flops.size())) return -1;
@@ -348,7 +348,7 @@ tadm_status layer_fwd(tadm_handle* h, int li, float* x, int B, int R, int ctx, i
   TRY(attention(a, s));
   // keys seen per query row: all of them, or the causal average
   const double keys = causal ? ctx + 0.5 * (R + 1) : static_cast<double>(ctx + R);
-  probe_end(h, s, pi, kProbeAttention, 4.0 * M * c.n_heads * keys * hd);
+  probe_end(h, s, pi, R < 128 ? kProbeAttentionShort : kProbeAttention, 4.0 * M * c.n_heads * keys * hd);
   EpiParams er{};
   er.resid = x;
   er.ldr = d;

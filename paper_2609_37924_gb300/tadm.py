@@ -305,7 +305,7 @@ class TadmModel:
         _check(self.lib.tadm_probe_enable(self.h, max_launches), self.h)
 
     EPI_NAMES = ["plain", "residual", "qkv_rope", "glu", "fusion_gate_hidden", "fusion_out", "output_head",
-                 "pa_up", "pa_silu", "pa_add", "pa_gate", "attention", "norms"]
+                 "pa_up", "pa_silu", "pa_add", "pa_gate", "attention", "norms", "attention_short_rows"]
     N_GEMM_KINDS = 11
 
     def tadm_probe_breakdown(self) -> dict:
