@@ -7,6 +7,7 @@
 // anchor cache of tadm_generate, the RoPE table and the status word.
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <string>
 #include <vector>
@@ -134,6 +135,17 @@ struct tadm_handle {
   tadm_counters counters{};
   cudaStream_t last_stream = nullptr;
   std::string err;
+
+  // CUDA graph of a repeated tadm_generate call (same sizes and pointers):
+  // the second such call is captured on an internal stream, later ones replay
+  // it.  The host-side results of the captured run (counters, context length)
+  // are restored on replay.
+  cudaStream_t gstream = nullptr;
+  cudaEvent_t gev_in = nullptr, gev_out = nullptr;
+  cudaGraphExec_t gexec = nullptr;
+  int64_t gkey[8] = {}, gkey_seen[8] = {};
+  tadm_counters gcounters{};
+  int gctx = 0;
 
   int es() const { return cfg.dtype ? 2 : 4; }
   int act_bf16() const { return cfg.dtype; }
@@ -752,7 +764,13 @@ tadm_status tadm_create(const tadm_config* cfg, const void* const* weights, int 
 }
 
 void tadm_destroy(tadm_handle* h) {
-  if (h) tadm_probe_enable(h, 0);
+  if (h) {
+    tadm_probe_enable(h, 0);
+    if (h->gexec) cudaGraphExecDestroy(h->gexec);
+    if (h->gev_in) cudaEventDestroy(h->gev_in);
+    if (h->gev_out) cudaEventDestroy(h->gev_out);
+    if (h->gstream) cudaStreamDestroy(h->gstream);
+  }
   delete h;
 }
 
@@ -911,6 +929,9 @@ tadm_status tadm_layer_cost(int L_S, int L_A, int L_D, int T, int K, int64_t* c_
   return TADM_OK;
 }
 
+tadm_status generate_loop(tadm_handle* h, const int32_t* prompt, int batch, int prompt_len, int32_t* out,
+                          int gen_len, int steps_per_block, int K, int block_len, cudaStream_t s);
+
 tadm_status tadm_generate(tadm_handle* h, const int32_t* prompt, int batch, int prompt_len, int32_t* out, int gen_len,
                           int steps_per_block, int K, int block_len, tadm_stream stream) {
   if (!h) return TADM_ERR_INVALID_ARG;
@@ -925,7 +946,68 @@ tadm_status tadm_generate(tadm_handle* h, const int32_t* prompt, int batch, int 
   TRYS(tadm_reset(h, batch));
   TRYS(check_ready(h, batch, R));
   h->last_stream = stream;
-  cudaStream_t s = stream;
+  static const bool graphs_on = [] {
+    const char* e = getenv("TADM_GRAPH");
+    return !(e && e[0] == '0');
+  }();
+  const int64_t key[8] = {batch, prompt_len, gen_len, steps_per_block, K, block_len,
+                          static_cast<int64_t>(reinterpret_cast<uintptr_t>(prompt)),
+                          static_cast<int64_t>(reinterpret_cast<uintptr_t>(out))};
+  if (!graphs_on || !h->probe_flops.empty()) return generate_loop(h, prompt, batch, prompt_len, out, gen_len,
+                                                                  steps_per_block, K, block_len, stream);
+  const bool seen = std::memcmp(key, h->gkey_seen, sizeof(key)) == 0;
+  std::memcpy(h->gkey_seen, key, sizeof(key));
+  if (!seen && !(h->gexec && std::memcmp(key, h->gkey, sizeof(key)) == 0))   // first call: eager
+    return generate_loop(h, prompt, batch, prompt_len, out, gen_len, steps_per_block, K, block_len, stream);
+  if (!h->gstream) {
+    if (cudaStreamCreateWithFlags(&h->gstream, cudaStreamNonBlocking) != cudaSuccess ||
+        cudaEventCreateWithFlags(&h->gev_in, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&h->gev_out, cudaEventDisableTiming) != cudaSuccess)
+      return fail(h, TADM_ERR_CUDA, "graph stream / events");
+  }
+  if (!(h->gexec && std::memcmp(key, h->gkey, sizeof(key)) == 0)) {
+    // second identical call: capture the whole generation on the internal stream
+    if (h->gexec) {
+      cudaGraphExecDestroy(h->gexec);
+      h->gexec = nullptr;
+    }
+    if (cudaStreamBeginCapture(h->gstream, cudaStreamCaptureModeThreadLocal) != cudaSuccess)
+      return fail(h, TADM_ERR_CUDA, "begin graph capture");
+    const tadm_status st = generate_loop(h, prompt, batch, prompt_len, out, gen_len, steps_per_block, K, block_len,
+                                         h->gstream);
+    cudaGraph_t g = nullptr;
+    const cudaError_t ce = cudaStreamEndCapture(h->gstream, &g);
+    if (st != TADM_OK) {
+      if (g) cudaGraphDestroy(g);
+      return st;
+    }
+    if (ce != cudaSuccess || !g) return fail(h, TADM_ERR_CUDA, "end graph capture: %s", cudaGetErrorString(ce));
+    const cudaError_t ie = cudaGraphInstantiate(&h->gexec, g, 0);
+    cudaGraphDestroy(g);
+    if (ie != cudaSuccess) {
+      h->gexec = nullptr;
+      return fail(h, TADM_ERR_CUDA, "graph instantiate: %s", cudaGetErrorString(ie));
+    }
+    std::memcpy(h->gkey, key, sizeof(key));
+    h->gcounters = h->counters;
+    h->gctx = h->ctx;
+  }
+  // replay, ordered after the caller's stream and before its next work
+  h->counters = h->gcounters;
+  h->ctx = h->gctx;
+  h->counters.kernel_launches = h->gcounters.kernel_launches;
+  if (cudaEventRecord(h->gev_in, stream) != cudaSuccess || cudaStreamWaitEvent(h->gstream, h->gev_in, 0) != cudaSuccess ||
+      cudaGraphLaunch(h->gexec, h->gstream) != cudaSuccess || cudaEventRecord(h->gev_out, h->gstream) != cudaSuccess ||
+      cudaStreamWaitEvent(stream, h->gev_out, 0) != cudaSuccess)
+    return fail(h, TADM_ERR_CUDA, "graph launch");
+  return TADM_OK;
+}
+
+// The issue loop of tadm_generate (Alg. 1 per block, prefill and commits).
+tadm_status generate_loop(tadm_handle* h, const int32_t* prompt, int batch, int prompt_len, int32_t* out,
+                          int gen_len, int steps_per_block, int K, int block_len, cudaStream_t s) {
+  const int total = prompt_len + gen_len;
+  const int R = block_len > 0 ? block_len : total;
   const tadm_config& c = h->cfg;
   TRY(fill_canvas(out, total, prompt, batch, prompt_len, total, c.vocab - 1, s));
   void* cache = h->at(h->off.h_int);

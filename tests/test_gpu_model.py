@@ -221,6 +221,32 @@ def test_generate_k1_equals_step_loop_and_counts(T):
     assert tm.tadm_get_counters()["anchor_calls"] == 3
 
 
+@pytest.mark.parametrize("block_len", [0, 16])
+def test_generate_graph_replay_matches_eager(T, block_len):
+    """tadm_generate runs its first call with given sizes and buffers eagerly,
+    captures the second into a CUDA graph and replays it from the third on:
+    the tokens and counters of all three are identical."""
+    m = wl.ModelConfig(**SMALL_BF16)
+    P, G = 16, 48
+    w = wl.Workload("t", m, batch=2, prompt_len=P, gen_len=G, steps_per_block=8 if block_len else 12, K=2,
+                    block_len=block_len)
+    B = 2
+    tm, _ = setup(T, m, B, max(P, block_len) if block_len else P + G, max_ctx=P + G if block_len else 0)
+    p = torch.from_numpy(wl.make_prompts(w, batch=B, seed=4)).cuda()
+    out = torch.empty((B, P + G), dtype=torch.int32, device="cuda")
+    runs, counts = [], []
+    for _ in range(4):
+        out.fill_(-7)
+        tm.tadm_generate(p, out, G, w.steps_per_block, 2, block_len)
+        tm.tadm_sync_status()
+        runs.append(out.cpu().numpy())
+        counts.append(tm.tadm_get_counters())
+    for r, c in zip(runs[1:], counts[1:]):
+        assert np.array_equal(r, runs[0])
+        assert c == counts[0]
+    assert np.all(runs[0] != m.mask_id) and np.array_equal(runs[0][:, :P], p.cpu().numpy())
+
+
 def test_carry_over_and_zero_masking_on_gpu(T):
     m = wl.ModelConfig(**SMALL_BF16)
     w = wl.Workload("t", m, batch=2, prompt_len=16, gen_len=48, steps_per_block=6, K=2)
