@@ -20,6 +20,9 @@ What it computes (paper section / equation it follows):
   transformer-layer cost: Eq. (anchor-cache-compute).
 * Masked-diffusion reverse step with zero-masking and carry-over unmasking:
   App. B.1.1, Eq. (mdlm-posterior-unk).
+* ReMDM remasking sampler (the paper's Pretraining sampler, NEXT row):
+  §5 Eq. (inf-post-TADM), App. B Eqs. (remdm-posterior, remdm-param), with
+  the linear schedule, nucleus p and Cap / Loop settings of App. C.2.
 * Block diffusion with a KV cache over committed blocks (the encoder prefills
   the context causally, the decoder denoises the active block
   bidirectionally): App. C.1, "Architecture Details".
@@ -178,6 +181,83 @@ def select_topk(z: np.ndarray, conf: np.ndarray, k: int, mask_id: int) -> np.nda
         return np.zeros(0, dtype=np.int64)
     order = np.lexsort((cand, -conf[cand]))  # primary: conf desc, secondary: position asc
     return cand[order[:k]]
+
+
+# ---------------------------------------------------------------------------
+# ReMDM remasking sampler (§5 Eq. inf-post-TADM; App. B Eqs. remdm-posterior,
+# remdm-param; sampler settings of App. C.2 "Sampler Details")
+# ---------------------------------------------------------------------------
+def remdm_alpha(t: float, kind: str, t_on: float, t_off: float, alpha_on: float) -> float:
+    """alpha_t of the reverse schedule.  "cap": the linear schedule, 1 - t.
+    "loop": alpha rises linearly from 0 at t = 1 to alpha_on at t_on, stays
+    at alpha_on down to t_off, then rises linearly to 1 at t = 0."""
+    if kind == "cap":
+        return 1.0 - t
+    if t > t_on:
+        return alpha_on * (1.0 - t) / (1.0 - t_on)
+    if t >= t_off:
+        return alpha_on
+    return alpha_on + (1.0 - alpha_on) * (t_off - t) / t_off
+
+
+def remdm_schedule(n: int, T: int, kind: str, eta: float, t_on: float = 0.55, t_off: float = 0.05,
+                   alpha_on: float = 0.9):
+    """(alpha_t, alpha_s, sigma_t, p_unmask) of reverse step n = 0..T-1 from
+    t = (T - n) / T to s = (T - n - 1) / T.  sigma_t is capped by
+    sigma_max = min(1, (1 - alpha_s) / alpha_t), the largest value that keeps
+    the posterior a distribution; "cap" uses min(eta, sigma_max) at every
+    step, "loop" uses it only inside the loop phase (alpha_t = alpha_s =
+    alpha_on) and 0 elsewhere.  p_unmask = (alpha_s - (1 - sigma) alpha_t) /
+    (1 - alpha_t) is the probability that a masked position takes a token."""
+    t = (T - n) / T
+    s = (T - n - 1) / T
+    a_t = remdm_alpha(t, kind, t_on, t_off, alpha_on)
+    a_s = remdm_alpha(s, kind, t_on, t_off, alpha_on)
+    sigma_max = min(1.0, (1.0 - a_s) / a_t) if a_t > 0.0 else 1.0
+    if kind == "cap" or (t <= t_on and s >= t_off):
+        sigma = min(eta, sigma_max)
+    else:
+        sigma = 0.0
+    p_unmask = (a_s - (1.0 - sigma) * a_t) / (1.0 - a_t)
+    return a_t, a_s, sigma, p_unmask
+
+
+def nucleus_sample(logits: np.ndarray, mask_id: int, top_p: float, u: float) -> int:
+    """One token of the nucleus (top-p) distribution of softmax(logits) over
+    ids != MASK.  Nucleus N = {v : q_v >= tau}, tau the largest probability
+    value such that the tokens at or above it hold >= top_p of the mass
+    (tokens tied at tau are all kept).  The token is the first v of N in id
+    order whose cumulative mass within N exceeds u * mass(N)."""
+    l = np.asarray(logits, dtype=np.float64).copy()
+    l[mask_id] = -np.inf
+    q = np.exp(l - np.max(l))
+    desc = np.sort(q)[::-1]
+    k = int(np.searchsorted(np.cumsum(desc), top_p * q.sum(), side="left"))
+    tau = desc[min(k, desc.size - 1)]
+    qn = np.where(q >= tau, q, 0.0)
+    c = np.cumsum(qn)
+    return int(np.nonzero(c > u * c[-1])[0][0])
+
+
+def remdm_step(z: np.ndarray, logits: np.ndarray, first_gen: int, sigma: float, p_unmask: float, top_p: float,
+               u: np.ndarray, mask_id: int):
+    """One reverse step of one sequence (Eq. inf-post-TADM).  z: [R] canvas,
+    logits: [R, V], u: [R, 3] uniforms (remask, unmask, token).  Positions
+    before first_gen (the prompt) never change; a generated token is remasked
+    with probability sigma; a masked position unmasks with probability
+    p_unmask to a nucleus sample of its logits.  Returns (z_s, action) with
+    action 0 keep, 1 remask, 2 unmask."""
+    out = z.copy()
+    act = np.zeros(z.shape[0], dtype=np.int32)
+    for r in range(first_gen, z.shape[0]):
+        if z[r] != mask_id:
+            if u[r, 0] < sigma:
+                out[r] = mask_id
+                act[r] = 1
+        elif u[r, 1] < p_unmask:
+            out[r] = nucleus_sample(logits[r], mask_id, top_p, u[r, 2])
+            act[r] = 2
+    return out, act
 
 
 def layer_cost(L_S: int, L_A: int, L_D: int, T: int, K: int):
@@ -451,6 +531,33 @@ class Oracle:
             self.commit_block(sess, zb)
             blocks.append(zb)
         return np.concatenate([prompts.astype(np.int32)] + blocks, axis=1)
+
+    def generate_remdm(self, prompts: np.ndarray, gen_len: int, T: int, K: int, kind: str, eta: float,
+                       top_p: float, uniforms, t_on: float = 0.55, t_off: float = 0.05, alpha_on: float = 0.9,
+                       step_hook=None) -> np.ndarray:
+        """Alg. 1 with the ReMDM remasking sampler on one canvas (prompt +
+        gen_len masks, single block): refresh when n mod K = 0, logits from
+        the fused prediction, then remdm_step per sequence.  ``uniforms(n)``
+        returns the [B, P + gen_len, 3] draws of step n."""
+        B, P = prompts.shape
+        mask = self.mask_id
+        z = np.concatenate([prompts.astype(np.int32), np.full((B, gen_len), mask, np.int32)], axis=1)
+        sess = self.new_session(B)
+        cache = None
+        for n in range(T):
+            if n % K == 0:
+                cache = self.anchor_forward(sess, z)
+            logits = self.denoise_logits(sess, z, cache)
+            _, _, sigma, p_un = remdm_schedule(n, T, kind, eta, t_on, t_off, alpha_on)
+            u = uniforms(n)
+            new = np.empty_like(z)
+            for b in range(B):
+                new[b], _ = remdm_step(z[b], logits[b], P, sigma, p_un, top_p, u[b], mask)
+            if step_hook is not None:
+                step_hook(n, z, logits, new)
+            z = new
+            self.counters["steps"] += 1
+        return z
 
     def _run_block(self, sess, z, T, K, G, block_idx, step_hook):
         cache = None

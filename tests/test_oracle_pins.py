@@ -487,3 +487,146 @@ def test_fusion_off_ignores_the_current_canvas():
         l0 = o.denoise_logits(o.new_session(2), z0, cache)
         l1 = o.denoise_logits(o.new_session(2), z1, cache)
         assert np.array_equal(l0, l1) == same
+
+
+# --------------------------------------------------------------------- ReMDM sampler (NEXT row)
+def test_remdm_sigma_zero_is_masked_diffusion_posterior():
+    """sigma_t = 0 recovers the masked-diffusion posterior (App. B, after Eq.
+    remdm-posterior): with the linear schedule a masked position unmasks with
+    probability (alpha_s - alpha_t) / (1 - alpha_t) = 1 / (T - n), and no
+    token is ever remasked."""
+    T = 17
+    for n in range(T):
+        a_t, a_s, sigma, p_un = O.remdm_schedule(n, T, "cap", 0.0)
+        assert sigma == 0.0
+        assert abs(p_un - 1.0 / (T - n)) < 1e-14
+        assert abs(a_t - n / T) < 1e-15 and abs(a_s - (n + 1) / T) < 1e-15
+    z = np.array([5, 9, 63, 63, 2, 63], np.int32)
+    u = np.full((6, 3), 0.0)
+    out, act = O.remdm_step(z, rng.standard_normal((6, 64)), 1, 0.0, 0.0, 0.9, u, 63)
+    assert np.array_equal(out, z) and not act.any()
+
+
+@pytest.mark.parametrize("kind,eta,T", [("cap", 0.04, 128), ("cap", 0.5, 9), ("loop", 0.02, 1024), ("loop", 0.02, 64)])
+def test_remdm_posterior_is_a_distribution(kind, eta, T):
+    """For every step both cases of Eq. remdm-posterior are distributions
+    (sigma within [0, sigma_max]) and the last step unmasks everything."""
+    for n in range(T):
+        a_t, a_s, sigma, p_un = O.remdm_schedule(n, T, kind, eta)
+        stay = (1.0 - a_s - sigma * a_t) / (1.0 - a_t)
+        assert 0.0 <= sigma <= 1.0 and 0.0 <= a_t <= a_s <= 1.0
+        assert -1e-12 <= p_un <= 1.0 + 1e-12 and stay >= -1e-12
+        assert abs(p_un + stay - 1.0) < 1e-12
+    _, a_s, sigma, p_un = O.remdm_schedule(T - 1, T, kind, eta)
+    assert a_s == 1.0 and sigma == 0.0 and abs(p_un - 1.0) < 1e-12
+
+
+def test_remdm_loop_phase_holds_alpha_on():
+    """ReMDM-Loop: alpha is alpha_on throughout the loop phase, where sigma =
+    eta; there the expected masked fraction 1 - alpha_on is a fixed point of
+    one step (unmasking and remasking balance); no remasking outside it."""
+    T, eta, a_on = 400, 0.02, 0.9
+    inside = 0
+    for n in range(T):
+        t, s = (T - n) / T, (T - n - 1) / T
+        a_t, a_s, sigma, p_un = O.remdm_schedule(n, T, "loop", eta, 0.55, 0.05, a_on)
+        if t <= 0.55 and s >= 0.05:
+            inside += 1
+            assert a_t == a_s == a_on and sigma == eta
+            m = 1.0 - a_on
+            assert abs(m * (1.0 - p_un) + (1.0 - m) * sigma - m) < 1e-12
+        else:
+            assert sigma == 0.0
+    assert inside == round((0.55 - 0.05) * T)
+
+
+def test_nucleus_sample_brute_force():
+    """Inverse-CDF sampling within the nucleus: on a grid of u the token
+    frequencies are the renormalised nucleus probabilities, the nucleus is
+    the smallest set of most probable tokens reaching top_p (built here by a
+    sorted walk), and MASK is never drawn."""
+    logits = np.array([0.3, 2.0, -1.0, 1.2, 2.0, 0.9, 5.0, 1.5])   # id 7 is MASK (largest after 6)
+    mask, top_p = 6, 0.8
+    q = np.exp(logits - logits[np.arange(8) != mask].max())
+    q[mask] = 0.0
+    order = sorted(range(8), key=lambda v: -q[v])
+    keep, acc = [], 0.0
+    for v in order:
+        if acc >= top_p * q.sum() and q[v] < q[keep[-1]]:
+            break
+        keep.append(v)
+        acc += q[v]
+    want = np.zeros(8)
+    want[keep] = q[keep] / q[keep].sum()
+    grid = (np.arange(20000) + 0.5) / 20000
+    got = np.bincount([O.nucleus_sample(logits, mask, top_p, u) for u in grid], minlength=8) / grid.size
+    assert got[mask] == 0.0
+    np.testing.assert_allclose(got, want, atol=1e-4)
+
+
+def test_nucleus_top_p_one_is_plain_categorical():
+    lg = rng.standard_normal(50)
+    q = np.exp(lg - lg.max())
+    q[49] = 0.0
+    c = np.cumsum(q) / q.sum()
+    for u in rng.random(200):
+        assert O.nucleus_sample(lg, 49, 1.0, u) == int(np.searchsorted(c, u, side="right"))
+
+
+def test_remdm_step_rates_and_prompt():
+    """Monte Carlo over the shared Philox draws: generated tokens are
+    remasked at rate sigma, masked positions unmask at rate p_unmask, the
+    prompt never changes and unmasked tokens come from the nucleus."""
+    V, R, P, mask = 32, 4000, 100, 31
+    z = np.where(rng.random(R) < 0.5, mask, rng.integers(0, 31, R)).astype(np.int32)
+    lg = rng.standard_normal((R, V))
+    u = wl.remdm_uniforms(11, 3, 1, R)[0]
+    out, act = O.remdm_step(z, lg, P, 0.3, 0.6, 0.9, u, mask)
+    assert np.array_equal(out[:P], z[:P])
+    gen = np.arange(R) >= P
+    tok, msk = gen & (z != mask), gen & (z == mask)
+    r1, r2 = (act[tok] == 1).mean(), (act[msk] == 2).mean()
+    assert abs(r1 - 0.3) < 4 * np.sqrt(0.3 * 0.7 / tok.sum()) and abs(r2 - 0.6) < 4 * np.sqrt(0.24 / msk.sum())
+    assert np.all(out[act == 2] != mask) and np.all(out[act == 1] == mask)
+
+
+def test_remdm_uniforms_follow_philox():
+    """The sampler's draws: block (n * B + b) * R + r of the REMD stream,
+    uniform j = (word j >> 8) * 2^-24."""
+    u = wl.remdm_uniforms(77, 5, 3, 11)
+    for b, r in ((0, 0), (2, 10), (1, 4)):
+        blk = (5 * 3 + b) * 11 + r
+        w = wl.philox4x32_10([blk & 0xFFFFFFFF, blk >> 32, wl.REMDM_STREAM, 0], [77, 0])
+        assert list(u[b, r]) == [(w[j] >> 8) / 16777216.0 for j in range(3)]
+
+
+def test_remdm_uniform_roles_and_edges():
+    """u[:, 0] alone decides remasking, u[:, 1] alone unmasking, u[:, 2] the
+    token; u = 0 draws the first nucleus token in id order (never a token of
+    zero nucleus mass)."""
+    mask = 9
+    z = np.array([1, 2, mask, mask], np.int32)
+    lg = np.zeros((4, 10))
+    lg[:, 7] = 6.0                      # token 7 alone holds 0.98 > 0.9 of the mass
+    u = np.array([[0.0, 0.99, 0.5], [0.99, 0.0, 0.5], [0.0, 0.99, 0.5], [0.99, 0.0, 0.0]])
+    out, act = O.remdm_step(z, lg, 0, 0.5, 0.5, 0.9, u, mask)
+    assert list(act) == [1, 0, 0, 2] and list(out) == [mask, 2, mask, 7]
+    assert O.nucleus_sample(lg[0], mask, 0.9, 0.0) == 7
+
+
+def test_remdm_loop_alpha_is_continuous():
+    """The Loop time warp is continuous: alpha(1) = 0, alpha(t_on) = alpha_on
+    from both sides, alpha(t_off) = alpha_on, alpha(0) = 1."""
+    f = lambda t: O.remdm_alpha(t, "loop", 0.55, 0.05, 0.9)  # noqa: E731
+    assert f(1.0) == 0.0 and f(0.0) == 1.0
+    for t in (0.55, 0.05):
+        assert abs(f(t + 1e-9) - 0.9) < 1e-7 and abs(f(t - 1e-9) - 0.9) < 1e-7
+
+
+def test_remdm_token_uses_its_own_uniform():
+    """The token of an unmasking position is drawn with u[:, 2]: two equally
+    likely tokens 3 and 7, u[:, 1] = 0.1 (unmask) and u[:, 2] = 0.9 give 7."""
+    lg = np.full((1, 10), -30.0)
+    lg[0, 3] = lg[0, 7] = 0.0
+    out, act = O.remdm_step(np.array([9], np.int32), lg, 0, 0.0, 0.5, 0.9, np.array([[0.99, 0.1, 0.9]]), 9)
+    assert act[0] == 2 and out[0] == 7

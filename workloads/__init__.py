@@ -36,6 +36,7 @@ _LIB = None
 _LIB_LOCK = threading.Lock()
 
 PROMPT_STREAM = 0x50524F4D  # stream id of prompt draws ("PROM")
+REMDM_STREAM = 0x52454D44   # stream id of the ReMDM sampler's draws ("REMD")
 
 
 # --------------------------------------------------------------------------
@@ -60,6 +61,7 @@ def _lib():
             u64, u32, i64 = ctypes.c_uint64, ctypes.c_uint32, ctypes.c_int64
             lib.wl_philox4x32_10.argtypes = [ctypes.POINTER(u32), ctypes.POINTER(u32), ctypes.POINTER(u32)]
             lib.wl_philox_u32.argtypes = [u64, u32, i64, ctypes.c_void_p]
+            lib.wl_philox_blocks.argtypes = [u64, u32, u64, i64, ctypes.c_void_p]
             lib.wl_normal_f32.argtypes = [u64, u32, i64, ctypes.c_double, ctypes.c_double, ctypes.c_void_p]
             lib.wl_normal_bf16.argtypes = [u64, u32, i64, ctypes.c_double, ctypes.c_double, ctypes.c_void_p]
             _LIB = lib
@@ -80,6 +82,24 @@ def philox_u32(seed: int, stream: int, n: int) -> np.ndarray:
     if n:
         _lib().wl_philox_u32(seed, stream, n, out.ctypes.data)
     return out
+
+
+def philox_blocks(seed: int, stream: int, first_block: int, n_blocks: int) -> np.ndarray:
+    """uint32 [n_blocks, 4]: the words of Philox blocks first_block .. (counter =
+    (block lo, block hi, stream, 0), key = (seed lo, seed hi))."""
+    out = np.empty((n_blocks, 4), dtype=np.uint32)
+    if n_blocks:
+        _lib().wl_philox_blocks(seed, stream, first_block, n_blocks, out.ctypes.data)
+    return out
+
+
+def remdm_uniforms(seed: int, step: int, batch: int, rows: int) -> np.ndarray:
+    """float64 [batch, rows, 3]: the ReMDM sampler's three uniforms in [0, 1)
+    for every canvas position of reverse step ``step`` (remask, unmask, token).
+    Position (b, r) of step n uses Philox block (n * batch + b) * rows + r of
+    REMDM_STREAM; uniform j = (word j >> 8) * 2^-24."""
+    w = philox_blocks(seed, REMDM_STREAM, (step * batch) * rows, batch * rows)
+    return ((w[:, :3] >> 8).astype(np.float64) * (1.0 / 16777216.0)).reshape(batch, rows, 3)
 
 
 def normal(seed: int, stream: int, n: int, mean: float, std: float, dtype: str) -> np.ndarray:

@@ -56,6 +56,12 @@ void wl_philox_u32(uint64_t seed, uint32_t stream, int64_t n, uint32_t* out) {
   }
 }
 
+/* Words of the blocks first_blk .. first_blk + n_blk - 1: out[4 * j + w] = word w of block first_blk + j. */
+void wl_philox_blocks(uint64_t seed, uint32_t stream, uint64_t first_blk, int64_t n_blk, uint32_t* out) {
+#pragma omp parallel for schedule(static)
+  for (int64_t j = 0; j < n_blk; ++j) block_words(seed, stream, first_blk + (uint64_t)j, out + 4 * j);
+}
+
 /* Box-Muller on one Philox block: 4 standard normals. */
 static void block_normals(uint64_t seed, uint32_t stream, uint64_t blk, double z[4]) {
   uint32_t w[4];
