@@ -46,6 +46,8 @@ def parse():
                     help="override reverse steps per block (short runs for launch-list profiles)")
     ap.add_argument("--G", type=int, default=None, help="override the generation length (short profiling runs)")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
+    ap.add_argument("--sampler", default="topk", choices=["topk", "remdm-cap", "remdm-loop"],
+                    help="with --sweep-workloads: the confidence top-k sampler or ReMDM (App. C.2 settings)")
     ap.add_argument("--fusion-off", action="store_true",
                     help="with --sweep-workloads: run the workloads with the fusion disabled (App. D naive reuse)")
     ap.add_argument("--sweep-workloads", default=None,
@@ -429,15 +431,28 @@ def workload_sweep(args):
             p = torch.from_numpy(wl.make_prompts(w)).cuda()
             out = torch.empty((B, w.total_len), dtype=torch.int32, device="cuda")
             res = {}
+            remdm = args.sampler.startswith("remdm")
+            if remdm:   # ReMDM sampler (App. C.2 settings): logits of the masked rows per step
+                if bl:
+                    raise SystemExit("the ReMDM sampler runs single-block workloads")
+                scratch = torch.empty((B * w.gen_len, m.vocab), dtype=torch.float32, device="cuda")
+                kind = args.sampler.split("-")[1]
+                eta = 0.04 if kind == "cap" else 0.02
+
+            def gen(K):
+                if remdm:
+                    tm.tadm_generate_remdm(p, out, w.gen_len, w.steps_per_block, K, kind, eta, 0.9, 1234, scratch)
+                else:
+                    tm.tadm_generate(p, out, w.gen_len, w.steps_per_block, K, bl)
             for K in (w.k_sweep or (w.K,)):
                 for _ in range(max(2, args.warmup)):   # the second identical call captures the CUDA graph
-                    tm.tadm_generate(p, out, w.gen_len, w.steps_per_block, K, bl)
+                    gen(K)
                 tm.tadm_sync_status()
                 e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
                 torch.cuda.synchronize()
                 e0.record()
                 for _ in range(args.steps):
-                    tm.tadm_generate(p, out, w.gen_len, w.steps_per_block, K, bl)
+                    gen(K)
                 e1.record()
                 tm.tadm_sync_status()
                 ms = e0.elapsed_time(e1) / args.steps
@@ -445,12 +460,15 @@ def workload_sweep(args):
                 res[K] = B * w.gen_len / (ms / 1000.0)
                 # one more generation with every GEMM launch bracketed by events (up to 400000 launches)
                 tm.tadm_probe_enable(400000)
-                tm.tadm_generate(p, out, w.gen_len, w.steps_per_block, K, bl)
+                gen(K)
                 n_l, g_ms, g_fl = tm.tadm_probe_read()
                 tm.tadm_probe_enable(0)
                 tm.tadm_sync_status()
                 g_tf = g_fl / (g_ms / 1000.0) / 1e12 if g_ms > 0 else None
-                print(json.dumps({"workload": name, "fusion": m.fusion, "batch": B, "K": K, "tokens_per_s": res[K],
+                done = out.cpu().numpy()
+                valid = bool((done != m.mask_id).all())
+                print(json.dumps({"workload": name, "fusion": m.fusion, "sampler": args.sampler, "all_unmasked": valid,
+                                  "batch": B, "K": K, "tokens_per_s": res[K],
                                   "ms_per_generation": ms,
                                   "vs_K1": res[K] / res[1] if 1 in res else None, "anchor_calls": c["anchor_calls"],
                                   "denoise_steps": c["denoise_steps"], "commit_passes": c["commit_passes"],

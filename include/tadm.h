@@ -315,6 +315,63 @@ TADM_API tadm_status tadm_attention(const void* q, const void* k, const void* v,
                            int n_heads, int n_kv_heads, int head_dim, int rows, int ctx,
                            int kv_stride, int causal, int dtype, tadm_stream stream);
 
+/* ------------------------------------------------------------ ReMDM sampler --
+ * The paper's Pretraining sampler in place of the confidence top-k: the
+ * remasking reverse step of §5 Eq. (inf-post-TADM) (App. B Eqs.
+ * remdm-posterior, remdm-param) with the fused prediction, nucleus (top-p)
+ * sampling and the ReMDM-Cap / ReMDM-Loop schedules of App. C.2.  Readings
+ * where the paper defers to ReMDM without restating it:
+ *  - kind 0 (Cap): alpha_t = 1 - t on t = (T - n) / T; sigma_t = min(eta,
+ *    sigma_max), sigma_max = min(1, (1 - alpha_s) / alpha_t);
+ *  - kind 1 (Loop): alpha rises linearly to alpha_on at t_on, stays there
+ *    to t_off, then rises to 1; sigma_t = min(eta, sigma_max) while alpha_t =
+ *    alpha_s = alpha_on, else 0;
+ *  - a generated token is remasked if u0 < sigma_t; a masked position takes a
+ *    token if u1 < p_unmask = (alpha_s - (1 - sigma_t) alpha_t) / (1 - alpha_t);
+ *    prompt positions never change;
+ *  - the token: nucleus N = {v != MASK : q_v >= tau}, tau the largest value
+ *    whose tokens hold >= top_p of the mass (ties kept); the first v of N in
+ *    id order whose cumulative mass in N exceeds u2 * mass(N);
+ *  - draws: Philox4x32-10 (Salmon et al., SC'11), counter (block lo, block
+ *    hi, 0x52454D44, 0), key (seed lo, seed hi), block (step * batch + b) *
+ *    rows + r for canvas position (b, r); u_j = (word j >> 8) * 2^-24. */
+
+/* Host only: out = {alpha_t, alpha_s, sigma_t, p_unmask} of reverse step n
+ * (0 .. T-1) of schedule `kind` (0 Cap, 1 Loop; t_on, t_off, alpha_on are
+ * read by Loop only).  INVALID_ARG for T < 1, n outside 0..T-1, eta < 0, or
+ * a Loop with 0 < t_off < t_on < 1 and 0 < alpha_on < 1 violated. */
+TADM_API tadm_status tadm_remdm_schedule(int kind, int T, int n, double eta, double t_on, double t_off,
+                                         double alpha_on, double out[4]);
+
+/* The three draws of every canvas position at reverse step `step`:
+ * out (device float [batch * rows * 3]) = (u0, u1, u2) per position in
+ * row-major (b, r) order. */
+TADM_API tadm_status tadm_remdm_uniforms(uint64_t seed, int step, int batch, int rows, float* out,
+                                         tadm_stream stream);
+
+/* One ReMDM reverse step on a canvas, from given logits.  z: device int32
+ * [batch, rows] (leading dimension ldz), updated in place; logits: device
+ * fp32 [batch * rows, vocab] (row stride ld_logits), row b * rows + r for
+ * position (b, r), read only; positions < first_gen never change; sigma and
+ * p_unmask as from tadm_remdm_schedule; action: device int32 [batch * rows],
+ * written with 0 keep, 1 remask, 2 unmask.  No allocation. */
+TADM_API tadm_status tadm_remdm_update(int32_t* z, int ldz, const float* logits, int ld_logits, int batch, int rows,
+                                       int first_gen, int vocab, int mask_id, double sigma, double p_unmask,
+                                       float top_p, uint64_t seed, int step, int32_t* action, tadm_stream stream);
+
+/* Whole generation with the ReMDM sampler (single block: prompt + gen_len
+ * masks): Alg. 1's refresh when n mod K == 0, the fused prediction every
+ * step, then the ReMDM step of schedule `kind` (eta; Loop with t_on 0.55,
+ * t_off 0.05, alpha_on 0.9 as in App. C.2).  logits_scratch: caller device
+ * fp32 buffer of at least batch * gen_len * vocab * 4 bytes (the logits of
+ * the masked rows of a step).  Positions still masked after the last step
+ * cannot occur: the last step unmasks every masked position.  The handle
+ * needs max_rows >= prompt_len + gen_len and no KV context. */
+TADM_API tadm_status tadm_generate_remdm(tadm_handle* h, const int32_t* prompt, int batch, int prompt_len,
+                                         int32_t* out, int gen_len, int steps, int K, int kind, double eta,
+                                         float top_p, uint64_t seed, float* logits_scratch, size_t scratch_bytes,
+                                         tadm_stream stream);
+
 #ifdef __cplusplus
 }
 #endif

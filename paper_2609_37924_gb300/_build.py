@@ -11,7 +11,8 @@ LIBDIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(LIBDIR, "libtadm.so")
 SOURCES = ["gemm_tc.cu", "gemm_simt.cu", "attention.cu", "rowops.cu", "sampler.cu", "tadm_api.cu", "head_static.cu", "splitk.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden"]
+FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
+         "-Xcompiler", "-ffp-contract=off"]   # host fp64 arithmetic exactly as written (no fused multiply-add)
 
 
 def _nvcc() -> str:

@@ -95,6 +95,13 @@ const char* confidence_rows(const float* logits, int rows, int vocab, int ld, in
                             int32_t* tok, cudaStream_t s);
 const char* combine_partials(const float* part, int rows, int n_tiles, float* conf, int32_t* tok,
                              cudaStream_t s, const int32_t* rows_idx = nullptr);
+// ReMDM sampler: the draws of a step; decide (and apply remasks); nucleus tokens of the unmasking rows
+const char* remdm_uniforms(uint64_t seed, int step, int B, int R, float* out, cudaStream_t s);
+const char* remdm_decide(int32_t* z, int ldz, int B, int R, int first_gen, int mask_id, double sigma,
+                         double p_unmask, uint64_t seed, int step, int32_t* act, cudaStream_t s);
+const char* remdm_sample(const float* logits, int ld, int n_rows, const int32_t* idx, const int32_t* act, int32_t* z,
+                         int ldz, int B, int R, int vocab, int mask_id, float top_p, uint64_t seed, int step,
+                         cudaStream_t s);
 const char* topk_unmask(int32_t* z, int ldz, const float* conf, const int32_t* tok, int batch, int rows, int k,
                         int mask_id, int32_t* selected, cudaStream_t s);
 

@@ -181,6 +181,191 @@ inline const char* err() {
   cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
 }
+// ------------------------------------------------------------ ReMDM sampler
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11): ten rounds of two
+// 32x32 -> 64-bit multiplies with the published multipliers and Weyl key
+// increments.
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint2 k) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    const uint32_t lo0 = 0xD2511F53u * c.x, hi0 = __umulhi(0xD2511F53u, c.x);
+    const uint32_t lo1 = 0xCD9E8D57u * c.z, hi1 = __umulhi(0xCD9E8D57u, c.z);
+    c = make_uint4(hi1 ^ c.y ^ k.x, lo1, hi0 ^ c.w ^ k.y, lo0);
+    k.x += 0x9E3779B9u;
+    k.y += 0xBB67AE85u;
+  }
+  return c;
+}
+
+constexpr uint32_t kRemdmStream = 0x52454D44u;   // "REMD"
+
+// The three draws of canvas position (b, r) at reverse step n: Philox block
+// (n * B + b) * R + r of the REMD stream, uniform j = (word j >> 8) * 2^-24.
+__device__ __forceinline__ void remdm_draws(uint64_t seed, int step, int B, int R, int b, int r, float (&u)[3]) {
+  const uint64_t blk = (static_cast<uint64_t>(step) * B + b) * static_cast<uint64_t>(R) + r;
+  const uint4 w = philox4x32_10(make_uint4(static_cast<uint32_t>(blk), static_cast<uint32_t>(blk >> 32), kRemdmStream, 0u),
+                                make_uint2(static_cast<uint32_t>(seed), static_cast<uint32_t>(seed >> 32)));
+  u[0] = static_cast<float>(w.x >> 8) * (1.0f / 16777216.0f);
+  u[1] = static_cast<float>(w.y >> 8) * (1.0f / 16777216.0f);
+  u[2] = static_cast<float>(w.z >> 8) * (1.0f / 16777216.0f);
+}
+
+__global__ void remdm_uniforms_kernel(uint64_t seed, int step, int B, int R, float* __restrict__ out) {
+  pdl_enter();
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= B * R) return;
+  float u[3];
+  remdm_draws(seed, step, B, R, i / R, i % R, u);
+  out[3 * i] = u[0];
+  out[3 * i + 1] = u[1];
+  out[3 * i + 2] = u[2];
+}
+
+// One thread per canvas position of the active rows: action 0 keep, 1 remask
+// (a generated token, u0 < sigma: written as MASK here), 2 unmask (a masked
+// position, u1 < p_unmask: its token is drawn by remdm_sample_kernel).  The
+// comparisons are in fp64, exactly as the oracle takes them.
+__global__ void remdm_decide_kernel(int32_t* __restrict__ z, int ldz, int B, int R, int first_gen, int mask_id,
+                                    double sigma, double p_unmask, uint64_t seed, int step, int32_t* __restrict__ act) {
+  pdl_enter();
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= B * R) return;
+  const int b = i / R, r = i - (i / R) * R;
+  int a = 0;
+  if (r >= first_gen) {
+    float u[3];
+    remdm_draws(seed, step, B, R, b, r, u);
+    int32_t* zp = z + static_cast<size_t>(b) * ldz + r;
+    if (*zp != mask_id) {
+      if (static_cast<double>(u[0]) < sigma) {
+        a = 1;
+        *zp = mask_id;
+      }
+    } else if (static_cast<double>(u[1]) < p_unmask) {
+      a = 2;
+    }
+  }
+  act[i] = a;
+}
+
+template <int NT>
+__device__ __forceinline__ float block_sum_f(float v, float* red) {
+  v = warp_sum(v);
+  __syncthreads();
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+  __syncthreads();
+  float t = 0.0f;
+#pragma unroll
+  for (int w = 0; w < NT / 32; ++w) t += red[w];
+  return t;
+}
+
+// One block per logits row j (canvas row idx[j], or j): for rows whose action
+// is 2, the nucleus (top-p) token of softmax over ids != MASK, by inverse CDF
+// in id order within the nucleus.  The nucleus threshold is the largest fp32
+// tau with sum_{q_v >= tau} q_v >= top_p * sum q (q = exp(l - max)), found by
+// bisection on the bit patterns of tau in [0, 1]; each thread owns a
+// contiguous id range, so the id-order prefix sum is a block scan of range
+// sums followed by one thread's walk of its range.
+template <int NT>
+__global__ void __launch_bounds__(NT) remdm_sample_kernel(const float* __restrict__ logits, int ld, int n_rows,
+                                                          const int32_t* __restrict__ idx, const int32_t* __restrict__ act,
+                                                          int32_t* __restrict__ z, int ldz, int B, int R, int vocab,
+                                                          int mask_id, float top_p, uint64_t seed, int step) {
+  pdl_enter();
+  __shared__ float red[NT / 32];
+  __shared__ float scan[NT];
+  __shared__ int pick;
+  const int j = blockIdx.x;
+  if (j >= n_rows) return;
+  const int row = idx ? idx[j] : j;
+  if (act[row] != 2) return;                     // uniform across the block
+  const int b = row / R, r = row - (row / R) * R;
+  const float* L = logits + static_cast<size_t>(j) * ld;
+  const int tid = threadIdx.x;
+  const int chunk = (vocab + NT - 1) / NT, v0 = tid * chunk, v1 = min(vocab, v0 + chunk);
+  float mx = -INFINITY;
+  for (int v = v0; v < v1; ++v)
+    if (v != mask_id) mx = fmaxf(mx, L[v]);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  __syncthreads();
+  if ((tid & 31) == 0) red[tid >> 5] = mx;
+  __syncthreads();
+  mx = red[0];
+#pragma unroll
+  for (int w = 1; w < NT / 32; ++w) mx = fmaxf(mx, red[w]);
+  // mass at or above tau (tau = 0: the whole mass)
+  auto mass_from = [&](float tau) {
+    float acc = 0.0f;
+    for (int v = v0; v < v1; ++v) {
+      const float q = v == mask_id ? 0.0f : expf(L[v] - mx);
+      acc += q >= tau && q > 0.0f ? q : 0.0f;
+    }
+    return block_sum_f<NT>(acc, red);
+  };
+  const float total = mass_from(0.0f);
+  const float target = top_p * total;
+  uint32_t lo = 0u, hi = 0x3F800001u;            // mass_from(lo) >= target > mass_from(hi)
+  while (hi - lo > 1u) {
+    const uint32_t mid = lo + (hi - lo) / 2u;
+    if (mass_from(__uint_as_float(mid)) >= target) lo = mid;
+    else hi = mid;
+  }
+  const float tau = __uint_as_float(lo);
+  // id-order inverse CDF within the nucleus
+  float mine = 0.0f;
+  for (int v = v0; v < v1; ++v) {
+    const float q = v == mask_id ? 0.0f : expf(L[v] - mx);
+    mine += q >= tau && q > 0.0f ? q : 0.0f;
+  }
+  scan[tid] = mine;
+  if (tid == 0) pick = -1;
+  __syncthreads();
+  for (int o = 1; o < NT; o <<= 1) {             // inclusive scan of the range sums (fixed order)
+    const float add = tid >= o ? scan[tid - o] : 0.0f;
+    __syncthreads();
+    scan[tid] += add;
+    __syncthreads();
+  }
+  float u[3];
+  remdm_draws(seed, step, B, R, b, r, u);
+  const float zn = scan[NT - 1];
+  const float goal = u[2] * zn;
+  const float before = tid > 0 ? scan[tid - 1] : 0.0f;
+  if (mine > 0.0f && before <= goal && goal < scan[tid]) {
+    // the walk re-adds this range in the same order; if rounding keeps it
+    // at or below the goal, the range's last nucleus token is the draw
+    float c = before;
+    int last = -1, got = -1;
+    for (int v = v0; v < v1; ++v) {
+      const float q = v == mask_id ? 0.0f : expf(L[v] - mx);
+      if (q >= tau && q > 0.0f) {
+        last = v;
+        c += q;
+        if (c > goal) {
+          got = v;
+          break;
+        }
+      }
+    }
+    pick = got >= 0 ? got : last;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    int v = pick;
+    if (v < 0) {                                  // rounding left the goal past the last range: its last token
+      for (int t = NT - 1; t >= 0 && v < 0; --t)
+        if ((t > 0 ? scan[t] - scan[t - 1] : scan[0]) > 0.0f) {
+          const int a0 = t * chunk, a1 = min(vocab, a0 + chunk);
+          for (int w = a1 - 1; w >= a0; --w)
+            if (w != mask_id && expf(L[w] - mx) >= tau && expf(L[w] - mx) > 0.0f) { v = w; break; }
+        }
+    }
+    z[static_cast<size_t>(b) * ldz + r] = v;
+  }
+}
+
 }  // namespace
 
 const char* confidence_rows(const float* logits, int rows, int vocab, int ld, int mask_id, float* conf, int32_t* tok,
@@ -208,6 +393,29 @@ const char* topk_unmask(int32_t* z, int ldz, const float* conf, const int32_t* t
                         int mask_id, int32_t* selected, cudaStream_t s) {
   if (batch <= 0 || rows <= 0 || k <= 0) return nullptr;
   launch_pdl(topk_kernel, batch, 256, 0, s, z, ldz, conf, tok, rows, k, mask_id, selected);
+  return err();
+}
+
+const char* remdm_uniforms(uint64_t seed, int step, int B, int R, float* out, cudaStream_t s) {
+  if (B * R <= 0) return nullptr;
+  launch_pdl(remdm_uniforms_kernel, (B * R + 255) / 256, 256, 0, s, seed, step, B, R, out);
+  return err();
+}
+
+const char* remdm_decide(int32_t* z, int ldz, int B, int R, int first_gen, int mask_id, double sigma,
+                         double p_unmask, uint64_t seed, int step, int32_t* act, cudaStream_t s) {
+  if (B * R <= 0) return nullptr;
+  launch_pdl(remdm_decide_kernel, (B * R + 255) / 256, 256, 0, s, z, ldz, B, R, first_gen, mask_id, sigma, p_unmask,
+             seed, step, act);
+  return err();
+}
+
+const char* remdm_sample(const float* logits, int ld, int n_rows, const int32_t* idx, const int32_t* act, int32_t* z,
+                         int ldz, int B, int R, int vocab, int mask_id, float top_p, uint64_t seed, int step,
+                         cudaStream_t s) {
+  if (n_rows <= 0) return nullptr;
+  launch_pdl(remdm_sample_kernel<256>, n_rows, 256, 0, s, logits, ld, n_rows, idx, act, z, ldz, B, R, vocab, mask_id,
+             top_p, seed, step);
   return err();
 }
 

@@ -5,6 +5,7 @@
 // device memory; the caller binds one workspace that is carved into the
 // activation buffers, the per-layer KV caches of block mode, the internal
 // anchor cache of tadm_generate, the RoPE table and the status word.
+#include <algorithm>
 #include <cstdarg>
 #include <cstdio>
 #include <cstdlib>
@@ -551,15 +552,18 @@ tadm_status run_fusion(tadm_handle* h, int B, int R, const void* cache, cudaStre
 // MASK go through the head: the sampler reads nothing else (carry-over), so
 // the result is the same; they are gathered by the final RMSNorm and their
 // (conf, tok) scattered back, the other rows get conf = -inf.
+// With masked_per_seq > 0 the head runs only on the rows that hold MASK
+// (masked_per_seq list entries per sequence, in h->off.idx); logits, if
+// written, then follow the list order when compact_logits is set.
 tadm_status run_D_head(tadm_handle* h, int B, int R, float* logits, cudaStream_t s, const int32_t* z = nullptr,
-                       int ldz = 0, int masked_per_seq = 0) {
+                       int ldz = 0, int masked_per_seq = 0, bool compact_logits = false) {
   const tadm_config& c = h->cfg;
   const int M = B * R, d = c.d_model;
   const int64_t Mmax = static_cast<int64_t>(h->max_batch) * h->max_rows;
   float* x = h->at<float>(h->off.x);
   TRYS(stack_fwd(h, c.n_shared + c.n_anchor, c.n_denoise, x, B, R, h->ctx, 0, s));
   void* norm = h->at(h->off.norm);
-  const bool compact = masked_per_seq > 0 && !logits && z;
+  const bool compact = masked_per_seq > 0 && z && (!logits || compact_logits);
   const int Mh = compact ? B * masked_per_seq : M;
   const int32_t* idx = compact ? h->at<int32_t>(h->off.idx) : nullptr;
   if (compact)
@@ -665,6 +669,34 @@ const char* plan_args_error(int P, int G, int T, int K, int bl) {
 }  // namespace
 
 // =========================================================================== C ABI
+// ReMDM schedule (the readings stated in tadm.h): {alpha_t, alpha_s, sigma, p_unmask} of step n.
+double remdm_alpha(double t, int kind, double t_on, double t_off, double alpha_on) {
+  if (kind == 0) return 1.0 - t;
+  if (t > t_on) return alpha_on * (1.0 - t) / (1.0 - t_on);
+  if (t >= t_off) return alpha_on;
+  return alpha_on + (1.0 - alpha_on) * (t_off - t) / t_off;
+}
+void remdm_step_constants(int kind, int T, int n, double eta, double t_on, double t_off, double alpha_on,
+                          double out[4]) {
+  const double t = static_cast<double>(T - n) / T, s = static_cast<double>(T - n - 1) / T;
+  const double a_t = remdm_alpha(t, kind, t_on, t_off, alpha_on), a_s = remdm_alpha(s, kind, t_on, t_off, alpha_on);
+  double sigma_max = 1.0;
+  if (a_t > 0.0) sigma_max = std::min(1.0, (1.0 - a_s) / a_t);
+  const bool remask = kind == 0 || (t <= t_on && s >= t_off);
+  const double sigma = remask ? std::min(eta, sigma_max) : 0.0;
+  out[0] = a_t;
+  out[1] = a_s;
+  out[2] = sigma;
+  out[3] = (a_s - (1.0 - sigma) * a_t) / (1.0 - a_t);
+}
+const char* remdm_args_error(int kind, double eta, double t_on, double t_off, double alpha_on) {
+  if (kind != 0 && kind != 1) return "kind must be 0 (Cap) or 1 (Loop)";
+  if (!(eta >= 0.0)) return "eta must be >= 0";
+  if (kind == 1 && !(0.0 < t_off && t_off < t_on && t_on < 1.0 && 0.0 < alpha_on && alpha_on < 1.0))
+    return "Loop needs 0 < t_off < t_on < 1 and 0 < alpha_on < 1";
+  return nullptr;
+}
+
 extern "C" {
 
 const char* tadm_status_string(tadm_status s) {
@@ -1132,6 +1164,77 @@ tadm_status tadm_attention(const void* q, const void* k, const void* v, void* o,
     return TADM_ERR_INVALID_ARG;
   AttnCall a{q, k, v, o, batch, n_heads, n_kv_heads, head_dim, rows, ctx, kv_stride, causal, dtype, nullptr};
   return attention(a, stream) ? TADM_ERR_CUDA : TADM_OK;
+}
+
+tadm_status tadm_remdm_schedule(int kind, int T, int n, double eta, double t_on, double t_off, double alpha_on,
+                                double out[4]) {
+  if (!out || T < 1 || n < 0 || n >= T || remdm_args_error(kind, eta, t_on, t_off, alpha_on))
+    return TADM_ERR_INVALID_ARG;
+  remdm_step_constants(kind, T, n, eta, t_on, t_off, alpha_on, out);
+  return TADM_OK;
+}
+
+tadm_status tadm_remdm_uniforms(uint64_t seed, int step, int batch, int rows, float* out, tadm_stream stream) {
+  if (!out || batch <= 0 || rows <= 0 || step < 0) return TADM_ERR_INVALID_ARG;
+  return remdm_uniforms(seed, step, batch, rows, out, stream) ? TADM_ERR_CUDA : TADM_OK;
+}
+
+tadm_status tadm_remdm_update(int32_t* z, int ldz, const float* logits, int ld_logits, int batch, int rows,
+                              int first_gen, int vocab, int mask_id, double sigma, double p_unmask, float top_p,
+                              uint64_t seed, int step, int32_t* action, tadm_stream stream) {
+  if (!z || !logits || !action || batch <= 0 || rows <= 0 || ldz < rows || vocab < 2 || ld_logits < vocab ||
+      mask_id < 0 || mask_id >= vocab || first_gen < 0 || step < 0 || !(top_p > 0.0f && top_p <= 1.0f) ||
+      !(sigma >= 0.0 && sigma <= 1.0) || !(p_unmask >= 0.0 && p_unmask <= 1.0 + 1e-12))
+    return TADM_ERR_INVALID_ARG;
+  if (remdm_decide(z, ldz, batch, rows, first_gen, mask_id, sigma, p_unmask, seed, step, action, stream) ||
+      remdm_sample(logits, ld_logits, batch * rows, nullptr, action, z, ldz, batch, rows, vocab, mask_id, top_p, seed,
+                   step, stream))
+    return TADM_ERR_CUDA;
+  return TADM_OK;
+}
+
+tadm_status tadm_generate_remdm(tadm_handle* h, const int32_t* prompt, int batch, int prompt_len, int32_t* out,
+                                int gen_len, int steps, int K, int kind, double eta, float top_p, uint64_t seed,
+                                float* logits_scratch, size_t scratch_bytes, tadm_stream stream) {
+  if (!h) return TADM_ERR_INVALID_ARG;
+  constexpr double t_on = 0.55, t_off = 0.05, alpha_on = 0.9;
+  if (const char* e = remdm_args_error(kind, eta, t_on, t_off, alpha_on)) return fail(h, TADM_ERR_INVALID_ARG, "%s", e);
+  if (!prompt || !out || !logits_scratch) return fail(h, TADM_ERR_INVALID_ARG, "NULL pointer");
+  if (prompt_len < 0 || gen_len <= 0 || steps < 1 || K < 1 || !(top_p > 0.0f && top_p <= 1.0f))
+    return fail(h, TADM_ERR_INVALID_ARG, "need gen_len > 0, steps >= 1, K >= 1, 0 < top_p <= 1");
+  if (h->max_ctx > 0) return fail(h, TADM_ERR_INVALID_ARG, "the ReMDM sampler runs single-block canvases (max_ctx = 0)");
+  const tadm_config& c = h->cfg;
+  const int total = prompt_len + gen_len, R = total;
+  const size_t need = static_cast<size_t>(batch) * gen_len * c.vocab * sizeof(float);
+  if (scratch_bytes < need) return fail(h, TADM_ERR_INVALID_ARG, "logits_scratch needs %zu bytes", need);
+  TRYS(tadm_reset(h, batch));
+  TRYS(check_ready(h, batch, R));
+  h->last_stream = stream;
+  cudaStream_t s = stream;
+  const int mask = c.vocab - 1;
+  int32_t* act = h->at<int32_t>(h->off.tok);   // per-position actions (the top-k token buffer is unused here)
+  TRY(fill_canvas(out, total, prompt, batch, prompt_len, total, mask, s));
+  void* cache = h->at(h->off.h_int);
+  for (int n = 0; n < steps; ++n) {
+    TRYS(run_S(h, out, total, batch, R, 0, s));
+    if (n % K == 0) {                          // Alg. 1 refresh test (T - i) mod K = 0
+      TRYS(run_A(h, batch, R, 0, cache, s));
+      h->counters.anchor_layers += c.n_anchor;
+      h->counters.anchor_calls += 1;
+    }
+    TRYS(run_fusion(h, batch, R, cache, s));
+    // logits of the rows that hold MASK (at most gen_len per sequence), in list order
+    TRYS(run_D_head(h, batch, R, logits_scratch, s, out, total, gen_len, true));
+    double k[4];
+    remdm_step_constants(kind, steps, n, eta, t_on, t_off, alpha_on, k);
+    TRY(remdm_decide(out, total, batch, R, prompt_len, mask, k[2], k[3], seed, n, act, s));
+    TRY(remdm_sample(logits_scratch, c.vocab, batch * gen_len, h->at<int32_t>(h->off.idx), act, out, total, batch,
+                     R, c.vocab, mask, top_p, seed, n, s));
+    h->counters.shared_layers += c.n_shared;
+    h->counters.denoise_layers += c.n_denoise;
+    h->counters.denoise_steps += 1;
+  }
+  return TADM_OK;
 }
 
 }  // extern "C"

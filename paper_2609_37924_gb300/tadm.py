@@ -24,6 +24,7 @@ ABI_FUNCTIONS = [
     "tadm_sync_status", "tadm_get_counters", "tadm_plan", "tadm_layer_cost", "tadm_gemm", "tadm_confidence",
     "tadm_topk_unmask", "tadm_attention", "tadm_probe_enable", "tadm_probe_read", "tadm_head_scratch_size",
     "tadm_head_confidence", "tadm_head_confidence_static", "tadm_probe_breakdown",
+    "tadm_remdm_schedule", "tadm_remdm_uniforms", "tadm_remdm_update", "tadm_generate_remdm",
 ]
 
 
@@ -96,6 +97,13 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "tadm_head_confidence": (I, [P, P, I, I, I, I, I, P, SZ, P, P, P]),
         "tadm_head_confidence_static": (I, [P, P, I, I, I, I, I, P, P, P]),
         "tadm_probe_enable": (I, [P, I]),
+        "tadm_remdm_schedule": (I, [I, I, I, ctypes.c_double, ctypes.c_double, ctypes.c_double, ctypes.c_double,
+                                    ctypes.POINTER(ctypes.c_double)]),
+        "tadm_remdm_uniforms": (I, [ctypes.c_uint64, I, I, I, P, P]),
+        "tadm_remdm_update": (I, [P, I, P, I, I, I, I, I, I, ctypes.c_double, ctypes.c_double, ctypes.c_float,
+                                  ctypes.c_uint64, I, P, P]),
+        "tadm_generate_remdm": (I, [P, P, I, I, P, I, I, I, I, ctypes.c_double, ctypes.c_float, ctypes.c_uint64, P,
+                                    SZ, P]),
         "tadm_probe_breakdown": (I, [P, I, ctypes.POINTER(I64), ctypes.POINTER(ctypes.c_double),
                                      ctypes.POINTER(ctypes.c_double)]),
         "tadm_probe_read": (I, [P, ctypes.POINTER(I64), ctypes.POINTER(ctypes.c_double),
@@ -215,6 +223,32 @@ def tadm_attention(q, k, v, o, n_heads: int, n_kv_heads: int, rows: int, ctx: in
                                          ctx, kv_stride, int(causal), dtype, _stream(stream)))
 
 
+REMDM_KINDS = {"cap": 0, "loop": 1}
+
+
+def tadm_remdm_schedule(kind: str, T: int, n: int, eta: float, t_on: float = 0.55, t_off: float = 0.05,
+                        alpha_on: float = 0.9):
+    """(alpha_t, alpha_s, sigma_t, p_unmask) of reverse step n (host only)."""
+    out = (ctypes.c_double * 4)()
+    _check(load_library().tadm_remdm_schedule(REMDM_KINDS[kind], T, n, eta, t_on, t_off, alpha_on, out))
+    return tuple(out)
+
+
+def tadm_remdm_uniforms(seed: int, step: int, batch: int, rows: int, out, stream=None):
+    """The sampler's draws of a step into out (device float [batch, rows, 3])."""
+    _check(load_library().tadm_remdm_uniforms(seed, step, batch, rows, _ptr(out), _stream(stream)))
+
+
+def tadm_remdm_update(z, logits, first_gen: int, mask_id: int, sigma: float, p_unmask: float, top_p: float,
+                      seed: int, step: int, action, stream=None):
+    """One ReMDM reverse step on z [batch, rows] from logits [batch * rows, vocab]."""
+    batch, rows = z.shape
+    vocab = logits.shape[1]
+    _check(load_library().tadm_remdm_update(_ptr(z), rows, _ptr(logits), vocab, batch, rows, first_gen, vocab,
+                                            mask_id, sigma, p_unmask, top_p, seed, step, _ptr(action),
+                                            _stream(stream)))
+
+
 # ---------------------------------------------------------------------------- model handle
 class TadmModel:
     """A handle plus its torch-allocated workspace.
@@ -297,6 +331,14 @@ class TadmModel:
         B, P = prompt.shape
         _check(self.lib.tadm_generate(self.h, _ptr(prompt), B, P, _ptr(out), gen_len, steps_per_block, K,
                                       block_len, _stream(stream)), self.h)
+
+    def tadm_generate_remdm(self, prompt, out, gen_len: int, steps: int, K: int, kind: str, eta: float,
+                            top_p: float, seed: int, logits_scratch, stream=None):
+        B, P = prompt.shape
+        _check(self.lib.tadm_generate_remdm(self.h, _ptr(prompt), B, P, _ptr(out), gen_len, steps, K,
+                                            REMDM_KINDS[kind], eta, top_p, seed, _ptr(logits_scratch),
+                                            logits_scratch.numel() * logits_scratch.element_size(),
+                                            _stream(stream)), self.h)
 
     def tadm_sync_status(self):
         _check(self.lib.tadm_sync_status(self.h), self.h)

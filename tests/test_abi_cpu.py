@@ -109,3 +109,22 @@ def test_invalid_configs_are_rejected(lib):
     cfg = lib.make_config(base)
     assert so.tadm_create(ctypes.byref(cfg), None, 0, 1, 1, 0, ctypes.byref(h)) == 1   # no weights
     assert not h.value
+
+
+@pytest.mark.parametrize("kind,eta,T", [("cap", 0.04, 128), ("cap", 0.3, 7), ("loop", 0.02, 1024), ("loop", 0.02, 96)])
+def test_remdm_schedule_matches_the_oracle_bit_exactly(lib, kind, eta, T):
+    """The library's host schedule and the oracle's, written apart from the
+    same readings, agree to the last bit at every step (the decisions u < sigma
+    and u < p_unmask are then taken identically on both sides)."""
+    for n in range(T):
+        assert lib.tadm_remdm_schedule(kind, T, n, eta) == O.remdm_schedule(n, T, kind, eta)
+
+
+def test_remdm_arguments_are_rejected(lib):
+    so = lib.load_library()
+    out = (ctypes.c_double * 4)()
+    for args in [(0, 0, 0, 0.04, 0.55, 0.05, 0.9), (0, 8, 8, 0.04, 0.55, 0.05, 0.9), (2, 8, 0, 0.04, 0.55, 0.05, 0.9),
+                 (0, 8, 0, -1.0, 0.55, 0.05, 0.9), (1, 8, 0, 0.02, 0.05, 0.55, 0.9), (1, 8, 0, 0.02, 0.55, 0.05, 1.0)]:
+        assert so.tadm_remdm_schedule(*args, out) == 1, args
+    # null buffers / out-of-range probabilities fail before any launch
+    assert so.tadm_remdm_update(None, 4, None, 8, 1, 4, 0, 8, 7, 0.1, 0.1, 0.9, 1, 0, None, None) == 1
