@@ -116,6 +116,7 @@ struct TcArgs {
   int b_split;             // >0: B tile = 128 rows at n*128 and 128 rows at b_split + n*128
   int n_tiles_n;
   int* status;
+  const int* m_dev;        // optional device row count (<= M): tiles past it are skipped
   EpiParams ep;
 };
 
@@ -182,7 +183,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
-  const int num_m = (args.M + BM - 1) / BM;
+  const int m_run = args.m_dev ? min(args.M, *args.m_dev) : args.M;   // read after pdl_enter
+  const int num_m = (m_run + BM - 1) / BM;
   const int tiles = num_m * args.n_tiles_n;
   const int units = tiles * args.splits;
   const int kblocks = (args.K + BK - 1) / BK;
@@ -376,7 +378,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
-  const int num_m2 = (args.M + 2 * BM - 1) / (2 * BM);
+  const int m_run = args.m_dev ? min(args.M, *args.m_dev) : args.M;   // read after pdl_enter
+  const int num_m2 = (m_run + 2 * BM - 1) / (2 * BM);
   const int units = num_m2 * args.n_tiles_n;
   const int u0 = static_cast<int>(blockIdx.x >> 1), ustep = static_cast<int>(gridDim.x >> 1);
   const int kblocks = (args.K + BK - 1) / BK;
@@ -607,6 +610,7 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
   if (g.epi == EPI_QKV && BN % g.ep.head_dim) return "head_dim must divide 256";
   if (g.epi == EPI_PA_GATE && g.N > BN) return "gate GEMM needs N <= 256";
   a.status = g.status;
+  a.m_dev = g.m_dev;
   a.ep = g.ep;
   a.ep.M = g.M;
   a.ep.N = g.N;
@@ -646,7 +650,7 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
                       m_pairs * a.n_tiles_n * 4 <= g_num_sms;
   const int pair_units = narrow ? m_pairs * ((g.N + 127) / 128) : m_pairs * a.n_tiles_n;
   const bool pairs_fill = pair_ok && 2 * pair_units * 5 >= g_num_sms * 2;
-  if (g.split_buf && !pairs_fill && tiles * 3 < g_num_sms * 2 && kblocks >= 8) {
+  if (g.split_buf && !g.m_dev && !pairs_fill && tiles * 3 < g_num_sms * 2 && kblocks >= 8) {
     int sp = std::min(std::min(g_num_sms / tiles, kblocks / 4), 16);
     const size_t per = static_cast<size_t>(g.M) * a.ldp * sizeof(float);
     while (sp > 1 && sp * per > g.split_bytes) --sp;

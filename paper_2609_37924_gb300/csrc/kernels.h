@@ -35,6 +35,7 @@ struct GemmCall {
   int epi;
   EpiParams ep;
   int* status;
+  const int* m_dev = nullptr;   // optional device row count <= M (tcgen05 path): tiles past it are skipped
   float* split_buf;      // fp32 partials for split-K (null: no split)
   size_t split_bytes;
   int launched;          // out: kernels launched
@@ -101,7 +102,9 @@ const char* remdm_decide(int32_t* z, int ldz, int B, int R, int first_gen, int m
                          double p_unmask, uint64_t seed, int step, int32_t* act, cudaStream_t s);
 const char* remdm_sample(const float* logits, int ld, int n_rows, const int32_t* idx, const int32_t* act, int32_t* z,
                          int ldz, int B, int R, int vocab, int mask_id, float top_p, uint64_t seed, int step,
-                         cudaStream_t s);
+                         cudaStream_t s, const int* count = nullptr);
+// rows with action 2 in row order into idx[0 .. *count), padded to `bound` entries
+const char* remdm_rows(const int32_t* act, int n, int bound, int32_t* idx, int* count, cudaStream_t s);
 const char* topk_unmask(int32_t* z, int ldz, const float* conf, const int32_t* tok, int batch, int rows, int k,
                         int mask_id, int32_t* selected, cudaStream_t s);
 

@@ -248,6 +248,42 @@ __global__ void remdm_decide_kernel(int32_t* __restrict__ z, int ldz, int B, int
   act[i] = a;
 }
 
+// One 1024-thread block: the rows with action 2 in row order, idx[0 .. count),
+// *count; entries count .. bound-1 repeat the first such row (or row 0), so
+// every entry names a valid row for gathers sized by the bound.
+__global__ void __launch_bounds__(1024) remdm_rows_kernel(const int32_t* __restrict__ act, int n, int bound,
+                                                          int32_t* __restrict__ idx, int* __restrict__ count) {
+  pdl_enter();
+  __shared__ int wsum[32];
+  __shared__ int base;
+  if (threadIdx.x == 0) base = 0;
+  __syncthreads();
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  for (int r0 = 0; r0 < n; r0 += 1024) {
+    const int r = r0 + threadIdx.x;
+    const bool on = r < n && act[r] == 2;
+    const unsigned ballot = __ballot_sync(0xffffffffu, on);
+    if (lane == 0) wsum[w] = __popc(ballot);
+    __syncthreads();
+    int before = base;
+    for (int i = 0; i < w; ++i) before += wsum[i];
+    const int j = before + __popc(ballot & ((1u << lane) - 1u));
+    if (on && j < bound) idx[j] = r;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int t = 0;
+      for (int i = 0; i < 32; ++i) t += wsum[i];
+      base += t;
+    }
+    __syncthreads();
+  }
+  const int cnt = min(base, bound);
+  __syncthreads();
+  const int fill = cnt > 0 ? idx[0] : 0;
+  for (int j = cnt + threadIdx.x; j < bound; j += 1024) idx[j] = fill;
+  if (threadIdx.x == 0) *count = cnt;
+}
+
 template <int NT>
 __device__ __forceinline__ float block_sum_f(float v, float* red) {
   v = warp_sum(v);
@@ -271,13 +307,14 @@ template <int NT>
 __global__ void __launch_bounds__(NT) remdm_sample_kernel(const float* __restrict__ logits, int ld, int n_rows,
                                                           const int32_t* __restrict__ idx, const int32_t* __restrict__ act,
                                                           int32_t* __restrict__ z, int ldz, int B, int R, int vocab,
-                                                          int mask_id, float top_p, uint64_t seed, int step) {
+                                                          int mask_id, float top_p, uint64_t seed, int step,
+                                                          const int* __restrict__ count) {
   pdl_enter();
   __shared__ float red[NT / 32];
   __shared__ float scan[NT];
   __shared__ int pick;
   const int j = blockIdx.x;
-  if (j >= n_rows) return;
+  if (j >= n_rows || (count && j >= *count)) return;
   const int row = idx ? idx[j] : j;
   if (act[row] != 2) return;                     // uniform across the block
   const int b = row / R, r = row - (row / R) * R;
@@ -366,6 +403,106 @@ __global__ void __launch_bounds__(NT) remdm_sample_kernel(const float* __restric
   }
 }
 
+// remdm_sample_kernel with the row's probabilities staged once in shared
+// memory (q_v = exp(l_v - max), 0 for MASK; vocab * 4 bytes of dynamic
+// shared memory): the bisection sums read shared memory with a strided
+// (bank-conflict-free) assignment, the id-order draw uses contiguous ranges.
+template <int NT>
+__global__ void __launch_bounds__(NT) remdm_sample_smem_kernel(const float* __restrict__ logits, int ld, int n_rows,
+                                                               const int32_t* __restrict__ idx,
+                                                               const int32_t* __restrict__ act, int32_t* __restrict__ z,
+                                                               int ldz, int B, int R, int vocab, int mask_id,
+                                                               float top_p, uint64_t seed, int step,
+                                                               const int* __restrict__ count) {
+  pdl_enter();
+  extern __shared__ float qs[];
+  __shared__ float red[NT / 32];
+  __shared__ float scan[NT];
+  __shared__ int pick;
+  const int j = blockIdx.x;
+  if (j >= n_rows || (count && j >= *count)) return;
+  const int row = idx ? idx[j] : j;
+  if (act[row] != 2) return;
+  const int b = row / R, r = row - (row / R) * R;
+  const float* L = logits + static_cast<size_t>(j) * ld;
+  const int tid = threadIdx.x;
+  float mx = -INFINITY;
+  for (int v = tid; v < vocab; v += NT) {
+    const float l = L[v];
+    qs[v] = l;
+    if (v != mask_id) mx = fmaxf(mx, l);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  if ((tid & 31) == 0) red[tid >> 5] = mx;
+  __syncthreads();
+  mx = red[0];
+#pragma unroll
+  for (int w = 1; w < NT / 32; ++w) mx = fmaxf(mx, red[w]);
+  for (int v = tid; v < vocab; v += NT) qs[v] = v == mask_id ? 0.0f : expf(qs[v] - mx);
+  auto mass_from = [&](float tau) {
+    float acc = 0.0f;
+    for (int v = tid; v < vocab; v += NT) {
+      const float q = qs[v];
+      acc += q >= tau && q > 0.0f ? q : 0.0f;
+    }
+    return block_sum_f<NT>(acc, red);
+  };
+  const float total = mass_from(0.0f);
+  const float target = top_p * total;
+  uint32_t lo = 0u, hi = 0x3F800001u;
+  while (hi - lo > 1u) {
+    const uint32_t mid = lo + (hi - lo) / 2u;
+    if (mass_from(__uint_as_float(mid)) >= target) lo = mid;
+    else hi = mid;
+  }
+  const float tau = __uint_as_float(lo);
+  const int chunk = (vocab + NT - 1) / NT, v0 = tid * chunk, v1 = min(vocab, v0 + chunk);
+  float mine = 0.0f;
+  for (int v = v0; v < v1; ++v) {
+    const float q = qs[v];
+    mine += q >= tau && q > 0.0f ? q : 0.0f;
+  }
+  scan[tid] = mine;
+  if (tid == 0) pick = -1;
+  __syncthreads();
+  for (int o = 1; o < NT; o <<= 1) {
+    const float add = tid >= o ? scan[tid - o] : 0.0f;
+    __syncthreads();
+    scan[tid] += add;
+    __syncthreads();
+  }
+  float u[3];
+  remdm_draws(seed, step, B, R, b, r, u);
+  const float goal = u[2] * scan[NT - 1];
+  const float before = tid > 0 ? scan[tid - 1] : 0.0f;
+  if (mine > 0.0f && before <= goal && goal < scan[tid]) {
+    float c = before;
+    int last = -1, got = -1;
+    for (int v = v0; v < v1; ++v) {
+      const float q = qs[v];
+      if (q >= tau && q > 0.0f) {
+        last = v;
+        c += q;
+        if (c > goal) {
+          got = v;
+          break;
+        }
+      }
+    }
+    pick = got >= 0 ? got : last;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    int v = pick;
+    for (int t = NT - 1; t >= 0 && v < 0; --t)   // rounding left the goal past every range: the last token
+      if ((t > 0 ? scan[t] - scan[t - 1] : scan[0]) > 0.0f)
+        for (int w = min(vocab, (t + 1) * chunk) - 1; w >= t * chunk; --w)
+          if (qs[w] >= tau && qs[w] > 0.0f) { v = w; break; }
+    z[static_cast<size_t>(b) * ldz + r] = v;
+  }
+}
+
 }  // namespace
 
 const char* confidence_rows(const float* logits, int rows, int vocab, int ld, int mask_id, float* conf, int32_t* tok,
@@ -412,10 +549,28 @@ const char* remdm_decide(int32_t* z, int ldz, int B, int R, int first_gen, int m
 
 const char* remdm_sample(const float* logits, int ld, int n_rows, const int32_t* idx, const int32_t* act, int32_t* z,
                          int ldz, int B, int R, int vocab, int mask_id, float top_p, uint64_t seed, int step,
-                         cudaStream_t s) {
+                         cudaStream_t s, const int* count) {
   if (n_rows <= 0) return nullptr;
-  launch_pdl(remdm_sample_kernel<256>, n_rows, 256, 0, s, logits, ld, n_rows, idx, act, z, ldz, B, R, vocab, mask_id,
-             top_p, seed, step);
+  const size_t smem = static_cast<size_t>(vocab) * sizeof(float);
+  if (smem <= 200u * 1024u) {   // the row's probabilities fit in shared memory
+    static bool attr = false;
+    if (!attr) {
+      if (cudaFuncSetAttribute(remdm_sample_smem_kernel<1024>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               200 * 1024) != cudaSuccess)
+        return "sampler smem attribute failed";
+      attr = true;
+    }
+    launch_pdl(remdm_sample_smem_kernel<1024>, n_rows, 1024, smem, s, logits, ld, n_rows, idx, act, z, ldz, B, R,
+               vocab, mask_id, top_p, seed, step, count);
+  } else {
+    launch_pdl(remdm_sample_kernel<256>, n_rows, 256, 0, s, logits, ld, n_rows, idx, act, z, ldz, B, R, vocab,
+               mask_id, top_p, seed, step, count);
+  }
+  return err();
+}
+
+const char* remdm_rows(const int32_t* act, int n, int bound, int32_t* idx, int* count, cudaStream_t s) {
+  launch_pdl(remdm_rows_kernel, 1, 1024, 0, s, act, n, bound, idx, count);
   return err();
 }
 

@@ -119,7 +119,7 @@ struct tadm_handle {
   size_t ws_bytes = 0, ws_need = 0;
   struct Off {
     size_t status, rope, c, x, h_int, norm, qbuf, kv, attn, glu, f_g, f_hid, f_pre, part, conf, tok, split, idx;
-    size_t attn_part;
+    size_t attn_part, act, cnt;
     size_t pa_z, pa_j, pa_mq, pa_mk, pa_mv, pa_mo, pa_r, pa_rb, pa_hid, pa_phi, pa_m, pa_dz, pa_f, pa_g, pa_mb;
   } off{};
   size_t kv_slab = 0;
@@ -269,6 +269,8 @@ void layout(tadm_handle* h) {
   f.part = take(M * h->n_part_tiles * 3 * 4);
   f.split = c.dtype ? take(gemm_tc_split_bytes()) : take(0);
   f.attn_part = c.dtype ? take(kAttnPartBytes) : take(0);
+  f.act = take(M * 4);       // ReMDM: per-position actions
+  f.cnt = take(256);         // ReMDM: device count of unmasking rows
   f.conf = take(M * 4);
   f.tok = take(M * 4);
   f.idx = take(M * 4);
@@ -292,7 +294,7 @@ void probe_end(tadm_handle* h, cudaStream_t s, int idx, int kind, double flops) 
 }
 
 tadm_status gemm(tadm_handle* h, const void* A, int64_t a_rows, int lda, const void* B, int ldb, int M, int N, int K,
-                 int epi, const EpiParams& ep, cudaStream_t s, bool out_f32 = false) {
+                 int epi, const EpiParams& ep, cudaStream_t s, bool out_f32 = false, const int* m_dev = nullptr) {
   GemmCall g{};
   g.A = A;
   g.B = B;
@@ -305,6 +307,7 @@ tadm_status gemm(tadm_handle* h, const void* A, int64_t a_rows, int lda, const v
   g.epi = epi;
   g.ep = ep;
   g.status = h->status();
+  g.m_dev = m_dev;
   if (h->cfg.dtype) {
     g.split_buf = h->at<float>(h->off.split);
     g.split_bytes = gemm_tc_split_bytes();
@@ -1212,7 +1215,11 @@ tadm_status tadm_generate_remdm(tadm_handle* h, const int32_t* prompt, int batch
   h->last_stream = stream;
   cudaStream_t s = stream;
   const int mask = c.vocab - 1;
-  int32_t* act = h->at<int32_t>(h->off.tok);   // per-position actions (the top-k token buffer is unused here)
+  int32_t* act = h->at<int32_t>(h->off.act);
+  int32_t* idx = h->at<int32_t>(h->off.idx);
+  int* cnt = h->at<int>(h->off.cnt);
+  const int bound = batch * gen_len;           // unmasking rows of a step: at most every generated position
+  const int64_t Mmax = static_cast<int64_t>(h->max_batch) * h->max_rows;
   TRY(fill_canvas(out, total, prompt, batch, prompt_len, total, mask, s));
   void* cache = h->at(h->off.h_int);
   for (int n = 0; n < steps; ++n) {
@@ -1223,13 +1230,24 @@ tadm_status tadm_generate_remdm(tadm_handle* h, const int32_t* prompt, int batch
       h->counters.anchor_calls += 1;
     }
     TRYS(run_fusion(h, batch, R, cache, s));
-    // logits of the rows that hold MASK (at most gen_len per sequence), in list order
-    TRYS(run_D_head(h, batch, R, logits_scratch, s, out, total, gen_len, true));
+    float* x = h->at<float>(h->off.x);
+    TRYS(stack_fwd(h, c.n_shared + c.n_anchor, c.n_denoise, x, batch, R, 0, 0, s));
+    // the decisions need only the draws and z_t: decide (remasks applied), then
+    // run the output head on the unmasking rows alone (device count)
     double k[4];
     remdm_step_constants(kind, steps, n, eta, t_on, t_off, alpha_on, k);
     TRY(remdm_decide(out, total, batch, R, prompt_len, mask, k[2], k[3], seed, n, act, s));
-    TRY(remdm_sample(logits_scratch, c.vocab, batch * gen_len, h->at<int32_t>(h->off.idx), act, out, total, batch,
-                     R, c.vocab, mask, top_p, seed, n, s));
+    TRY(remdm_rows(act, batch * R, bound, idx, cnt, s));
+    void* norm = h->at(h->off.norm);
+    TRY(rmsnorm_rows(x, bound, c.d_model, h->final_norm, c.dtype, c.norm_eps, norm, c.d_model, h->act_bf16(), s, idx));
+    EpiParams e{};
+    e.part = h->at<float>(h->off.part);
+    e.mask_id = mask;
+    e.logits = logits_scratch;
+    e.ld_logits = c.vocab;
+    TRYS(gemm(h, norm, Mmax, c.d_model, h->lm_head, c.d_model, bound, c.vocab, c.d_model, EPI_LMHEAD, e, s, false, cnt));
+    TRY(remdm_sample(logits_scratch, c.vocab, bound, idx, act, out, total, batch, R, c.vocab, mask, top_p, seed, n, s,
+                     cnt));
     h->counters.shared_layers += c.n_shared;
     h->counters.denoise_layers += c.n_denoise;
     h->counters.denoise_steps += 1;
