@@ -23,6 +23,8 @@ What it computes (paper section / equation it follows):
 * ReMDM remasking sampler (the paper's Pretraining sampler, NEXT row):
   §5 Eq. (inf-post-TADM), App. B Eqs. (remdm-posterior, remdm-param), with
   the linear schedule, nucleus p and Cap / Loop settings of App. C.2.
+* DiffusionGemma entropy-bound sampler with self-conditioning (the paper's
+  Post-train sampler, NEXT row): Alg. 2 with the App. C.1 settings.
 * Block diffusion with a KV cache over committed blocks (the encoder prefills
   the context causally, the decoder denoises the active block
   bidirectionally): App. C.1, "Architecture Details".
@@ -260,6 +262,42 @@ def remdm_step(z: np.ndarray, logits: np.ndarray, first_gen: int, sigma: float, 
     return out, act
 
 
+# ---------------------------------------------------------------------------
+# DiffusionGemma entropy-bound sampler (Alg. 2, App. C.1 "Sampler Details")
+# ---------------------------------------------------------------------------
+def eb_temperature(n: int, T: int, tau_max: float, tau_min: float) -> float:
+    """tau_n = tau_min + (tau_max - tau_min) n / T for n = T .. 1 (Alg. 2)."""
+    return tau_min + (tau_max - tau_min) * n / T
+
+
+def eb_row(logits: np.ndarray, tau: float, mask_id: int, u: float):
+    """Per position of Alg. 2: p = softmax(l / tau) over ids != MASK, the
+    argmax (ties to the lowest id), the entropy H = -sum p log p, and a draw
+    from Cat(p) by inverse CDF in id order (first v whose cumulative p
+    exceeds u).  Returns (p, argmax, H, draw)."""
+    l = np.asarray(logits, dtype=np.float64) / tau
+    l[mask_id] = -np.inf
+    e = np.exp(l - np.max(l))
+    p = e / e.sum()
+    nz = p > 0
+    H = float(-np.sum(p[nz] * np.log(p[nz])))
+    c = np.cumsum(p)
+    draw = int(np.nonzero(c > u * c[-1])[0][0])
+    return p, int(np.argmax(p)), H, draw
+
+
+def eb_accept(H: np.ndarray, eta: float) -> np.ndarray:
+    """Alg. 2's accepted set: positions in ascending entropy (ties to the
+    lower position), pi_m accepted when C_m - M_m <= eta, C_m the summed
+    entropy of the first m and M_m their maximum (= H of pi_m)."""
+    order = np.lexsort((np.arange(H.size), H))
+    C = np.cumsum(H[order])
+    M = np.maximum.accumulate(H[order])
+    ok = np.zeros(H.size, dtype=bool)
+    ok[order[C - M <= eta]] = True
+    return ok
+
+
 def layer_cost(L_S: int, L_A: int, L_D: int, T: int, K: int):
     """Eq. (anchor-cache-compute): (C_full, C_cache) transformer-layer calls."""
     c_full = T * (L_S + L_A + L_D)
@@ -354,9 +392,12 @@ class Oracle:
         return x
 
     # -- S, A, D (§3.1) -----------------------------------------------------
-    def S(self, z: np.ndarray, pos, seq, causal=False, keep_kv=False, count=True) -> np.ndarray:
-        """Shared network: token embedding, then L_S backbone layers."""
+    def S(self, z: np.ndarray, pos, seq, causal=False, keep_kv=False, count=True, add=None) -> np.ndarray:
+        """Shared network: token embedding (+ ``add``, the self-conditioning
+        signal of Alg. 2), then L_S backbone layers."""
         c = self.W("embed")[z.astype(np.int64)]
+        if add is not None:
+            c = c + add
         return self.stack("shared", self.m.n_shared, c, pos, seq, causal, keep_kv, count)
 
     def A(self, c, pos, seq, causal=False, keep_kv=False, count=True) -> np.ndarray:
@@ -556,6 +597,61 @@ class Oracle:
             if step_hook is not None:
                 step_hook(n, z, logits, new)
             z = new
+            self.counters["steps"] += 1
+        return z
+
+    def generate_entropy_bound(self, prompts: np.ndarray, gen_len: int, T: int, K: int, eta: float,
+                               tau_max: float, tau_min: float, uniforms, self_cond: bool = True,
+                               step_hook=None) -> np.ndarray:
+        """Alg. 2 (DiffusionGemma entropy-bound sampling) with the anchor
+        cache of Alg. 1 on one canvas (prompt + gen_len generated positions,
+        single block).  The canvas starts as uniform noise over ids != MASK;
+        step i = 0 .. T-1 is Alg. 2's n = T - i: refresh when i mod K = 0,
+        logits of the fused prediction with the self-conditioning signal s
+        added to the input embedding of the generated positions, p, argmax,
+        entropy and a draw per position, s <- p E; for n > 1 accepted
+        positions take their draw and the others fresh noise; n = 1 returns
+        the argmax canvas.  ``uniforms(i)`` gives [B, P + gen_len, 3] draws of
+        step i (draw, noise token, unused); step T gives the initial noise.
+        ``step_hook(n, z, new_z, H)`` sees each step's canvas before and after
+        and the entropies of the generated positions."""
+        B, P = prompts.shape
+        V, mask, d = self.m.vocab, self.mask_id, self.m.d_model
+        L = P + gen_len
+        pos = np.arange(L)
+        E = self.W("embed")
+        u = uniforms(T)
+        z = np.concatenate([prompts.astype(np.int32),
+                            np.floor(u[:, P:, 1] * (V - 1)).astype(np.int32)], axis=1)
+        s = np.zeros((B, L, d))
+        cache = [None] * B
+        for i in range(T):
+            n = T - i
+            if i % K == 0:
+                for b in range(B):
+                    c = self.S(z[b], pos, None, count=False, add=s[b])
+                    cache[b] = self.make_cache(c, self.A(c, pos, None, count=(b == 0)))
+                self.counters["anchor_calls"] += 1
+            tau = eb_temperature(n, T, tau_max, tau_min)
+            u = uniforms(i)
+            new_z, new_s, Hs = z.copy(), np.zeros_like(s), np.zeros((B, gen_len))
+            for b in range(B):
+                c = self.S(z[b], pos, None, count=(b == 0), add=s[b])
+                logits = self.lm_head(self.D_hidden(self.fuse(c, cache[b]), pos, None, count=(b == 0)))
+                H, draw, am = np.zeros(gen_len), np.zeros(gen_len, np.int32), np.zeros(gen_len, np.int32)
+                for g in range(gen_len):
+                    p, am[g], H[g], draw[g] = eb_row(logits[P + g], tau, mask, u[b, P + g, 0])
+                    new_s[b, P + g] = p @ E
+                if n > 1:
+                    noise = np.floor(u[b, P:, 1] * (V - 1)).astype(np.int32)
+                    new_z[b, P:] = np.where(eb_accept(H, eta), draw, noise)
+                else:
+                    new_z[b, P:] = am
+                Hs[b] = H
+            if step_hook is not None:
+                step_hook(n, z, new_z, Hs)
+            z = new_z
+            s = new_s if self_cond else np.zeros_like(s)
             self.counters["steps"] += 1
         return z
 

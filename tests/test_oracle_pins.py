@@ -630,3 +630,152 @@ def test_remdm_token_uses_its_own_uniform():
     lg[0, 3] = lg[0, 7] = 0.0
     out, act = O.remdm_step(np.array([9], np.int32), lg, 0, 0.0, 0.5, 0.9, np.array([[0.99, 0.1, 0.9]]), 9)
     assert act[0] == 2 and out[0] == 7
+
+
+# ---------------------------------------------------------- entropy-bound sampler (Alg. 2, NEXT row)
+def test_eb_temperature_is_linear_between_the_limits():
+    T = 48
+    assert O.eb_temperature(T, T, 0.8, 0.4) == 0.8 and abs(O.eb_temperature(0, T, 0.8, 0.4) - 0.4) < 1e-15
+    d = [O.eb_temperature(n, T, 0.8, 0.4) - O.eb_temperature(n - 1, T, 0.8, 0.4) for n in range(1, T + 1)]
+    assert np.allclose(d, 0.4 / T, atol=1e-15)
+
+
+def test_eb_row_closed_forms():
+    """Uniform logits: p uniform over the V-1 ids != MASK and H = log(V-1);
+    argmax ties go to the lowest id; a dominant logit gives H -> 0; the draws
+    on a grid of u reproduce p (inverse CDF in id order)."""
+    V, mask = 9, 8
+    p, am, H, _ = O.eb_row(np.zeros(V), 0.7, mask, 0.3)
+    assert np.allclose(p[:mask], 1 / 8) and p[mask] == 0.0 and am == 0 and abs(H - np.log(8)) < 1e-12
+    lg = np.zeros(V)
+    lg[5] = 60.0
+    assert O.eb_row(lg, 0.5, mask, 0.9)[2] < 1e-30 and O.eb_row(lg, 0.5, mask, 0.9)[1] == 5
+    lg = rng.standard_normal(V)
+    p = O.eb_row(lg, 0.6, mask, 0.0)[0]
+    q = np.exp(lg[:mask] / 0.6 - (lg[:mask] / 0.6).max())
+    assert np.allclose(p[:mask], q / q.sum())
+    grid = (np.arange(20000) + 0.5) / 20000
+    got = np.bincount([O.eb_row(lg, 0.6, mask, u)[3] for u in grid], minlength=V) / grid.size
+    assert np.allclose(got, p, atol=1e-4)
+
+
+def test_eb_accept_against_a_direct_loop():
+    """Accepted set of Alg. 2 by brute force: walk the positions in ascending
+    entropy and accept a position while the entropy of the ones before it
+    sums to at most eta; at least the lowest-entropy position is accepted."""
+    assert list(O.eb_accept(np.array([0.2, 0.2, 0.2]), 0.1)) == [True, False, False]
+    assert list(O.eb_accept(np.array([0.05, 0.01, 0.3, 0.02]), 0.1)) == [True, True, True, True]
+    for _ in range(50):
+        H = rng.random(30) * rng.choice([0.01, 0.1, 1.0])
+        eta = rng.choice([0.0, 0.05, 0.5])
+        want = np.zeros(30, bool)
+        acc = 0.0
+        for r in sorted(range(30), key=lambda i: (H[i], i)):
+            if acc <= eta:
+                want[r] = True
+            acc += H[r]
+        assert np.array_equal(O.eb_accept(H, eta), want)
+
+
+def test_eb_one_step_is_the_argmax_of_the_noise_canvas():
+    """T = 1 (n = 1 only): the output is the argmax of the fused prediction
+    on the initial noise canvas, which the test rebuilds from the network."""
+    o = tiny_oracle()
+    P, G, V = 3, 5, o.m.vocab
+    prompts = rng.integers(0, V - 1, (2, P)).astype(np.int32)
+    draws = lambda i: wl.remdm_uniforms(3, i, 2, P + G)  # noqa: E731
+    out = o.generate_entropy_bound(prompts, G, 1, 1, 0.1, 0.8, 0.4, draws)
+    u = draws(1)
+    for b in range(2):
+        z = np.concatenate([prompts[b], np.floor(u[b, P:, 1] * (V - 1)).astype(np.int32)])
+        pos = np.arange(P + G)
+        c = o.S(z, pos, None)
+        logits = o.lm_head(o.D_hidden(o.fuse(c, o.make_cache(c, o.A(c, pos, None))), pos, None))
+        assert np.array_equal(out[b, P:], np.argmax(np.where(np.arange(V) == o.mask_id, -np.inf, logits[P:]), -1))
+        assert np.array_equal(out[b, :P], prompts[b])
+
+
+def test_eb_unbounded_accepts_every_draw_and_refreshes_per_alg1():
+    """eta = inf accepts every position, so before the last step the canvas
+    is the categorical draws; the anchor refreshes ceil(T / K) times."""
+    o = tiny_oracle()
+    P, G = 2, 4
+    prompts = np.array([[1, 2]], np.int32)
+    seen = []
+    draws = lambda i: (seen.append(i), wl.remdm_uniforms(9, i, 1, P + G))[1]  # noqa: E731
+    o.counters["anchor_calls"] = 0
+    out = o.generate_entropy_bound(prompts, G, 5, 2, np.inf, 0.8, 0.4, draws)
+    assert o.counters["anchor_calls"] == 3 and seen == [5, 0, 1, 2, 3, 4]
+    assert out.shape == (1, P + G) and np.all(out != o.mask_id)
+
+
+def test_eb_draw_intervals_are_half_open():
+    """Cat(p) by inverse CDF: id v owns [c_{v-1}, c_v), so u on an edge
+    belongs to the next id (uniform p = 1/8, exact binary fractions)."""
+    lg = np.zeros(9)
+    assert [O.eb_row(lg, 1.0, 8, u)[3] for u in (0.0, 0.124, 0.125, 0.25, 0.875, 0.9999)] == [0, 0, 1, 2, 7, 7]
+
+
+def test_eb_rejected_positions_are_renoised_uniformly():
+    """eta < 0 accepts nothing: every generated position of a step n > 1
+    becomes floor(u1 (V - 1)) of that step's draws, an id != MASK, and the
+    prompt stays; with eta = inf every position keeps its categorical draw."""
+    o = tiny_oracle()
+    P, G, V = 2, 6, o.m.vocab
+    prompts = np.array([[3, 4]], np.int32)
+    draws = lambda i: wl.remdm_uniforms(21, i, 1, P + G)  # noqa: E731
+    seen = []
+    o.generate_entropy_bound(prompts, G, 3, 1, -1.0, 0.8, 0.4, draws,
+                             step_hook=lambda n, z, new, H: seen.append((n, new.copy(), H.copy())))
+    assert [n for n, _, _ in seen] == [3, 2, 1]
+    for i, (n, new, H) in enumerate(seen[:2]):
+        want = np.floor(draws(i)[0, P:, 1] * (V - 1)).astype(np.int32)
+        assert np.array_equal(new[0, P:], want) and np.array_equal(new[0, :P], prompts[0])
+        assert np.all(H >= 0) and np.all(H <= np.log(V - 1) + 1e-12)
+
+
+def test_eb_self_conditioning_feeds_p_E_into_the_next_step():
+    """T = 2, K = 2, eta = inf: step n = 2 runs on the noise canvas with s = 0
+    and every position takes its draw; step n = 1 (tau = 0.6) embeds that
+    canvas plus s = p_2 E, reuses the anchor cache of step n = 2 and returns
+    the argmax.  Without self-conditioning the second step sees s = 0.  The
+    entropies of step n = 1 carry the difference (the argmax may not)."""
+    o = tiny_oracle()
+    P, G, V = 2, 5, o.m.vocab
+    prompts = np.array([[7, 1]], np.int32)
+    draws = lambda i: wl.remdm_uniforms(33, i, 1, P + G)  # noqa: E731
+    pos, E = np.arange(P + G), o.W("embed")
+    z = np.concatenate([prompts[0], np.floor(draws(2)[0, P:, 1] * (V - 1)).astype(np.int32)])
+    c = o.S(z, pos, None)
+    cache = o.make_cache(c, o.A(c, pos, None))
+    lg = o.lm_head(o.D_hidden(o.fuse(c, cache), pos, None))
+    s = np.zeros((P + G, o.m.d_model))
+    for g in range(G):
+        p, _, _, z[P + g] = O.eb_row(lg[P + g], 0.8, o.mask_id, draws(0)[0, P + g, 0])
+        s[P + g] = p @ E
+    H1 = {}
+    for sc, add in ((True, s), (False, None)):
+        c = o.S(z, pos, None, add=add)
+        lg = o.lm_head(o.D_hidden(o.fuse(c, cache), pos, None))
+        rows = [O.eb_row(lg[P + g], 0.6, o.mask_id, 0.5) for g in range(G)]
+        H1[sc] = np.array([r[2] for r in rows])
+        seen = []
+        got = o.generate_entropy_bound(prompts, G, 2, 2, np.inf, 0.8, 0.4, draws, self_cond=sc,
+                                       step_hook=lambda n, z0, new, H: seen.append((n, H.copy())))
+        assert np.array_equal(got[0, P:], [r[1] for r in rows]), sc
+        assert [n for n, _ in seen] == [2, 1] and np.allclose(seen[1][1][0], H1[sc], rtol=1e-12, atol=0), sc
+    assert np.max(np.abs(H1[True] - H1[False])) > 1e-6
+
+
+def test_eb_signal_enters_as_an_embedding_offset():
+    """The self-conditioning signal is added to the token embedding: adding
+    E[v] - E[z_l] at position l gives the shared network's output for the
+    canvas with z_l replaced by v."""
+    o = tiny_oracle()
+    z = np.array([1, 5, 9, 2, 4], np.int32)
+    pos, E = np.arange(5), o.W("embed")
+    add = np.zeros((5, o.m.d_model))
+    add[3] = E[11] - E[2]
+    z2 = z.copy()
+    z2[3] = 11
+    assert np.allclose(o.S(z, pos, None, add=add), o.S(z2, pos, None), rtol=1e-12, atol=1e-12)
