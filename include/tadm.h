@@ -372,6 +372,63 @@ TADM_API tadm_status tadm_generate_remdm(tadm_handle* h, const int32_t* prompt, 
                                          float top_p, uint64_t seed, float* logits_scratch, size_t scratch_bytes,
                                          tadm_stream stream);
 
+/* ---------------------------------------------------- entropy-bound sampler --
+ * The paper's Post-training sampler (App. C.1 "Sampler Details", Alg. 2:
+ * DiffusionGemma entropy-bound sampling) with Alg. 1's anchor cache.  Per
+ * reverse step n = T .. 1 and generated position l:
+ *  - tau_n = tau_min + (tau_max - tau_min) n / T; p = softmax(L / tau_n) over
+ *    the ids != MASK (MASK = vocab - 1 gets p = 0); the argmax takes the
+ *    lowest id among equal logits; H = -sum p log p;
+ *  - n > 1: the draw from Cat(p) is the first id whose cumulative p exceeds
+ *    u0 (id order); positions sorted by ascending H (ties to the lower
+ *    position) with C_m the summed and M_m the largest entropy of the first
+ *    m: pi_m keeps its draw when C_m - M_m <= eta, every other generated
+ *    position takes the re-noise token floor(u1 (vocab - 1)); n = 1: every
+ *    generated position takes its argmax;
+ *  - self-conditioning: s = p E (E the embedding table) is added to the
+ *    input embedding of the generated positions at the next step; s = 0 at
+ *    n = T;
+ *  - readings: the initial canvas z_T is the prompt followed by re-noise
+ *    tokens of step T; refresh at step i = T - n when i mod K == 0; the
+ *    anchor pass of a refresh step embeds the same canvas plus s;
+ *  - draws: the ReMDM Philox stream above, (u0, u1, unused) of position
+ *    (b, r) at step i = T - n, and step T for the initial canvas.
+ * Arithmetic: fp32 logits, exponentials and sums; the accepted set from the
+ * fp32 entropies with fp64 partial sums. */
+
+/* One step of Alg. 2 from given logits.  z: device int32 [batch, rows]
+ * (leading dimension ldz); the positions first_gen .. rows-1 (G = rows -
+ * first_gen, 1 <= G <= 16384) are rewritten, the others never change.
+ * logits: device fp32, row b * G + g (stride ld_logits) for position
+ * (b, first_gen + g), read only.  tau > 0 is tau_n; last = 1 for n = 1
+ * (argmax only; entropy, probs and eta unused), else 0.  entropy: device
+ * fp32 [batch * G], written with H (n > 1).  probs (optional, may be NULL):
+ * written with p, row stride ld_probs, fp32 (probs_dtype 0) or bf16 (1).
+ * No allocation; INVALID_ARG for bad sizes, NaN eta or tau <= 0. */
+TADM_API tadm_status tadm_eb_update(int32_t* z, int ldz, const float* logits, int ld_logits, int batch, int rows,
+                                    int first_gen, int vocab, int mask_id, double tau, double eta, int last,
+                                    uint64_t seed, int step, float* entropy, void* probs, int probs_dtype,
+                                    int ld_probs, tadm_stream stream);
+
+/* Bytes of caller scratch that tadm_generate_entropy_bound needs: the
+ * logits of the generated rows (fp32 [batch * gen_len, vocab]), with
+ * self-conditioning p ([batch * gen_len, vocab]) and E^T ([d_model, vocab])
+ * in the model's element type and s (fp32 [batch * gen_len, d_model]), and
+ * the entropies (fp32 [batch * gen_len]); 256-byte aligned segments. */
+TADM_API tadm_status tadm_eb_scratch_bytes(const tadm_handle* h, int batch, int gen_len, int self_cond,
+                                           size_t* bytes);
+
+/* Whole generation with the entropy-bound sampler on one canvas (prompt +
+ * gen_len generated positions, bidirectional; the handle needs max_rows >=
+ * prompt_len + gen_len and no KV context): `steps` = T reverse steps,
+ * anchor refresh every K, eta, tau_max >= tau_min > 0, self_cond 0/1.
+ * scratch: device, 256-byte aligned, at least tadm_eb_scratch_bytes.
+ * out: device int32 [batch, prompt_len + gen_len]. */
+TADM_API tadm_status tadm_generate_entropy_bound(tadm_handle* h, const int32_t* prompt, int batch, int prompt_len,
+                                                 int32_t* out, int gen_len, int steps, int K, double eta,
+                                                 double tau_max, double tau_min, int self_cond, uint64_t seed,
+                                                 void* scratch, size_t scratch_bytes, tadm_stream stream);
+
 #ifdef __cplusplus
 }
 #endif

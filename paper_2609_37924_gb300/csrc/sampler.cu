@@ -503,6 +503,231 @@ __global__ void __launch_bounds__(NT) remdm_sample_smem_kernel(const float* __re
   }
 }
 
+
+// ------------------------------------------------------- entropy-bound sampler
+// Alg. 2 (App. C.1).  The draws reuse the Philox stream above: u0 picks the
+// categorical draw, u1 the re-noise token floor(u1 (V - 1)) of a rejected
+// position; the initial canvas is the re-noise of step T.
+__device__ __forceinline__ int eb_noise_token(uint64_t seed, int step, int B, int R, int b, int r, int vocab) {
+  float u[3];
+  remdm_draws(seed, step, B, R, b, r, u);
+  const uint64_t k = static_cast<uint64_t>(u[1] * 16777216.0f);   // exact: u1 = k * 2^-24
+  return static_cast<int>((k * static_cast<uint64_t>(vocab - 1)) >> 24);
+}
+
+__global__ void eb_noise_kernel(int32_t* __restrict__ z, int ldz, int B, int R, int first, int vocab, uint64_t seed,
+                                int step) {
+  pdl_enter();
+  const int G = R - first;
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= B * G) return;
+  const int b = i / G, r = first + (i - b * G);
+  z[static_cast<size_t>(b) * ldz + r] = eb_noise_token(seed, step, B, R, b, r, vocab);
+}
+
+// idx[b * G + g] = b * R + first + g: the canvas rows of the generated positions
+__global__ void eb_rows_kernel(int32_t* __restrict__ idx, int B, int R, int first) {
+  pdl_enter();
+  const int G = R - first;
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= B * G) return;
+  const int b = i / G;
+  idx[i] = b * R + first + (i - b * G);
+}
+
+// One block per generated position j = b * G + g (canvas row first + g):
+// a_v = (l_v - max) / tau, e_v = exp(a_v) (0 for MASK), Z = sum e_v,
+// W = sum e_v a_v, so p = e / Z and H = -sum p log p = log Z - W / Z
+// (clamped at 0).  The argmax takes the lowest id among equal logits; the
+// draw is the first id whose cumulative e exceeds u0 * Z (each thread owns a
+// contiguous id range: a block scan of the range sums in fixed order, then
+// one thread's walk of its range).  last (n = 1): z takes the argmax and
+// nothing else is written; otherwise z takes the draw, H[j] the entropy and,
+// when p is given, p[j, v] = e_v / Z.  SMEM keeps e in dynamic shared memory
+// (vocab * 4 bytes).
+template <int NT, bool SMEM>
+__global__ void __launch_bounds__(NT) eb_row_kernel(const float* __restrict__ logits, int ld, int G, int first,
+                                                    int32_t* __restrict__ z, int ldz, int B, int R, int vocab,
+                                                    int mask_id, float inv_tau, int last, uint64_t seed, int step,
+                                                    void* __restrict__ p, int p_bf16, int ldp, float* __restrict__ H) {
+  pdl_enter();
+  extern __shared__ float es[];
+  __shared__ float sv[32];
+  __shared__ int si[32];
+  __shared__ float scan[NT];
+  __shared__ int pick;
+  const int j = blockIdx.x, tid = threadIdx.x;
+  const int b = j / G, r = first + (j - b * G);
+  const float* L = logits + static_cast<size_t>(j) * ld;
+  int32_t* zp = z + static_cast<size_t>(b) * ldz + r;
+  float mx = -INFINITY;
+  int am = -1;
+  for (int v = tid; v < vocab; v += NT) {
+    const float l = L[v];
+    if (SMEM) es[v] = l;
+    if (v != mask_id && better(l, v, mx, am)) { mx = l; am = v; }
+  }
+  block_argmax<NT>(mx, am, sv, si);
+  if (last) {
+    if (tid == 0) *zp = am;
+    return;
+  }
+  float Z = 0.0f, W = 0.0f;
+  for (int v = tid; v < vocab; v += NT) {
+    const float a = ((SMEM ? es[v] : L[v]) - mx) * inv_tau;
+    const float e = v == mask_id ? 0.0f : expf(a);
+    if (e > 0.0f) {
+      Z += e;
+      W = fmaf(e, a, W);
+    }
+    if (SMEM) es[v] = e;
+  }
+  Z = block_sum_f<NT>(Z, sv);
+  W = block_sum_f<NT>(W, sv);
+  const float ent0 = logf(Z) - W / Z;
+  const float ent = ent0 > 0.0f ? ent0 : 0.0f;      // rounding below 0 (and -0) -> +0: keys sort by bits
+  auto e_of = [&](int v) -> float {
+    if (SMEM) return es[v];
+    return v == mask_id ? 0.0f : expf((L[v] - mx) * inv_tau);
+  };
+  const int chunk = (vocab + NT - 1) / NT, v0 = tid * chunk, v1 = min(vocab, v0 + chunk);
+  float mine = 0.0f;
+  if (v1 > v0) {                                    // start at lane-rotated ids: no shared-memory bank conflicts
+    int v = SMEM ? v0 + (tid & 31) % (v1 - v0) : v0;
+    for (int k = v0; k < v1; ++k) {
+      mine += e_of(v);
+      if (++v == v1) v = v0;
+    }
+  }
+  __syncthreads();
+  scan[tid] = mine;
+  if (tid == 0) pick = -1;
+  __syncthreads();
+  for (int o = 1; o < NT; o <<= 1) {               // inclusive scan of the range sums (fixed order)
+    const float add = tid >= o ? scan[tid - o] : 0.0f;
+    __syncthreads();
+    scan[tid] += add;
+    __syncthreads();
+  }
+  float u[3];
+  remdm_draws(seed, step, B, R, b, r, u);
+  const float goal = u[0] * scan[NT - 1];
+  const float before = tid > 0 ? scan[tid - 1] : 0.0f;
+  if (mine > 0.0f && before <= goal && goal < scan[tid]) {
+    float c = before;
+    int lastv = -1, got = -1;
+    for (int v = v0; v < v1; ++v) {
+      const float e = e_of(v);
+      if (e > 0.0f) {
+        lastv = v;
+        c += e;
+        if (c > goal) {
+          got = v;
+          break;
+        }
+      }
+    }
+    pick = got >= 0 ? got : lastv;
+  }
+  if (p) {                                          // p = e / Z for the self-conditioning product
+    const float iz = 1.0f / Z;
+    if (p_bf16) {
+      bf16* o = static_cast<bf16*>(p) + static_cast<size_t>(j) * ldp;
+      for (int v = tid; v < vocab; v += NT) o[v] = __float2bfloat16_rn(e_of(v) * iz);
+    } else {
+      float* o = static_cast<float*>(p) + static_cast<size_t>(j) * ldp;
+      for (int v = tid; v < vocab; v += NT) o[v] = e_of(v) * iz;
+    }
+  }
+  __syncthreads();
+  if (tid == 0) {
+    int v = pick;
+    for (int t = NT - 1; t >= 0 && v < 0; --t)     // rounding left the goal past every range: the last token
+      if ((t > 0 ? scan[t] - scan[t - 1] : scan[0]) > 0.0f)
+        for (int w = min(vocab, (t + 1) * chunk) - 1; w >= t * chunk; --w)
+          if (e_of(w) > 0.0f) { v = w; break; }
+    *zp = v < 0 ? am : v;
+    H[j] = ent;
+  }
+}
+
+// One block per sequence: the G entropies sorted ascending (ties to the lower
+// position) as 64-bit keys (H bits, position) by a bitonic sort in shared
+// memory (H >= 0, so the fp32 bit patterns order like the values); C_m of
+// the sorted order by an fp64 block scan; position pi_m keeps its draw when
+// C_m - H_{pi_m} <= eta (H_{pi_m} = M_m in ascending order), otherwise it
+// takes the re-noise token.  keys: n2 = next power of two >= G entries.
+template <int NT>
+__global__ void __launch_bounds__(NT) eb_accept_kernel(const float* __restrict__ H, int G, int n2, int first,
+                                                       int32_t* __restrict__ z, int ldz, int B, int R, int vocab,
+                                                       double eta, uint64_t seed, int step) {
+  pdl_enter();
+  extern __shared__ unsigned long long keys[];
+  __shared__ double part[NT];
+  const int b = blockIdx.x, tid = threadIdx.x;
+  for (int i = tid; i < n2; i += NT)
+    keys[i] = i < G ? (static_cast<unsigned long long>(__float_as_uint(H[static_cast<size_t>(b) * G + i])) << 32) |
+                          static_cast<unsigned>(i)
+                    : ~0ull;
+  __syncthreads();
+  for (int k = 2; k <= n2; k <<= 1)
+    for (int jj = k >> 1; jj > 0; jj >>= 1) {
+      for (int i = tid; i < n2; i += NT) {
+        const int l = i ^ jj;
+        if (l > i) {
+          const unsigned long long a = keys[i], c = keys[l];
+          const bool up = (i & k) == 0;
+          if ((a > c) == up) {
+            keys[i] = c;
+            keys[l] = a;
+          }
+        }
+      }
+      __syncthreads();
+    }
+  const int per = (n2 + NT - 1) / NT, m0 = tid * per, m1 = min(n2, m0 + per);
+  double mine = 0.0;
+  for (int m = m0; m < m1; ++m)
+    if (static_cast<unsigned>(keys[m]) < static_cast<unsigned>(G)) mine += __uint_as_float(keys[m] >> 32);
+  part[tid] = mine;
+  __syncthreads();
+  for (int o = 1; o < NT; o <<= 1) {               // inclusive scan of the range sums
+    const double add = tid >= o ? part[tid - o] : 0.0;
+    __syncthreads();
+    part[tid] += add;
+    __syncthreads();
+  }
+  double c = tid > 0 ? part[tid - 1] : 0.0;
+  for (int m = m0; m < m1; ++m) {
+    const unsigned g = static_cast<unsigned>(keys[m]);
+    if (g >= static_cast<unsigned>(G)) continue;
+    const double h = __uint_as_float(keys[m] >> 32);
+    c += h;
+    if (!(c - h <= eta)) {
+      const int r = first + static_cast<int>(g);
+      z[static_cast<size_t>(b) * ldz + r] = eb_noise_token(seed, step, B, R, b, r, vocab);
+    }
+  }
+}
+
+// E^T: out[c, r] = in[r, c] for a rows x cols matrix (32 x 32 shared tiles;
+// T is the element's bit container: float or uint16_t for bf16)
+template <class T>
+__global__ void transpose_kernel(const T* __restrict__ in, int rows, int cols, T* __restrict__ out) {
+  pdl_enter();
+  __shared__ T t[32][33];
+  const int r0 = blockIdx.x * 32, c0 = blockIdx.y * 32;
+  for (int y = threadIdx.y; y < 32; y += 8) {
+    const int r = r0 + y, c = c0 + threadIdx.x;
+    if (r < rows && c < cols) t[y][threadIdx.x] = in[static_cast<size_t>(r) * cols + c];
+  }
+  __syncthreads();
+  for (int y = threadIdx.y; y < 32; y += 8) {
+    const int c = c0 + y, r = r0 + threadIdx.x;
+    if (r < rows && c < cols) out[static_cast<size_t>(c) * rows + r] = t[threadIdx.x][y];
+  }
+}
+
 }  // namespace
 
 const char* confidence_rows(const float* logits, int rows, int vocab, int ld, int mask_id, float* conf, int32_t* tok,
@@ -571,6 +796,77 @@ const char* remdm_sample(const float* logits, int ld, int n_rows, const int32_t*
 
 const char* remdm_rows(const int32_t* act, int n, int bound, int32_t* idx, int* count, cudaStream_t s) {
   launch_pdl(remdm_rows_kernel, 1, 1024, 0, s, act, n, bound, idx, count);
+  return err();
+}
+
+const char* eb_noise(int32_t* z, int ldz, int B, int R, int first, int vocab, uint64_t seed, int step, cudaStream_t s) {
+  const int n = B * (R - first);
+  if (n <= 0) return nullptr;
+  launch_pdl(eb_noise_kernel, (n + 255) / 256, 256, 0, s, z, ldz, B, R, first, vocab, seed, step);
+  return err();
+}
+
+const char* eb_rows(int32_t* idx, int B, int R, int first, cudaStream_t s) {
+  const int n = B * (R - first);
+  if (n <= 0) return nullptr;
+  launch_pdl(eb_rows_kernel, (n + 255) / 256, 256, 0, s, idx, B, R, first);
+  return err();
+}
+
+const char* eb_row(const float* logits, int ld, int B, int R, int first, int32_t* z, int ldz, int vocab, int mask_id,
+                   float inv_tau, int last, uint64_t seed, int step, void* p, int p_bf16, int ldp, float* H,
+                   cudaStream_t s) {
+  const int G = R - first, n = B * G;
+  if (n <= 0) return nullptr;
+  const size_t smem = static_cast<size_t>(vocab) * sizeof(float);
+  if (smem <= 200u * 1024u) {   // the row's exponentials fit in shared memory
+    static bool attr = false;
+    if (!attr) {
+      if (cudaFuncSetAttribute(eb_row_kernel<1024, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024) !=
+          cudaSuccess)
+        return "entropy-bound sampler smem attribute failed";
+      attr = true;
+    }
+    launch_pdl(eb_row_kernel<1024, true>, n, 1024, smem, s, logits, ld, G, first, z, ldz, B, R, vocab, mask_id,
+               inv_tau, last, seed, step, p, p_bf16, ldp, H);
+  } else {
+    launch_pdl(eb_row_kernel<512, false>, n, 512, 0, s, logits, ld, G, first, z, ldz, B, R, vocab, mask_id, inv_tau,
+               last, seed, step, p, p_bf16, ldp, H);
+  }
+  return err();
+}
+
+int eb_max_gen() { return 16384; }
+
+const char* eb_accept(const float* H, int B, int R, int first, int32_t* z, int ldz, int vocab, double eta,
+                      uint64_t seed, int step, cudaStream_t s) {
+  const int G = R - first;
+  if (B <= 0 || G <= 0) return nullptr;
+  if (G > eb_max_gen()) return "entropy-bound sampler: more than 16384 generated positions per sequence";
+  int n2 = 1;
+  while (n2 < G) n2 <<= 1;
+  static bool attr = false;
+  if (!attr) {
+    if (cudaFuncSetAttribute(eb_accept_kernel<1024>, cudaFuncAttributeMaxDynamicSharedMemorySize, 16384 * 8) !=
+        cudaSuccess)
+      return "entropy-bound accept smem attribute failed";
+    attr = true;
+  }
+  launch_pdl(eb_accept_kernel<1024>, B, 1024, static_cast<size_t>(n2) * 8, s, H, G, n2, first, z, ldz, B, R, vocab,
+             eta, seed, step);
+  return err();
+}
+
+const char* transpose(const void* in, int rows, int cols, int bf16, void* out, cudaStream_t s) {
+  if (rows <= 0 || cols <= 0) return nullptr;
+  if ((cols + 31) / 32 > 65535) return "transpose: too many columns";
+  const dim3 grid((rows + 31) / 32, (cols + 31) / 32), block(32, 8);
+  if (bf16)
+    launch_pdl(transpose_kernel<uint16_t>, grid, block, 0, s, static_cast<const uint16_t*>(in), rows, cols,
+               static_cast<uint16_t*>(out));
+  else
+    launch_pdl(transpose_kernel<float>, grid, block, 0, s, static_cast<const float*>(in), rows, cols,
+               static_cast<float*>(out));
   return err();
 }
 

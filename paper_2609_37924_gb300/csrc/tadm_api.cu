@@ -387,10 +387,13 @@ tadm_status stack_fwd(tadm_handle* h, int first, int n, float* x, int B, int R, 
 }
 
 // S: c = embed(z) then L_S layers (c lives in the workspace).
-tadm_status run_S(tadm_handle* h, const int32_t* z, int ldz, int B, int R, int causal, cudaStream_t s) {
+// `add` (optional): the self-conditioning signal of rows add_first .. R-1 of
+// each sequence, fp32 [B * (R - add_first), d], added to their embedding.
+tadm_status run_S(tadm_handle* h, const int32_t* z, int ldz, int B, int R, int causal, cudaStream_t s,
+                  const float* add = nullptr, int add_first = 0) {
   const tadm_config& c = h->cfg;
   float* cbuf = h->at<float>(h->off.c);
-  TRY(embed_rows(z, ldz, B, R, h->embed, c.dtype, c.d_model, c.vocab, cbuf, nullptr, s));
+  TRY(embed_rows(z, ldz, B, R, h->embed, c.dtype, c.d_model, c.vocab, cbuf, nullptr, s, add, add_first));
   return stack_fwd(h, 0, c.n_shared, cbuf, B, R, h->ctx, causal, s);
 }
 
@@ -1248,6 +1251,151 @@ tadm_status tadm_generate_remdm(tadm_handle* h, const int32_t* prompt, int batch
     TRYS(gemm(h, norm, Mmax, c.d_model, h->lm_head, c.d_model, bound, c.vocab, c.d_model, EPI_LMHEAD, e, s, false, cnt));
     TRY(remdm_sample(logits_scratch, c.vocab, bound, idx, act, out, total, batch, R, c.vocab, mask, top_p, seed, n, s,
                      cnt));
+    h->counters.shared_layers += c.n_shared;
+    h->counters.denoise_layers += c.n_denoise;
+    h->counters.denoise_steps += 1;
+  }
+  return TADM_OK;
+}
+
+}  // extern "C"
+
+// ------------------------------------------------------------ entropy-bound sampler
+namespace {
+
+// Caller scratch of the entropy-bound generation, in this order (each
+// segment 256-byte aligned): logits fp32 [n, V]; p [n, V] and E^T [d, V]
+// (model element type) and s fp32 [n, d] when self-conditioning; H fp32 [n];
+// n = batch * gen_len.
+struct EbScratch {
+  size_t logits, p, et, sig, ent, total;
+};
+
+EbScratch eb_layout(const tadm_config& c, int batch, int gen_len, int self_cond) {
+  const size_t n = static_cast<size_t>(batch) * gen_len, es = c.dtype ? 2 : 4;
+  EbScratch L{};
+  size_t o = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = o;
+    o = align_up(o + bytes, 256);
+    return at;
+  };
+  L.logits = take(n * c.vocab * 4);
+  if (self_cond) {
+    L.p = take(n * c.vocab * es);
+    L.et = take(static_cast<size_t>(c.d_model) * c.vocab * es);
+    L.sig = take(n * c.d_model * 4);
+  }
+  L.ent = take(n * 4);
+  L.total = o;
+  return L;
+}
+
+const char* eb_args_error(int steps, int K, double eta, double tau_max, double tau_min, int self_cond) {
+  if (steps < 1 || K < 1) return "need steps >= 1 and K >= 1";
+  if (eta != eta) return "eta is NaN";
+  if (!(tau_min > 0.0) || !(tau_max >= tau_min) || !(tau_max < 1e30)) return "need 0 < tau_min <= tau_max";
+  if (self_cond != 0 && self_cond != 1) return "self_cond must be 0 or 1";
+  return nullptr;
+}
+
+}  // namespace
+
+extern "C" {
+
+tadm_status tadm_eb_update(int32_t* z, int ldz, const float* logits, int ld_logits, int batch, int rows, int first_gen,
+                           int vocab, int mask_id, double tau, double eta, int last, uint64_t seed, int step,
+                           float* entropy, void* probs, int probs_dtype, int ld_probs, tadm_stream stream) {
+  const int G = rows - first_gen;
+  if (!z || !logits || batch <= 0 || rows <= 0 || first_gen < 0 || G <= 0 || ldz < rows || vocab < 2 ||
+      ld_logits < vocab || mask_id < 0 || mask_id >= vocab || step < 0 || !(tau > 0.0) || eta != eta ||
+      (last != 0 && last != 1) || (!last && !entropy) || (probs && ld_probs < vocab) ||
+      (probs_dtype != 0 && probs_dtype != 1) || G > eb_max_gen())
+    return TADM_ERR_INVALID_ARG;
+  cudaStream_t s = stream;
+  if (eb_row(logits, ld_logits, batch, rows, first_gen, z, ldz, vocab, mask_id, static_cast<float>(1.0 / tau), last,
+             seed, step, last ? nullptr : probs, probs_dtype, ld_probs, entropy, s))
+    return TADM_ERR_CUDA;
+  if (!last && eb_accept(entropy, batch, rows, first_gen, z, ldz, vocab, eta, seed, step, s)) return TADM_ERR_CUDA;
+  return TADM_OK;
+}
+
+tadm_status tadm_eb_scratch_bytes(const tadm_handle* h, int batch, int gen_len, int self_cond, size_t* bytes) {
+  if (!h || !bytes || batch <= 0 || gen_len <= 0 || (self_cond != 0 && self_cond != 1)) return TADM_ERR_INVALID_ARG;
+  *bytes = eb_layout(h->cfg, batch, gen_len, self_cond).total;
+  return TADM_OK;
+}
+
+tadm_status tadm_generate_entropy_bound(tadm_handle* h, const int32_t* prompt, int batch, int prompt_len,
+                                        int32_t* out, int gen_len, int steps, int K, double eta, double tau_max,
+                                        double tau_min, int self_cond, uint64_t seed, void* scratch,
+                                        size_t scratch_bytes, tadm_stream stream) {
+  if (!h) return TADM_ERR_INVALID_ARG;
+  if (const char* e = eb_args_error(steps, K, eta, tau_max, tau_min, self_cond))
+    return fail(h, TADM_ERR_INVALID_ARG, "%s", e);
+  if (!prompt || !out || !scratch) return fail(h, TADM_ERR_INVALID_ARG, "NULL pointer");
+  if (prompt_len < 0 || gen_len <= 0 || gen_len > eb_max_gen())
+    return fail(h, TADM_ERR_INVALID_ARG, "need 0 < gen_len <= %d", eb_max_gen());
+  if (h->max_ctx > 0)
+    return fail(h, TADM_ERR_INVALID_ARG, "the entropy-bound sampler runs single-block canvases (max_ctx = 0)");
+  const tadm_config& c = h->cfg;
+  if (self_cond && c.dtype && c.vocab % 8)
+    return fail(h, TADM_ERR_INVALID_ARG, "self-conditioning on a bf16 model needs vocab % 8 == 0");
+  const EbScratch L = eb_layout(c, batch, gen_len, self_cond);
+  if (scratch_bytes < L.total || reinterpret_cast<uintptr_t>(scratch) % 256)
+    return fail(h, TADM_ERR_INVALID_ARG, "scratch needs %zu bytes, 256-byte aligned", L.total);
+  const int total = prompt_len + gen_len, R = total, n_rows = batch * gen_len;
+  TRYS(tadm_reset(h, batch));
+  TRYS(check_ready(h, batch, R));
+  h->last_stream = stream;
+  cudaStream_t s = stream;
+  const int mask = c.vocab - 1;
+  char* base = static_cast<char*>(scratch);
+  float* logits = reinterpret_cast<float*>(base + L.logits);
+  float* ent = reinterpret_cast<float*>(base + L.ent);
+  void* p = self_cond ? base + L.p : nullptr;
+  void* et = self_cond ? base + L.et : nullptr;
+  float* sig = self_cond ? reinterpret_cast<float*>(base + L.sig) : nullptr;
+  int32_t* idx = h->at<int32_t>(h->off.idx);
+  const int64_t Mmax = static_cast<int64_t>(h->max_batch) * h->max_rows;
+  if (self_cond) TRY(transpose(h->embed, c.vocab, c.d_model, c.dtype, et, s));   // E^T [d, V] for s = p E
+  TRY(fill_canvas(out, total, prompt, batch, prompt_len, total, mask, s));
+  TRY(eb_noise(out, total, batch, R, prompt_len, c.vocab, seed, steps, s));       // z_T: noise of step T
+  TRY(eb_rows(idx, batch, R, prompt_len, s));
+  void* cache = h->at(h->off.h_int);
+  for (int i = 0; i < steps; ++i) {
+    const int n = steps - i;                      // Alg. 2's n = T .. 1
+    TRYS(run_S(h, out, total, batch, R, 0, s, self_cond && i > 0 ? sig : nullptr, prompt_len));
+    if (i % K == 0) {                             // Alg. 1 refresh test (T - i) mod K = 0
+      TRYS(run_A(h, batch, R, 0, cache, s));
+      h->counters.anchor_layers += c.n_anchor;
+      h->counters.anchor_calls += 1;
+    }
+    TRYS(run_fusion(h, batch, R, cache, s));
+    float* x = h->at<float>(h->off.x);
+    TRYS(stack_fwd(h, c.n_shared + c.n_anchor, c.n_denoise, x, batch, R, 0, 0, s));
+    void* norm = h->at(h->off.norm);
+    TRY(rmsnorm_rows(x, n_rows, c.d_model, h->final_norm, c.dtype, c.norm_eps, norm, c.d_model, h->act_bf16(), s,
+                     idx));
+    EpiParams e{};
+    e.part = h->at<float>(h->off.part);
+    e.mask_id = mask;
+    e.logits = logits;
+    e.ld_logits = c.vocab;
+    TRYS(gemm(h, norm, Mmax, c.d_model, h->lm_head, c.d_model, n_rows, c.vocab, c.d_model, EPI_LMHEAD, e, s));
+    const double tau = tau_min + (tau_max - tau_min) * n / steps;
+    const int last = n == 1;
+    TRY(eb_row(logits, c.vocab, batch, R, prompt_len, out, total, c.vocab, mask, static_cast<float>(1.0 / tau), last,
+               seed, i, last ? nullptr : p, c.dtype, c.vocab, ent, s));
+    if (!last) {
+      if (self_cond) {                            // s = p E for the next step's embedding
+        EpiParams es{};
+        es.out = sig;
+        es.ldo = c.d_model;
+        TRYS(gemm(h, p, n_rows, c.vocab, et, c.vocab, n_rows, c.d_model, c.vocab, EPI_STORE, es, s, true));
+      }
+      TRY(eb_accept(ent, batch, R, prompt_len, out, total, c.vocab, eta, seed, i, s));
+    }
     h->counters.shared_layers += c.n_shared;
     h->counters.denoise_layers += c.n_denoise;
     h->counters.denoise_steps += 1;

@@ -25,6 +25,7 @@ ABI_FUNCTIONS = [
     "tadm_topk_unmask", "tadm_attention", "tadm_probe_enable", "tadm_probe_read", "tadm_head_scratch_size",
     "tadm_head_confidence", "tadm_head_confidence_static", "tadm_probe_breakdown",
     "tadm_remdm_schedule", "tadm_remdm_uniforms", "tadm_remdm_update", "tadm_generate_remdm",
+    "tadm_eb_update", "tadm_eb_scratch_bytes", "tadm_generate_entropy_bound",
 ]
 
 
@@ -104,6 +105,9 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
                                   ctypes.c_uint64, I, P, P]),
         "tadm_generate_remdm": (I, [P, P, I, I, P, I, I, I, I, ctypes.c_double, ctypes.c_float, ctypes.c_uint64, P,
                                     SZ, P]),
+        "tadm_eb_update": (I, [P, I, P, I, I, I, I, I, I, ctypes.c_double, ctypes.c_double, I, ctypes.c_uint64, I, P, P, I, I, P]),
+        "tadm_eb_scratch_bytes": (I, [P, I, I, I, ctypes.POINTER(SZ)]),
+        "tadm_generate_entropy_bound": (I, [P, P, I, I, P, I, I, I, ctypes.c_double, ctypes.c_double, ctypes.c_double, I, ctypes.c_uint64, P, SZ, P]),
         "tadm_probe_breakdown": (I, [P, I, ctypes.POINTER(I64), ctypes.POINTER(ctypes.c_double),
                                      ctypes.POINTER(ctypes.c_double)]),
         "tadm_probe_read": (I, [P, ctypes.POINTER(I64), ctypes.POINTER(ctypes.c_double),
@@ -249,6 +253,22 @@ def tadm_remdm_update(z, logits, first_gen: int, mask_id: int, sigma: float, p_u
                                             _stream(stream)))
 
 
+
+def tadm_eb_update(z, logits, first_gen: int, mask_id: int, tau: float, eta: float, last: bool, seed: int,
+                   step: int, entropy, probs=None, stream=None):
+    """One entropy-bound step (Alg. 2) on z [batch, rows] from the logits of
+    the generated positions [batch * (rows - first_gen), vocab]; entropy
+    [batch * (rows - first_gen)] fp32; probs optional (fp32 or bf16)."""
+    batch, rows = z.shape
+    vocab = logits.shape[1]
+    p_dtype = 0
+    if probs is not None:
+        p_dtype = {"torch.float32": 0, "torch.bfloat16": 1}[str(probs.dtype)]
+    _check(load_library().tadm_eb_update(_ptr(z), rows, _ptr(logits), vocab, batch, rows, first_gen, vocab, mask_id,
+                                         tau, eta, int(bool(last)), seed, step, _ptr(entropy),
+                                         _ptr(probs) if probs is not None else None, p_dtype,
+                                         probs.shape[1] if probs is not None else 0, _stream(stream)))
+
 # ---------------------------------------------------------------------------- model handle
 class TadmModel:
     """A handle plus its torch-allocated workspace.
@@ -339,6 +359,22 @@ class TadmModel:
                                             REMDM_KINDS[kind], eta, top_p, seed, _ptr(logits_scratch),
                                             logits_scratch.numel() * logits_scratch.element_size(),
                                             _stream(stream)), self.h)
+
+    def tadm_eb_scratch_bytes(self, batch: int, gen_len: int, self_cond: bool = True) -> int:
+        out = ctypes.c_size_t(0)
+        _check(self.lib.tadm_eb_scratch_bytes(self.h, batch, gen_len, int(bool(self_cond)), ctypes.byref(out)), self.h)
+        return out.value
+
+    def tadm_generate_entropy_bound(self, prompt, out, gen_len: int, steps: int, K: int, eta: float,
+                                    tau_max: float, tau_min: float, seed: int, scratch, self_cond: bool = True,
+                                    stream=None):
+        """Alg. 2 generation; scratch: a device buffer of at least
+        tadm_eb_scratch_bytes(batch, gen_len, self_cond) bytes."""
+        B, P = prompt.shape
+        _check(self.lib.tadm_generate_entropy_bound(self.h, _ptr(prompt), B, P, _ptr(out), gen_len, steps, K, eta,
+                                                    tau_max, tau_min, int(bool(self_cond)), seed, _ptr(scratch),
+                                                    scratch.numel() * scratch.element_size(), _stream(stream)),
+               self.h)
 
     def tadm_sync_status(self):
         _check(self.lib.tadm_sync_status(self.h), self.h)

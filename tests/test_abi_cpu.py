@@ -128,3 +128,23 @@ def test_remdm_arguments_are_rejected(lib):
         assert so.tadm_remdm_schedule(*args, out) == 1, args
     # null buffers / out-of-range probabilities fail before any launch
     assert so.tadm_remdm_update(None, 4, None, 8, 1, 4, 0, 8, 7, 0.1, 0.1, 0.9, 1, 0, None, None) == 1
+
+
+def test_entropy_bound_arguments_are_rejected(lib):
+    """tadm_eb_update checks its arguments before any launch (the pointers
+    below are never dereferenced)."""
+    so = lib.load_library()
+    fake = ctypes.c_void_p(256)
+    good = dict(z=fake, ldz=8, logits=fake, ld=16, batch=2, rows=8, first=3, vocab=16, mask=15, tau=0.6, eta=0.1,
+                last=0, seed=1, step=0, ent=fake, probs=None, pd=0, ldp=0)
+    bad = [dict(z=None), dict(logits=None), dict(first=8), dict(first=-1), dict(ldz=7), dict(ld=15), dict(mask=16),
+           dict(tau=0.0), dict(tau=-1.0), dict(eta=float("nan")), dict(last=2), dict(ent=None), dict(step=-1),
+           dict(probs=fake, ldp=15), dict(probs=fake, ldp=16, pd=2), dict(rows=20000, ldz=20000, first=0)]
+    for over in bad:
+        a = {**good, **over}
+        st = so.tadm_eb_update(a["z"], a["ldz"], a["logits"], a["ld"], a["batch"], a["rows"], a["first"], a["vocab"],
+                               a["mask"], a["tau"], a["eta"], a["last"], a["seed"], a["step"], a["ent"], a["probs"],
+                               a["pd"], a["ldp"], None)
+        assert st == 1, over
+    size = ctypes.c_size_t()
+    assert so.tadm_eb_scratch_bytes(None, 1, 1, 1, ctypes.byref(size)) == 1
