@@ -46,8 +46,9 @@ def parse():
                     help="override reverse steps per block (short runs for launch-list profiles)")
     ap.add_argument("--G", type=int, default=None, help="override the generation length (short profiling runs)")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
-    ap.add_argument("--sampler", default="topk", choices=["topk", "remdm-cap", "remdm-loop"],
-                    help="with --sweep-workloads: the confidence top-k sampler or ReMDM (App. C.2 settings)")
+    ap.add_argument("--sampler", default="topk", choices=["topk", "remdm-cap", "remdm-loop", "entropy-bound"],
+                    help="with --sweep-workloads: the confidence top-k sampler, ReMDM (App. C.2 settings) or the "
+                         "entropy-bound sampler with self-conditioning (App. C.1 settings)")
     ap.add_argument("--fusion-off", action="store_true",
                     help="with --sweep-workloads: run the workloads with the fusion disabled (App. D naive reuse)")
     ap.add_argument("--sweep-workloads", default=None,
@@ -379,6 +380,16 @@ def kernel_bench(args):
         o = torch.empty((B * R, H * hd), device="cuda", dtype=torch.bfloat16)
         run = lambda: tadm.tadm_attention(q, k, v, o, H, Hkv, R, 0, False, dtype=1)  # noqa: E731
         flops = 4.0 * B * H * R * R * hd
+    elif kind == "ebrow":
+        # ebrow:rows,V  one entropy-bound sampler step (Alg. 2) on fp32 logits of `rows` positions of one
+        # sequence: per-position softmax/entropy/draw with p written as bf16, then the accept kernel
+        rows, V = (int(x) for x in shape.split(","))
+        logits = torch.randn((rows, V), device="cuda", generator=g) * 3.0
+        z = torch.zeros((1, rows), dtype=torch.int32, device="cuda")
+        ent = torch.empty(rows, dtype=torch.float32, device="cuda")
+        probs = torch.empty((rows, V), dtype=torch.bfloat16, device="cuda")
+        run = lambda: tadm.tadm_eb_update(z, logits, 0, V - 1, 0.6, 0.1, False, 1, 0, ent, probs)  # noqa: E731
+        flops = 0.0
     else:
         M, N, K = (int(x) for x in shape.split(","))
         A = torch.randn((M, K), device="cuda", generator=g).to(torch.bfloat16)
@@ -399,6 +410,9 @@ def kernel_bench(args):
     line = {"kernel": kind, "shape": shape, "ms": ms, "tflops": flops / (ms / 1000.0) / 1e12}
     if kind == "attnctx":   # K and V bytes read once per launch
         line["kv_gbs"] = 2 * k.numel() * (ctx + R) / stride * 2 / (ms / 1000.0) / 1e9
+    if kind == "ebrow":     # algorithmic bytes: the fp32 logits read once, p written once as bf16
+        line["gbs"] = rows * V * (4 + 2) / (ms / 1000.0) / 1e9
+        del line["tflops"]
     print(json.dumps(line), flush=True)
 
 
@@ -438,14 +452,24 @@ def workload_sweep(args):
                 scratch = torch.empty((B * w.gen_len, m.vocab), dtype=torch.float32, device="cuda")
                 kind = args.sampler.split("-")[1]
                 eta = 0.04 if kind == "cap" else 0.02
+            ebs = args.sampler == "entropy-bound"
+            if ebs:     # App. C.1: eta 0.1, tau 0.8 -> 0.4, self-conditioning on
+                if bl:
+                    raise SystemExit("the entropy-bound sampler runs single-block workloads")
+                scratch = torch.empty(tm.tadm_eb_scratch_bytes(B, w.gen_len, True), dtype=torch.uint8,
+                                      device="cuda")
 
             def gen(K):
-                if remdm:
+                if ebs:
+                    tm.tadm_generate_entropy_bound(p, out, w.gen_len, w.steps_per_block, K, 0.1, 0.8, 0.4, 1234,
+                                                   scratch, True)
+                elif remdm:
                     tm.tadm_generate_remdm(p, out, w.gen_len, w.steps_per_block, K, kind, eta, 0.9, 1234, scratch)
                 else:
                     tm.tadm_generate(p, out, w.gen_len, w.steps_per_block, K, bl)
             for K in (w.k_sweep or (w.K,)):
-                for _ in range(max(2, args.warmup)):   # the second identical call captures the CUDA graph
+                # the second identical top-k call captures the CUDA graph; the other samplers run eagerly
+                for _ in range(max(2 if args.sampler == "topk" else 1, args.warmup)):
                     gen(K)
                 tm.tadm_sync_status()
                 e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)

@@ -403,18 +403,22 @@ TADM_API tadm_status tadm_generate_remdm(tadm_handle* h, const int32_t* prompt, 
  * (b, first_gen + g), read only.  tau > 0 is tau_n; last = 1 for n = 1
  * (argmax only; entropy, probs and eta unused), else 0.  entropy: device
  * fp32 [batch * G], written with H (n > 1).  probs (optional, may be NULL):
- * written with p, row stride ld_probs, fp32 (probs_dtype 0) or bf16 (1).
- * No allocation; INVALID_ARG for bad sizes, NaN eta or tau <= 0. */
+ * written with q = exp((L - max) / tau) (0 for MASK), row stride ld_probs,
+ * fp32 (probs_dtype 0) or bf16 (1); z_sum (optional): fp32 [batch * G],
+ * written with Z = sum q, so that p = q / Z.  No allocation; INVALID_ARG for
+ * bad sizes, NaN eta or tau <= 0. */
 TADM_API tadm_status tadm_eb_update(int32_t* z, int ldz, const float* logits, int ld_logits, int batch, int rows,
                                     int first_gen, int vocab, int mask_id, double tau, double eta, int last,
                                     uint64_t seed, int step, float* entropy, void* probs, int probs_dtype,
-                                    int ld_probs, tadm_stream stream);
+                                    int ld_probs, float* z_sum, tadm_stream stream);
 
 /* Bytes of caller scratch that tadm_generate_entropy_bound needs: the
  * logits of the generated rows (fp32 [batch * gen_len, vocab]), with
- * self-conditioning p ([batch * gen_len, vocab]) and E^T ([d_model, vocab])
- * in the model's element type and s (fp32 [batch * gen_len, d_model]), and
- * the entropies (fp32 [batch * gen_len]); 256-byte aligned segments. */
+ * self-conditioning q ([batch * gen_len, vocab]) and E^T ([d_model, vocab])
+ * in the model's element type, q E (fp32 [batch * gen_len, d_model]) and Z
+ * (fp32 [batch * gen_len]), and the entropies (fp32 [batch * gen_len]);
+ * 256-byte aligned segments.  The self-conditioning signal s = p E is
+ * applied as (q E) / Z in the next step's embedding. */
 TADM_API tadm_status tadm_eb_scratch_bytes(const tadm_handle* h, int batch, int gen_len, int self_cond,
                                            size_t* bytes);
 

@@ -68,10 +68,11 @@ const char* attention(const AttnCall& a, cudaStream_t s);
 
 // row kernels (act = bf16 when act_bf16 else fp32)
 // out (and out2) = E[z]; with `add`, rows r >= add_first of sequence b also add
-// add[(b * (rows - add_first) + r - add_first) * d ..] (the self-conditioning signal)
+// add[a * d ..] / add_div[a] (add_div optional), a = b * (rows - add_first) + r - add_first
+// (the self-conditioning signal)
 const char* embed_rows(const int32_t* z, int ldz, int batch, int rows, const void* E, int e_bf16, int d,
                        int vocab, float* out, float* out2, cudaStream_t s, const float* add = nullptr,
-                       int add_first = 0);
+                       int add_first = 0, const float* add_div = nullptr);
 const char* rmsnorm_rows(const float* x, int M, int d, const void* gain, int w_bf16, float eps, void* out,
                          int ldo, int act_bf16, cudaStream_t s, const int32_t* rows_idx = nullptr);
 // per sequence: the rows still holding MASK (first `per_seq` of them, in order) -> idx[b * per_seq + j]
@@ -113,9 +114,11 @@ const char* topk_unmask(int32_t* z, int ldz, const float* conf, const int32_t* t
 // entropy-bound sampler (Alg. 2): the generated positions first .. R-1 of each sequence
 const char* eb_noise(int32_t* z, int ldz, int B, int R, int first, int vocab, uint64_t seed, int step, cudaStream_t s);
 const char* eb_rows(int32_t* idx, int B, int R, int first, cudaStream_t s);
+// part (optional): the output head's [rows][n_tiles][3] partials of these logits (max and argmax from them);
+// q (optional): exp((l - max) / tau) per id; H: entropies; Zs (optional): Z = sum q per row
 const char* eb_row(const float* logits, int ld, int B, int R, int first, int32_t* z, int ldz, int vocab, int mask_id,
-                   float inv_tau, int last, uint64_t seed, int step, void* p, int p_bf16, int ldp, float* H,
-                   cudaStream_t s);
+                   float inv_tau, int last, uint64_t seed, int step, const float* part, int n_tiles, void* q,
+                   int q_bf16, int ldq, float* H, float* Zs, cudaStream_t s);
 int eb_max_gen();
 const char* eb_accept(const float* H, int B, int R, int first, int32_t* z, int ldz, int vocab, double eta,
                       uint64_t seed, int step, cudaStream_t s);

@@ -37,7 +37,7 @@ __device__ __forceinline__ float ldw(const void* w, int bf, int i) {
 
 __global__ void embed_kernel(const int32_t* __restrict__ z, int ldz, int rows, int M, const void* __restrict__ E,
                              int e_bf16, int d, int vocab, float* __restrict__ out, float* __restrict__ out2,
-                             const float* __restrict__ add, int add_first) {
+                             const float* __restrict__ add, int add_first, const float* __restrict__ add_div) {
   pdl_enter();
   const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (m >= M) return;
@@ -46,17 +46,17 @@ __global__ void embed_kernel(const int32_t* __restrict__ z, int ldz, int rows, i
   tok = tok < 0 ? 0 : (tok >= vocab ? vocab - 1 : tok);  // ids are validated by the caller; never read outside E
   float* o = out + static_cast<size_t>(m) * d;
   float* o2 = out2 ? out2 + static_cast<size_t>(m) * d : nullptr;
-  const float* a = add && r >= add_first
-                       ? add + (static_cast<size_t>(b) * (rows - add_first) + (r - add_first)) * d
-                       : nullptr;
+  const size_t ar = static_cast<size_t>(b) * (rows - add_first) + (r - add_first);
+  const float* a = add && r >= add_first ? add + ar * d : nullptr;
+  const float sc = a && add_div ? 1.0f / add_div[ar] : 1.0f;
   if (e_bf16) {
     const bf16* e = static_cast<const bf16*>(E) + static_cast<size_t>(tok) * d;
     for (int j = lane * 2; j < d; j += 64) {
       float2 v = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(e + j));
       if (a) {
         const float2 t = *reinterpret_cast<const float2*>(a + j);
-        v.x += t.x;
-        v.y += t.y;
+        v.x = fmaf(t.x, sc, v.x);
+        v.y = fmaf(t.y, sc, v.y);
       }
       *reinterpret_cast<float2*>(o + j) = v;
       if (o2) *reinterpret_cast<float2*>(o2 + j) = v;
@@ -67,10 +67,10 @@ __global__ void embed_kernel(const int32_t* __restrict__ z, int ldz, int rows, i
       float4 v = *reinterpret_cast<const float4*>(e + j);
       if (a) {
         const float4 t = *reinterpret_cast<const float4*>(a + j);
-        v.x += t.x;
-        v.y += t.y;
-        v.z += t.z;
-        v.w += t.w;
+        v.x = fmaf(t.x, sc, v.x);
+        v.y = fmaf(t.y, sc, v.y);
+        v.z = fmaf(t.z, sc, v.z);
+        v.w = fmaf(t.w, sc, v.w);
       }
       *reinterpret_cast<float4*>(o + j) = v;
       if (o2) *reinterpret_cast<float4*>(o2 + j) = v;
@@ -312,13 +312,14 @@ inline const char* err() {
 }  // namespace
 
 const char* embed_rows(const int32_t* z, int ldz, int batch, int rows, const void* E, int e_bf16, int d, int vocab,
-                       float* out, float* out2, cudaStream_t s, const float* add, int add_first) {
+                       float* out, float* out2, cudaStream_t s, const float* add, int add_first,
+                       const float* add_div) {
   const int M = batch * rows;
   if (M <= 0) return nullptr;
   if (d % 4) return "d_model must be a multiple of 4";
   if (add && (add_first < 0 || add_first > rows)) return "self-conditioning rows out of range";
   launch_pdl(embed_kernel, rows_grid(M), WPB * 32, 0, s, z, ldz, rows, M, E, e_bf16, d, vocab, out, out2, add,
-             add_first);
+             add_first, add_div);
   return err();
 }
 

@@ -535,119 +535,225 @@ __global__ void eb_rows_kernel(int32_t* __restrict__ idx, int B, int R, int firs
   idx[i] = b * R + first + (i - b * G);
 }
 
-// One block per generated position j = b * G + g (canvas row first + g):
-// a_v = (l_v - max) / tau, e_v = exp(a_v) (0 for MASK), Z = sum e_v,
-// W = sum e_v a_v, so p = e / Z and H = -sum p log p = log Z - W / Z
-// (clamped at 0).  The argmax takes the lowest id among equal logits; the
-// draw is the first id whose cumulative e exceeds u0 * Z (each thread owns a
-// contiguous id range: a block scan of the range sums in fixed order, then
-// one thread's walk of its range).  last (n = 1): z takes the argmax and
-// nothing else is written; otherwise z takes the draw, H[j] the entropy and,
-// when p is given, p[j, v] = e_v / Z.  SMEM keeps e in dynamic shared memory
-// (vocab * 4 bytes).
-template <int NT, bool SMEM>
+// One block per generated position j = b * G + g (canvas row first + g) of
+// Alg. 2's step, reading the fp32 logits once:
+//  - the row max and argmax (lowest id among equal logits, MASK excluded)
+//    come from the output head's per-tile partials when `part` is given
+//    (the same fp32 values the head wrote as logits), else from a first
+//    pass over the row; last (n = 1): z takes the argmax, nothing else runs;
+//  - each warp owns a contiguous segment of the row and sums, with
+//    coalesced vector loads, e_v = exp(a_v), a_v = (l_v - max) / tau (0 for
+//    MASK), into Z and W = sum e_v a_v; q[j, v] = e_v is written when q is
+//    given (p = q / Z); H = log Z - W / Z (clamped at +0);
+//  - the draw, the first id whose cumulative e exceeds u0 Z: the segment
+//    holding it from the warps' sums in order, then one block-wide re-read
+//    of that segment (each thread a contiguous sub-range, a block scan, one
+//    thread's walk);
+//  - outputs: z (the draw), H[j], Zs[j] = Z (optional).
+// VEC = 4: float4 loads (vocab, ld, ldq multiples of 4, 16-byte aligned rows).
+template <int NT, int VEC>
 __global__ void __launch_bounds__(NT) eb_row_kernel(const float* __restrict__ logits, int ld, int G, int first,
                                                     int32_t* __restrict__ z, int ldz, int B, int R, int vocab,
                                                     int mask_id, float inv_tau, int last, uint64_t seed, int step,
-                                                    void* __restrict__ p, int p_bf16, int ldp, float* __restrict__ H) {
+                                                    const float* __restrict__ part, int n_tiles,
+                                                    void* __restrict__ q, int q_bf16, int ldq,
+                                                    float* __restrict__ H, float* __restrict__ Zs) {
   pdl_enter();
-  extern __shared__ float es[];
-  __shared__ float sv[32];
-  __shared__ int si[32];
-  __shared__ float scan[NT];
-  __shared__ int pick;
-  const int j = blockIdx.x, tid = threadIdx.x;
+  constexpr int NW = NT / 32, U = 4;
+  __shared__ float sv[32], segZ[NW], segW[NW], wsc[NW];
+  __shared__ int si[32], sh_seg, sh_pick, sh_last;
+  __shared__ float sh_goal;
+  const int j = blockIdx.x, tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
   const int b = j / G, r = first + (j - b * G);
   const float* L = logits + static_cast<size_t>(j) * ld;
   int32_t* zp = z + static_cast<size_t>(b) * ldz + r;
   float mx = -INFINITY;
   int am = -1;
-  for (int v = tid; v < vocab; v += NT) {
-    const float l = L[v];
-    if (SMEM) es[v] = l;
-    if (v != mask_id && better(l, v, mx, am)) { mx = l; am = v; }
+  if (part) {
+    const float* pr = part + static_cast<size_t>(j) * n_tiles * 3;
+    for (int t = tid; t < n_tiles; t += NT) {
+      const int i = __float_as_int(pr[3 * t + 2]);
+      if (i >= 0 && better(pr[3 * t], i, mx, am)) { mx = pr[3 * t]; am = i; }
+    }
+  } else {
+    for (int v0 = tid * VEC; v0 < vocab; v0 += NT * VEC * U) {
+      float x[U][VEC];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int v = v0 + u * NT * VEC;
+        if (v < vocab) {
+          if constexpr (VEC == 4) {
+            const float4 t = *reinterpret_cast<const float4*>(L + v);
+            x[u][0] = t.x, x[u][1] = t.y, x[u][2] = t.z, x[u][3] = t.w;
+          } else {
+            x[u][0] = L[v];
+          }
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+#pragma unroll
+        for (int k = 0; k < VEC; ++k) {
+          const int v = v0 + u * NT * VEC + k;
+          if (v < vocab && v != mask_id && better(x[u][k], v, mx, am)) { mx = x[u][k]; am = v; }
+        }
+    }
   }
   block_argmax<NT>(mx, am, sv, si);
   if (last) {
     if (tid == 0) *zp = am;
     return;
   }
-  float Z = 0.0f, W = 0.0f;
-  for (int v = tid; v < vocab; v += NT) {
-    const float a = ((SMEM ? es[v] : L[v]) - mx) * inv_tau;
-    const float e = v == mask_id ? 0.0f : expf(a);
-    if (e > 0.0f) {
-      Z += e;
-      W = fmaf(e, a, W);
-    }
-    if (SMEM) es[v] = e;
-  }
-  Z = block_sum_f<NT>(Z, sv);
-  W = block_sum_f<NT>(W, sv);
-  const float ent0 = logf(Z) - W / Z;
-  const float ent = ent0 > 0.0f ? ent0 : 0.0f;      // rounding below 0 (and -0) -> +0: keys sort by bits
-  auto e_of = [&](int v) -> float {
-    if (SMEM) return es[v];
-    return v == mask_id ? 0.0f : expf((L[v] - mx) * inv_tau);
-  };
-  const int chunk = (vocab + NT - 1) / NT, v0 = tid * chunk, v1 = min(vocab, v0 + chunk);
-  float mine = 0.0f;
-  if (v1 > v0) {                                    // start at lane-rotated ids: no shared-memory bank conflicts
-    int v = SMEM ? v0 + (tid & 31) % (v1 - v0) : v0;
-    for (int k = v0; k < v1; ++k) {
-      mine += e_of(v);
-      if (++v == v1) v = v0;
-    }
-  }
-  __syncthreads();
-  scan[tid] = mine;
-  if (tid == 0) pick = -1;
-  __syncthreads();
-  for (int o = 1; o < NT; o <<= 1) {               // inclusive scan of the range sums (fixed order)
-    const float add = tid >= o ? scan[tid - o] : 0.0f;
-    __syncthreads();
-    scan[tid] += add;
-    __syncthreads();
-  }
-  float u[3];
-  remdm_draws(seed, step, B, R, b, r, u);
-  const float goal = u[0] * scan[NT - 1];
-  const float before = tid > 0 ? scan[tid - 1] : 0.0f;
-  if (mine > 0.0f && before <= goal && goal < scan[tid]) {
-    float c = before;
-    int lastv = -1, got = -1;
-    for (int v = v0; v < v1; ++v) {
-      const float e = e_of(v);
-      if (e > 0.0f) {
-        lastv = v;
-        c += e;
-        if (c > goal) {
-          got = v;
-          break;
+  // warp segments: S floats each (a multiple of 4), the last one shorter
+  const int S = (vocab + NW * 4 - 1) / (NW * 4) * 4;
+  auto e_of = [&](float l, int v) { return v == mask_id ? 0.0f : expf((l - mx) * inv_tau); };
+  {
+    const int lo = w * S, hi = min(vocab, lo + S);
+    float Z = 0.0f, W = 0.0f;
+    for (int v0 = lo + lane * VEC; v0 < hi; v0 += 32 * VEC * U) {
+      float x[U][VEC];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int v = v0 + u * 32 * VEC;
+        if (v < hi) {
+          if constexpr (VEC == 4) {
+            const float4 t = *reinterpret_cast<const float4*>(L + v);
+            x[u][0] = t.x, x[u][1] = t.y, x[u][2] = t.z, x[u][3] = t.w;
+          } else {
+            x[u][0] = L[v];
+          }
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const int v = v0 + u * 32 * VEC;
+        if (v >= hi) continue;
+        float e[VEC];
+#pragma unroll
+        for (int k = 0; k < VEC; ++k) {
+          const float a = (x[u][k] - mx) * inv_tau;
+          e[k] = v + k == mask_id ? 0.0f : expf(a);
+          if (e[k] > 0.0f) {
+            Z += e[k];
+            W = fmaf(e[k], a, W);
+          }
+        }
+        if (q) {
+          if (q_bf16) {
+            bf16* o = static_cast<bf16*>(q) + static_cast<size_t>(j) * ldq + v;
+            if constexpr (VEC == 4) {
+              __nv_bfloat162 p0 = __floats2bfloat162_rn(e[0], e[1]), p1 = __floats2bfloat162_rn(e[2], e[3]);
+              uint2 pk;
+              pk.x = *reinterpret_cast<uint32_t*>(&p0);
+              pk.y = *reinterpret_cast<uint32_t*>(&p1);
+              *reinterpret_cast<uint2*>(o) = pk;
+            } else {
+              o[0] = __float2bfloat16_rn(e[0]);
+            }
+          } else {
+            float* o = static_cast<float*>(q) + static_cast<size_t>(j) * ldq + v;
+            if constexpr (VEC == 4) *reinterpret_cast<float4*>(o) = make_float4(e[0], e[1], e[2], e[3]);
+            else o[0] = e[0];
+          }
         }
       }
     }
-    pick = got >= 0 ? got : lastv;
-  }
-  if (p) {                                          // p = e / Z for the self-conditioning product
-    const float iz = 1.0f / Z;
-    if (p_bf16) {
-      bf16* o = static_cast<bf16*>(p) + static_cast<size_t>(j) * ldp;
-      for (int v = tid; v < vocab; v += NT) o[v] = __float2bfloat16_rn(e_of(v) * iz);
-    } else {
-      float* o = static_cast<float*>(p) + static_cast<size_t>(j) * ldp;
-      for (int v = tid; v < vocab; v += NT) o[v] = e_of(v) * iz;
+    // fixed-order warp sums (the segment sums of the draw)
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      Z += __shfl_xor_sync(0xffffffffu, Z, o);
+      W += __shfl_xor_sync(0xffffffffu, W, o);
+    }
+    if (lane == 0) {
+      segZ[w] = Z;
+      segW[w] = W;
     }
   }
   __syncthreads();
   if (tid == 0) {
-    int v = pick;
-    for (int t = NT - 1; t >= 0 && v < 0; --t)     // rounding left the goal past every range: the last token
-      if ((t > 0 ? scan[t] - scan[t - 1] : scan[0]) > 0.0f)
-        for (int w = min(vocab, (t + 1) * chunk) - 1; w >= t * chunk; --w)
-          if (e_of(w) > 0.0f) { v = w; break; }
+    float u[3];
+    remdm_draws(seed, step, B, R, b, r, u);
+    float Zt = 0.0f, Wt = 0.0f;
+    for (int i = 0; i < NW; ++i) {
+      Zt += segZ[i];
+      Wt += segW[i];
+    }
+    const float goal = u[0] * Zt;
+    float c = 0.0f;
+    int seg = -1, lastseg = -1;
+    float before = 0.0f;
+    for (int i = 0; i < NW; ++i) {
+      if (segZ[i] > 0.0f) {
+        if (seg < 0 && c + segZ[i] > goal) {
+          seg = i;
+          before = c;
+        }
+        lastseg = i;
+      }
+      c += segZ[i];
+    }
+    if (seg < 0) {                                  // rounding left the goal past every segment: the last one
+      seg = lastseg;
+      before = c - segZ[lastseg >= 0 ? lastseg : 0];
+    }
+    sh_seg = seg;
+    sh_goal = goal - before;
+    sh_pick = -1;
+    sh_last = -1;
+    const float ent = logf(Zt) - Wt / Zt;
+    H[j] = ent > 0.0f ? ent : 0.0f;                 // rounding below 0 (and -0) -> +0: keys sort by bits
+    if (Zs) Zs[j] = Zt;
+  }
+  __syncthreads();
+  const int seg = sh_seg;
+  if (seg >= 0) {
+    const int lo = seg * S, hi = min(vocab, lo + S);
+    const int c = (hi - lo + NT - 1) / NT, a0 = min(hi, lo + tid * c), a1 = min(hi, a0 + c);
+    float mine = 0.0f;
+    int lastv = -1;
+    for (int v = a0; v < a1; ++v) {
+      const float e = e_of(L[v], v);
+      mine += e;
+      if (e > 0.0f) lastv = v;
+    }
+    // block inclusive scan of the sub-range sums (warp shuffles, then the warp
+    // totals); each thread's interval starts exactly where its predecessor's ends
+    float inc = mine;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const float t = __shfl_up_sync(0xffffffffu, inc, o);
+      if (lane >= o) inc += t;
+    }
+    float exc = __shfl_up_sync(0xffffffffu, inc, 1);
+    if (lane == 0) exc = 0.0f;
+    if (lane == 31) wsc[w] = inc;
+    if (lastv >= 0) atomicMax(&sh_last, lastv);
+    __syncthreads();
+    float wb = 0.0f;
+    for (int i = 0; i < w; ++i) wb += wsc[i];
+    inc += wb;
+    const float before = exc + wb, goal = sh_goal;
+    if (mine > 0.0f && before <= goal && goal < inc) {
+      float run = before;
+      int got = -1;
+      for (int v = a0; v < a1; ++v) {
+        const float e = e_of(L[v], v);
+        if (e > 0.0f) {
+          run += e;
+          if (run > goal) {
+            got = v;
+            break;
+          }
+        }
+      }
+      sh_pick = got >= 0 ? got : lastv;             // rounding kept the walk at or below the goal: the range's last
+    }
+    __syncthreads();
+  }
+  if (tid == 0) {
+    int v = seg >= 0 ? sh_pick : -1;
+    if (v < 0 && seg >= 0) v = sh_last;             // no sub-range held the goal: the segment's last token
     *zp = v < 0 ? am : v;
-    H[j] = ent;
   }
 }
 
@@ -814,25 +920,18 @@ const char* eb_rows(int32_t* idx, int B, int R, int first, cudaStream_t s) {
 }
 
 const char* eb_row(const float* logits, int ld, int B, int R, int first, int32_t* z, int ldz, int vocab, int mask_id,
-                   float inv_tau, int last, uint64_t seed, int step, void* p, int p_bf16, int ldp, float* H,
-                   cudaStream_t s) {
+                   float inv_tau, int last, uint64_t seed, int step, const float* part, int n_tiles, void* q,
+                   int q_bf16, int ldq, float* H, float* Zs, cudaStream_t s) {
   const int G = R - first, n = B * G;
   if (n <= 0) return nullptr;
-  const size_t smem = static_cast<size_t>(vocab) * sizeof(float);
-  if (smem <= 200u * 1024u) {   // the row's exponentials fit in shared memory
-    static bool attr = false;
-    if (!attr) {
-      if (cudaFuncSetAttribute(eb_row_kernel<1024, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024) !=
-          cudaSuccess)
-        return "entropy-bound sampler smem attribute failed";
-      attr = true;
-    }
-    launch_pdl(eb_row_kernel<1024, true>, n, 1024, smem, s, logits, ld, G, first, z, ldz, B, R, vocab, mask_id,
-               inv_tau, last, seed, step, p, p_bf16, ldp, H);
-  } else {
-    launch_pdl(eb_row_kernel<512, false>, n, 512, 0, s, logits, ld, G, first, z, ldz, B, R, vocab, mask_id, inv_tau,
-               last, seed, step, p, p_bf16, ldp, H);
-  }
+  const bool vec = vocab % 4 == 0 && ld % 4 == 0 && reinterpret_cast<uintptr_t>(logits) % 16 == 0 &&
+                   (!q || (ldq % 4 == 0 && reinterpret_cast<uintptr_t>(q) % 16 == 0));
+  if (vec)
+    launch_pdl(eb_row_kernel<512, 4>, n, 512, 0, s, logits, ld, G, first, z, ldz, B, R, vocab, mask_id, inv_tau, last,
+               seed, step, part, n_tiles, q, q_bf16, ldq, H, Zs);
+  else
+    launch_pdl(eb_row_kernel<512, 1>, n, 512, 0, s, logits, ld, G, first, z, ldz, B, R, vocab, mask_id, inv_tau, last,
+               seed, step, part, n_tiles, q, q_bf16, ldq, H, Zs);
   return err();
 }
 

@@ -388,12 +388,13 @@ tadm_status stack_fwd(tadm_handle* h, int first, int n, float* x, int B, int R, 
 
 // S: c = embed(z) then L_S layers (c lives in the workspace).
 // `add` (optional): the self-conditioning signal of rows add_first .. R-1 of
-// each sequence, fp32 [B * (R - add_first), d], added to their embedding.
+// each sequence, fp32 [B * (R - add_first), d], added to their embedding
+// (divided by add_div[row] when add_div is given).
 tadm_status run_S(tadm_handle* h, const int32_t* z, int ldz, int B, int R, int causal, cudaStream_t s,
-                  const float* add = nullptr, int add_first = 0) {
+                  const float* add = nullptr, int add_first = 0, const float* add_div = nullptr) {
   const tadm_config& c = h->cfg;
   float* cbuf = h->at<float>(h->off.c);
-  TRY(embed_rows(z, ldz, B, R, h->embed, c.dtype, c.d_model, c.vocab, cbuf, nullptr, s, add, add_first));
+  TRY(embed_rows(z, ldz, B, R, h->embed, c.dtype, c.d_model, c.vocab, cbuf, nullptr, s, add, add_first, add_div));
   return stack_fwd(h, 0, c.n_shared, cbuf, B, R, h->ctx, causal, s);
 }
 
@@ -1264,11 +1265,12 @@ tadm_status tadm_generate_remdm(tadm_handle* h, const int32_t* prompt, int batch
 namespace {
 
 // Caller scratch of the entropy-bound generation, in this order (each
-// segment 256-byte aligned): logits fp32 [n, V]; p [n, V] and E^T [d, V]
-// (model element type) and s fp32 [n, d] when self-conditioning; H fp32 [n];
+// segment 256-byte aligned): logits fp32 [n, V]; with self-conditioning
+// q = exp((l - max) / tau) [n, V] and E^T [d, V] (model element type), the
+// unnormalised signal q E fp32 [n, d] and Z = sum q fp32 [n]; H fp32 [n];
 // n = batch * gen_len.
 struct EbScratch {
-  size_t logits, p, et, sig, ent, total;
+  size_t logits, p, et, sig, zs, ent, total;
 };
 
 EbScratch eb_layout(const tadm_config& c, int batch, int gen_len, int self_cond) {
@@ -1285,6 +1287,7 @@ EbScratch eb_layout(const tadm_config& c, int batch, int gen_len, int self_cond)
     L.p = take(n * c.vocab * es);
     L.et = take(static_cast<size_t>(c.d_model) * c.vocab * es);
     L.sig = take(n * c.d_model * 4);
+    L.zs = take(n * 4);
   }
   L.ent = take(n * 4);
   L.total = o;
@@ -1305,7 +1308,8 @@ extern "C" {
 
 tadm_status tadm_eb_update(int32_t* z, int ldz, const float* logits, int ld_logits, int batch, int rows, int first_gen,
                            int vocab, int mask_id, double tau, double eta, int last, uint64_t seed, int step,
-                           float* entropy, void* probs, int probs_dtype, int ld_probs, tadm_stream stream) {
+                           float* entropy, void* probs, int probs_dtype, int ld_probs, float* z_sum,
+                           tadm_stream stream) {
   const int G = rows - first_gen;
   if (!z || !logits || batch <= 0 || rows <= 0 || first_gen < 0 || G <= 0 || ldz < rows || vocab < 2 ||
       ld_logits < vocab || mask_id < 0 || mask_id >= vocab || step < 0 || !(tau > 0.0) || eta != eta ||
@@ -1314,7 +1318,7 @@ tadm_status tadm_eb_update(int32_t* z, int ldz, const float* logits, int ld_logi
     return TADM_ERR_INVALID_ARG;
   cudaStream_t s = stream;
   if (eb_row(logits, ld_logits, batch, rows, first_gen, z, ldz, vocab, mask_id, static_cast<float>(1.0 / tau), last,
-             seed, step, last ? nullptr : probs, probs_dtype, ld_probs, entropy, s))
+             seed, step, nullptr, 0, last ? nullptr : probs, probs_dtype, ld_probs, entropy, z_sum, s))
     return TADM_ERR_CUDA;
   if (!last && eb_accept(entropy, batch, rows, first_gen, z, ldz, vocab, eta, seed, step, s)) return TADM_ERR_CUDA;
   return TADM_OK;
@@ -1356,6 +1360,8 @@ tadm_status tadm_generate_entropy_bound(tadm_handle* h, const int32_t* prompt, i
   void* p = self_cond ? base + L.p : nullptr;
   void* et = self_cond ? base + L.et : nullptr;
   float* sig = self_cond ? reinterpret_cast<float*>(base + L.sig) : nullptr;
+  float* zs = self_cond ? reinterpret_cast<float*>(base + L.zs) : nullptr;
+  const int head_tiles = c.dtype ? gemm_tc_tiles_n(c.vocab, EPI_LMHEAD) : gemm_simt_tiles_n(c.vocab, EPI_LMHEAD);
   int32_t* idx = h->at<int32_t>(h->off.idx);
   const int64_t Mmax = static_cast<int64_t>(h->max_batch) * h->max_rows;
   if (self_cond) TRY(transpose(h->embed, c.vocab, c.d_model, c.dtype, et, s));   // E^T [d, V] for s = p E
@@ -1365,7 +1371,7 @@ tadm_status tadm_generate_entropy_bound(tadm_handle* h, const int32_t* prompt, i
   void* cache = h->at(h->off.h_int);
   for (int i = 0; i < steps; ++i) {
     const int n = steps - i;                      // Alg. 2's n = T .. 1
-    TRYS(run_S(h, out, total, batch, R, 0, s, self_cond && i > 0 ? sig : nullptr, prompt_len));
+    TRYS(run_S(h, out, total, batch, R, 0, s, self_cond && i > 0 ? sig : nullptr, prompt_len, zs));
     if (i % K == 0) {                             // Alg. 1 refresh test (T - i) mod K = 0
       TRYS(run_A(h, batch, R, 0, cache, s));
       h->counters.anchor_layers += c.n_anchor;
@@ -1385,10 +1391,11 @@ tadm_status tadm_generate_entropy_bound(tadm_handle* h, const int32_t* prompt, i
     TRYS(gemm(h, norm, Mmax, c.d_model, h->lm_head, c.d_model, n_rows, c.vocab, c.d_model, EPI_LMHEAD, e, s));
     const double tau = tau_min + (tau_max - tau_min) * n / steps;
     const int last = n == 1;
+    // max and argmax from the head's partials; q = exp((l - max) / tau) and Z for s = (q E) / Z
     TRY(eb_row(logits, c.vocab, batch, R, prompt_len, out, total, c.vocab, mask, static_cast<float>(1.0 / tau), last,
-               seed, i, last ? nullptr : p, c.dtype, c.vocab, ent, s));
+               seed, i, e.part, head_tiles, last ? nullptr : p, c.dtype, c.vocab, ent, zs, s));
     if (!last) {
-      if (self_cond) {                            // s = p E for the next step's embedding
+      if (self_cond) {                            // q E; the next step's embedding adds it divided by Z
         EpiParams es{};
         es.out = sig;
         es.ldo = c.d_model;

@@ -105,9 +105,11 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
                                   ctypes.c_uint64, I, P, P]),
         "tadm_generate_remdm": (I, [P, P, I, I, P, I, I, I, I, ctypes.c_double, ctypes.c_float, ctypes.c_uint64, P,
                                     SZ, P]),
-        "tadm_eb_update": (I, [P, I, P, I, I, I, I, I, I, ctypes.c_double, ctypes.c_double, I, ctypes.c_uint64, I, P, P, I, I, P]),
+        "tadm_eb_update": (I, [P, I, P, I, I, I, I, I, I, ctypes.c_double, ctypes.c_double, I, ctypes.c_uint64, I,
+                               P, P, I, I, P, P]),
         "tadm_eb_scratch_bytes": (I, [P, I, I, I, ctypes.POINTER(SZ)]),
-        "tadm_generate_entropy_bound": (I, [P, P, I, I, P, I, I, I, ctypes.c_double, ctypes.c_double, ctypes.c_double, I, ctypes.c_uint64, P, SZ, P]),
+        "tadm_generate_entropy_bound": (I, [P, P, I, I, P, I, I, I, ctypes.c_double, ctypes.c_double,
+                                            ctypes.c_double, I, ctypes.c_uint64, P, SZ, P]),
         "tadm_probe_breakdown": (I, [P, I, ctypes.POINTER(I64), ctypes.POINTER(ctypes.c_double),
                                      ctypes.POINTER(ctypes.c_double)]),
         "tadm_probe_read": (I, [P, ctypes.POINTER(I64), ctypes.POINTER(ctypes.c_double),
@@ -255,10 +257,11 @@ def tadm_remdm_update(z, logits, first_gen: int, mask_id: int, sigma: float, p_u
 
 
 def tadm_eb_update(z, logits, first_gen: int, mask_id: int, tau: float, eta: float, last: bool, seed: int,
-                   step: int, entropy, probs=None, stream=None):
+                   step: int, entropy, probs=None, z_sum=None, stream=None):
     """One entropy-bound step (Alg. 2) on z [batch, rows] from the logits of
     the generated positions [batch * (rows - first_gen), vocab]; entropy
-    [batch * (rows - first_gen)] fp32; probs optional (fp32 or bf16)."""
+    [batch * (rows - first_gen)] fp32; probs (optional, fp32 or bf16) gets
+    q = exp((l - max) / tau) and z_sum (optional, fp32) Z = sum q."""
     batch, rows = z.shape
     vocab = logits.shape[1]
     p_dtype = 0
@@ -267,7 +270,7 @@ def tadm_eb_update(z, logits, first_gen: int, mask_id: int, tau: float, eta: flo
     _check(load_library().tadm_eb_update(_ptr(z), rows, _ptr(logits), vocab, batch, rows, first_gen, vocab, mask_id,
                                          tau, eta, int(bool(last)), seed, step, _ptr(entropy),
                                          _ptr(probs) if probs is not None else None, p_dtype,
-                                         probs.shape[1] if probs is not None else 0, _stream(stream)))
+                                         probs.shape[1] if probs is not None else 0, _ptr(z_sum), _stream(stream)))
 
 # ---------------------------------------------------------------------------- model handle
 class TadmModel:

@@ -144,7 +144,7 @@ def test_entropy_bound_arguments_are_rejected(lib):
         a = {**good, **over}
         st = so.tadm_eb_update(a["z"], a["ldz"], a["logits"], a["ld"], a["batch"], a["rows"], a["first"], a["vocab"],
                                a["mask"], a["tau"], a["eta"], a["last"], a["seed"], a["step"], a["ent"], a["probs"],
-                               a["pd"], a["ldp"], None)
+                               a["pd"], a["ldp"], None, None)
         assert st == 1, over
     size = ctypes.c_size_t()
     assert so.tadm_eb_scratch_bytes(None, 1, 1, 1, ctypes.byref(size)) == 1

@@ -194,6 +194,10 @@ WORKLOADS: Dict[str, Workload] = {
                           steps_per_block=32, K=4, block_len=32, k_sweep=(1, 4)),
     "sweep": Workload("sweep", BLOCK, batch=32, prompt_len=512, gen_len=2048, steps_per_block=16, K=4,
                       block_len=32, k_sweep=(1, 2, 4, 8, 16)),
+    # the post-training sampler settings of App. C.1: one 256-token canvas after the prompt, 48 reverse
+    # steps, anchor refresh K in {1, 2, 3}
+    "posttrain_canvas": Workload("posttrain_canvas", POSTTRAIN, batch=8, prompt_len=256, gen_len=256,
+                                 steps_per_block=48, K=2, k_sweep=(1, 2, 3)),
 }
 
 
