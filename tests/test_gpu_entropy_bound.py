@@ -195,3 +195,92 @@ def test_generate_entropy_bound_bf16_completes(T):
     assert np.array_equal(outs[0], outs[1]) and not np.array_equal(outs[0], outs[2])
     assert np.all(outs[0] != m.mask_id) and np.array_equal(outs[0][:, :P], p.cpu().numpy())
     tm.close()
+
+
+def test_eb_update_at_the_post_train_launch_shape(T):
+    """The sampler launch of the post-train canvas workload (batch 8, 256
+    generated positions after a 256-token prompt, V = 262144): on sampled
+    rows argmax exact, entropy within the fp32 bound, draws exact or on a
+    CDF edge; for every sequence the accepted set and re-noise tokens exact
+    given the kernel's entropies; the prompt untouched and no MASK."""
+    B, P, G, V, tau, eta, seed, step = 8, 256, 256, 262144, 0.6, 0.1, 77, 9
+    R, mask = P + G, V - 1
+    rng = np.random.default_rng(5)
+    logits = np.empty((B * G, V), np.float32)
+    for j in range(B * G):                          # mixed flat and peaked rows, as in the generation
+        logits[j] = rng.standard_normal(V, dtype=np.float32) * np.float32((0.5, 2.0, 6.0)[j % 3])
+    lt = torch.from_numpy(logits).cuda()
+    z0 = rng.integers(0, V - 1, (B, R)).astype(np.int32)
+    ent = torch.empty(B * G, dtype=torch.float32, device="cuda")
+    z = torch.from_numpy(z0).cuda()
+    T.tadm_eb_update(z, lt, P, mask, tau, eta, True, seed, step, ent)
+    am = z.cpu().numpy()
+    z = torch.from_numpy(z0).cuda()
+    T.tadm_eb_update(z, lt, P, mask, tau, float("inf"), False, seed, step, ent)
+    draws, H = z.cpu().numpy(), ent.cpu().numpy().astype(np.float64)
+    z = torch.from_numpy(z0).cuda()
+    T.tadm_eb_update(z, lt, P, mask, tau, eta, False, seed, step, ent)
+    acc = z.cpu().numpy()
+    torch.cuda.synchronize()
+    u = wl.remdm_uniforms(seed, step, B, R)
+    for out in (am, draws, acc):
+        assert np.array_equal(out[:, :P], z0[:, :P]) and np.all(out[:, P:] != mask)
+    edge = 0
+    for j in rng.choice(B * G, 24, replace=False):
+        b, g = divmod(int(j), G)
+        l64 = logits[j].astype(np.float64)
+        p, a_max, h, d = O.eb_row(l64, tau, mask, u[b, P + g, 0])
+        assert am[b, P + g] == a_max, (b, g)
+        mean_a = float(np.sum(p[p > 0] * (l64[p > 0] - l64[:mask].max()) / tau))
+        assert abs(H[j] - h) <= h_tol(V, mean_a), (b, g, H[j], h)
+        if draws[b, P + g] != d:
+            edge += 1
+            assert draw_valid(l64, tau, mask, u[b, P + g, 0], draws[b, P + g]), (b, g)
+    assert edge <= 1, edge
+    for b in range(B):
+        Hb = H[b * G:(b + 1) * G]
+        order = np.lexsort((np.arange(G), Hb))
+        margin = np.abs(np.cumsum(Hb[order]) - Hb[order] - eta)
+        close = np.zeros(G, bool)
+        close[order[margin < 1e-9]] = True
+        want = np.where(O.eb_accept(Hb, eta), draws[b, P:], np.floor(u[b, P:, 1] * (V - 1)).astype(np.int32))
+        assert np.array_equal(acc[b, P:][~close], want[~close]), b
+
+
+def test_generate_entropy_bound_one_step_bf16_argmax(T):
+    """T = 1 on the bf16 test model: the output is the argmax of the fused
+    prediction on step 1's noise canvas, taken by the sampler from the
+    tcgen05 output head's per-tile partials.  Against the oracle's fp64
+    logits (std 0.32): equal wherever the oracle's top-2 gap exceeds 2e-2,
+    about 15x the bf16 path's typical logit error (rel-L2 4e-3, ~1.3e-3
+    absolute), and >= 90 % overall."""
+    m = wl.ModelConfig(vocab=4096, d_model=256, n_heads=4, n_kv_heads=2, head_dim=64, ffn=768, n_anchor=3,
+                       n_denoise=2, dtype="bf16")
+    B, P, G, seed = 2, 16, 48, 23
+    w = wl.Workload("t", m, batch=B, prompt_len=P, gen_len=G, steps_per_block=1, K=1)
+    host = wl.make_weights(m, seed=4)
+    tm = T.TadmModel(m, T.upload_weights(m, host), max_batch=B, max_rows=P + G)
+    prompts = wl.make_prompts(w, batch=B, seed=6)
+    out = torch.empty((B, P + G), dtype=torch.int32, device="cuda")
+    scratch = torch.empty(tm.tadm_eb_scratch_bytes(B, G, True), dtype=torch.uint8, device="cuda")
+    tm.tadm_generate_entropy_bound(torch.from_numpy(prompts).cuda(), out, G, 1, 1, 0.1, 0.8, 0.4, seed, scratch, True)
+    tm.tadm_sync_status()
+    got = out.cpu().numpy()
+    tm.close()
+    o = O.Oracle(m, host)
+    u = wl.remdm_uniforms(seed, 1, B, P + G)
+    pos = np.arange(P + G)
+    agree = total = 0
+    for b in range(B):
+        zb = np.concatenate([prompts[b], np.floor(u[b, P:, 1] * (m.vocab - 1)).astype(np.int32)])
+        c = o.S(zb, pos, None)
+        lg = o.lm_head(o.D_hidden(o.fuse(c, o.make_cache(c, o.A(c, pos, None))), pos, None))[P:]
+        lg[:, m.mask_id] = -np.inf
+        top2 = np.sort(lg, axis=1)[:, -2:]
+        sure = top2[:, 1] - top2[:, 0] > 2e-2
+        ref = np.argmax(lg, axis=1)
+        assert np.array_equal(got[b, P:][sure], ref[sure]), b
+        assert np.array_equal(got[b, :P], prompts[b])
+        agree += int(np.sum(got[b, P:] == ref))
+        total += G
+    assert agree >= 0.90 * total, (agree, total)
