@@ -66,6 +66,42 @@ def dist_env():
     return rank, world, local
 
 
+class Ranks:
+    """The replicas of a multi-GPU run: one process per GPU, each generating
+    its own sequences, no exchange on the data path.  Only the timing needs
+    the group: a barrier on both sides of the timed region and the maximum
+    of the per-rank times (tensors on `device`: "cuda" under NCCL, "cpu"
+    under gloo)."""
+
+    def __init__(self, world: int, device: str = "cuda"):
+        self.world, self.device = world, device
+
+    def barrier(self):
+        if self.world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    def max(self, x: float) -> float:
+        if self.world == 1:
+            return x
+        import torch
+        import torch.distributed as dist
+        t = torch.tensor([x], dtype=torch.float64, device=self.device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+
+def whole_job_rate(world: int, units_per_step: int, steps: int, ms: float) -> float:
+    """Units all ranks processed per second over the slowest rank's time."""
+    return world * units_per_step * steps / (ms / 1000.0)
+
+
+def replica_prompts(w, rank: int):
+    """Each replica's own seeded prompts (rank 0 keeps the workload's)."""
+    import workloads as wl
+    return wl.make_prompts(w, seed=w.seed + 1000 * rank)
+
+
 def load_peaks():
     try:
         return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
@@ -202,7 +238,6 @@ def reference_arm(args):
 
 # ----------------------------------------------------------------------------- GPU arm
 def gpu_arm(args):
-    import numpy as np
     import torch
     import torch.distributed as dist
 
@@ -227,7 +262,7 @@ def gpu_arm(args):
     host_w = wl.make_weights(m, seed=w.seed)
     dev_w = upload_weights(m, host_w)
     del host_w
-    prompts = wl.make_prompts(w, seed=w.seed + 1000 * rank)         # each replica its own prompts
+    prompts = replica_prompts(w, rank)
     bl = w.block_len
     max_rows = max(w.prompt_len, bl) if bl else w.total_len
     tm = TadmModel(m, dev_w, max_batch=B, max_rows=max_rows, max_ctx=w.total_len if bl else 0)
@@ -238,9 +273,10 @@ def gpu_arm(args):
     def one(Kv):
         tm.tadm_generate(p_dev, out, w.gen_len, w.steps_per_block, Kv, bl, stream)
 
+    ranks = Ranks(world, "cuda")
+
     def barrier():
-        if world > 1:
-            dist.barrier()
+        ranks.barrier()
         torch.cuda.synchronize()
 
     def timed(Kv, steps, probe=False, warm=True):
@@ -264,11 +300,7 @@ def gpu_arm(args):
         if probe:
             tm.tadm_probe_enable(0)
         tm.tadm_sync_status()
-        if world > 1:
-            t = torch.tensor([ms], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ms = float(t.item())
-        return ms, launches, pr
+        return ranks.max(ms), launches, pr
 
     clocks = ClockSampler(local)
     ms, launches, _ = timed(K, args.steps)
@@ -277,13 +309,13 @@ def gpu_arm(args):
     # bracketed by events (the events add gaps, so the headline is not taken here)
     _, _, probe = timed(K, 1, probe=True, warm=False)
     tokens_per_step = B * w.gen_len
-    value = world * tokens_per_step * args.steps / (ms / 1000.0)
+    value = whole_job_rate(world, tokens_per_step, args.steps, ms)
     sweep = {}
     for s in [int(x) for x in args.sweep.split(",") if x.strip()]:
         if s == K:
             continue
         ms_s, _, _ = timed(s, args.steps)
-        sweep[str(s)] = world * tokens_per_step * args.steps / (ms_s / 1000.0)
+        sweep[str(s)] = whole_job_rate(world, tokens_per_step, args.steps, ms_s)
     sweep[str(K)] = value
 
     # e2e: public API with host buffers (pinned prompt in, tokens out), copies inside the timed region
@@ -296,13 +328,10 @@ def gpu_arm(args):
     for _ in range(0 if args.no_e2e else args.steps):
         res = tm.generate(hp, w.gen_len, w.steps_per_block, K, bl)
     barrier()
-    e2e_s = max(time.perf_counter() - t0, 1e-9)
-    if world > 1:
-        t = torch.tensor([e2e_s], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t.item())
-    e2e = None if args.no_e2e else {"value": world * tokens_per_step * args.steps / e2e_s, "unit": "tokens/s",
-           "h2d_bytes_per_step": int(hp.numel() * 4), "d2h_bytes_per_step": int(res.numel() * 4)}
+    e2e_s = ranks.max(max(time.perf_counter() - t0, 1e-9))
+    e2e = None if args.no_e2e else {"value": whole_job_rate(world, tokens_per_step, args.steps, 1000.0 * e2e_s),
+                                    "unit": "tokens/s", "h2d_bytes_per_step": int(hp.numel() * 4),
+                                    "d2h_bytes_per_step": int(res.numel() * 4)}
 
     peaks = load_peaks()
     (n_launch, gemm_ms, gemm_flops), gemm_kinds = probe
