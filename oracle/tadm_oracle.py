@@ -32,7 +32,7 @@ What it computes (paper section / equation it follows):
   with grouped KV heads, SwiGLU / GeGLU FFN), the layer type the workloads
   name; the paper treats it as a black box.
 
-Readings where the paper is silent (each one is listed in the design doc):
+Readings where the paper is silent:
 * sampler P: confidence top-k within the active block; conf = max softmax
   probability over the vocabulary without MASK, k_n = floor((n+1)G/T) -
   floor(nG/T), ties broken toward the lower position;
