@@ -148,3 +148,31 @@ def test_entropy_bound_arguments_are_rejected(lib):
         assert st == 1, over
     size = ctypes.c_size_t()
     assert so.tadm_eb_scratch_bytes(None, 1, 1, 1, ctypes.byref(size)) == 1
+
+
+@pytest.mark.parametrize("name,batch,gen", [("posttrain_canvas", 8, 256), ("small", 16, 768), ("tiny", 1, 96)])
+def test_entropy_bound_scratch_layout(lib, name, batch, gen):
+    """tadm_eb_scratch_bytes follows the header's layout: 256-byte aligned
+    segments of logits fp32 [n, V]; with self-conditioning q [n, V] and E^T
+    [d, V] in the model's element type, q E fp32 [n, d] and Z fp32 [n]; H
+    fp32 [n] (n = batch * gen_len).  The handle is host state only: it is
+    created over placeholder (aligned, never dereferenced) weight pointers."""
+    so = lib.load_library()
+    m = wl.WORKLOADS[name].model
+    cfg = lib.make_config(m)
+    n_w = so.tadm_weight_count(ctypes.byref(cfg))
+    ptrs = (ctypes.c_void_p * n_w)(*[256 * (i + 1) for i in range(n_w)])
+    h = ctypes.c_void_p()
+    assert so.tadm_create(ctypes.byref(cfg), ptrs, n_w, batch, 512 + gen, 0, ctypes.byref(h)) == 0
+    try:
+        al = lambda x: (x + 255) // 256 * 256  # noqa: E731
+        n, V, d, es = batch * gen, m.vocab, m.d_model, 2 if m.dtype == "bf16" else 4
+        want = {1: al(n * V * 4) + al(n * V * es) + al(d * V * es) + al(n * d * 4) + al(n * 4) + al(n * 4),
+                0: al(n * V * 4) + al(n * 4)}
+        for sc in (0, 1):
+            got = ctypes.c_size_t()
+            assert so.tadm_eb_scratch_bytes(h, batch, gen, sc, ctypes.byref(got)) == 0
+            assert got.value == want[sc], (sc, got.value, want[sc])
+        assert so.tadm_eb_scratch_bytes(h, 0, gen, 1, ctypes.byref(got)) == 1
+    finally:
+        so.tadm_destroy(h)
