@@ -176,3 +176,46 @@ def test_entropy_bound_scratch_layout(lib, name, batch, gen):
         assert so.tadm_eb_scratch_bytes(h, 0, gen, 1, ctypes.byref(got)) == 1
     finally:
         so.tadm_destroy(h)
+
+
+def test_sampler_generations_reject_bad_arguments_before_any_launch(lib):
+    """tadm_generate_entropy_bound and tadm_generate_remdm refuse bad
+    arguments on the host (status 1 and a message) on a host-only handle over
+    placeholder pointers, which no accepted call could dereference here."""
+    so = lib.load_library()
+    m = wl.ModelConfig(vocab=4096, d_model=256, n_heads=4, n_kv_heads=2, head_dim=64, ffn=768, n_anchor=3,
+                       n_denoise=2, dtype="bf16")
+    cfg = lib.make_config(m)
+    n_w = so.tadm_weight_count(ctypes.byref(cfg))
+    ptrs = (ctypes.c_void_p * n_w)(*[256 * (i + 1) for i in range(n_w)])
+    hs = {}
+    for ctx in (0, 256):
+        hs[ctx] = ctypes.c_void_p()
+        assert so.tadm_create(ctypes.byref(cfg), ptrs, n_w, 2, 96, ctx, ctypes.byref(hs[ctx])) == 0
+    try:
+        P, G, fake = 16, 64, ctypes.c_void_p(1 << 20)
+        need = ctypes.c_size_t()
+        assert so.tadm_eb_scratch_bytes(hs[0], 2, G, 1, ctypes.byref(need)) == 0
+        good = dict(h=hs[0], prompt=fake, batch=2, P=P, out=fake, G=G, steps=8, K=2, eta=0.1, tmax=0.8, tmin=0.4,
+                    sc=1, seed=1, scratch=fake, nbytes=need.value)
+        bad = [(dict(steps=0), "steps"), (dict(K=0), "K"), (dict(eta=float("nan")), "NaN"),
+               (dict(tmin=0.0), "tau"), (dict(tmax=0.3), "tau"), (dict(sc=2), "self_cond"),
+               (dict(prompt=None), "NULL"), (dict(scratch=None), "NULL"), (dict(G=0), "gen_len"),
+               (dict(G=20000), "gen_len"), (dict(h=hs[256]), "single-block"),
+               (dict(nbytes=need.value - 1), "scratch"), (dict(scratch=ctypes.c_void_p((1 << 20) + 128)), "aligned")]
+        for over, word in bad:
+            a = {**good, **over}
+            st = so.tadm_generate_entropy_bound(a["h"], a["prompt"], a["batch"], a["P"], a["out"], a["G"], a["steps"],
+                                                a["K"], a["eta"], a["tmax"], a["tmin"], a["sc"], a["seed"],
+                                                a["scratch"], a["nbytes"], None)
+            assert st == 1, over
+            assert word in so.tadm_last_error(a["h"]).decode(), (over, so.tadm_last_error(a["h"]))
+        # ReMDM: unknown schedule kind, top_p out of range, scratch too small, a KV-context handle
+        for over in [dict(kind=2), dict(top_p=0.0), dict(top_p=1.5), dict(nbytes=16), dict(h=hs[256])]:
+            a = {**dict(h=hs[0], kind=0, top_p=0.9, nbytes=2 * G * m.vocab * 4), **over}
+            st = so.tadm_generate_remdm(a["h"], fake, 2, P, fake, G, 8, 2, a["kind"], 0.04, a["top_p"], 1, fake,
+                                        a["nbytes"], None)
+            assert st == 1, over
+    finally:
+        for h in hs.values():
+            so.tadm_destroy(h)
