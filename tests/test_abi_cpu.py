@@ -219,3 +219,34 @@ def test_sampler_generations_reject_bad_arguments_before_any_launch(lib):
     finally:
         for h in hs.values():
             so.tadm_destroy(h)
+
+
+def test_generate_refuses_bad_arguments_and_missing_workspace(lib):
+    """tadm_generate's host checks on a host-only handle: a block length
+    that does not divide the generation, K or steps < 1, block mode without
+    a prompt or beyond the KV capacity, NULL buffers and a batch above the
+    handle's are INVALID_ARG; valid arguments without a bound workspace are
+    STATE; a misaligned or short workspace is refused before it is bound."""
+    so = lib.load_library()
+    m = wl.WORKLOADS["block"].model
+    cfg = lib.make_config(m)
+    n_w = so.tadm_weight_count(ctypes.byref(cfg))
+    ptrs = (ctypes.c_void_p * n_w)(*[256 * (i + 1) for i in range(n_w)])
+    h = ctypes.c_void_p()
+    assert so.tadm_create(ctypes.byref(cfg), ptrs, n_w, 4, 512, 2048, ctypes.byref(h)) == 0
+    try:
+        fake = ctypes.c_void_p(1 << 20)
+        good = dict(prompt=fake, batch=4, P=512, out=fake, G=1536, T=16, K=4, bl=32)
+        for over in [dict(bl=40), dict(K=0), dict(T=0), dict(G=0), dict(P=0), dict(G=2048), dict(prompt=None),
+                     dict(out=None), dict(batch=5), dict(batch=0)]:
+            a = {**good, **over}
+            st = so.tadm_generate(h, a["prompt"], a["batch"], a["P"], a["out"], a["G"], a["T"], a["K"], a["bl"], None)
+            assert st == 1, (over, so.tadm_last_error(h))
+        st = so.tadm_generate(h, fake, 4, 512, fake, 1536, 16, 4, 32, None)
+        assert st == 6 and b"workspace" in so.tadm_last_error(h)
+        need = ctypes.c_size_t()
+        assert so.tadm_workspace_size(h, ctypes.byref(need)) == 0 and need.value > 0
+        assert so.tadm_bind_workspace(h, ctypes.c_void_p((1 << 20) + 16), need.value) == 1
+        assert so.tadm_bind_workspace(h, fake, need.value - 1) == 4
+    finally:
+        so.tadm_destroy(h)
