@@ -779,3 +779,57 @@ def test_eb_signal_enters_as_an_embedding_offset():
     z2 = z.copy()
     z2[3] = 11
     assert np.allclose(o.S(z, pos, None, add=add), o.S(z2, pos, None), rtol=1e-12, atol=1e-12)
+
+
+# ------------------------------------------------------------ output head, block-mode context
+def test_output_head_normalises_the_hidden_state():
+    """logits = RMSNorm(y) W_out^T: a constant row y = a 1 normalises to
+    sign(a) gain, so its logits are sign(a) (W_out gain)_v in closed form,
+    and scaling y leaves the logits unchanged up to the eps term."""
+    o = tiny_oracle()
+    d = o.m.d_model
+    W, g = o.W("lm_head"), o.W("final_norm")
+    for a in (0.37, -2.5):
+        np.testing.assert_allclose(o.lm_head(np.full((1, d), a)), np.sign(a) * (W @ g)[None, :], rtol=1e-5)
+    y = rng.standard_normal((4, d))
+    np.testing.assert_allclose(o.lm_head(7.0 * y), o.lm_head(y), rtol=1e-5, atol=1e-8)
+
+
+def test_block_context_holds_the_committed_tokens():
+    """Block mode: the first step of block 2 sees a context equal to a
+    one-pass prefill of the prompt followed by block 1's final tokens (its
+    logits rebuilt from a fresh session), so the committed rows are the
+    block's tokens in their own order."""
+    o = tiny_oracle(n_shared=1)
+    logs = {}
+    prompts, out = _gen(o, K=2, block_len=4, G=8, T=4,
+                        hook=lambda b, n, z, r: logs.setdefault((b, n), (z.copy(), r["logits"])))
+    z10, l10 = logs[(1, 0)]
+    P = prompts.shape[1]
+    o2 = O.Oracle(o.m, o._raw)
+    sess = o2.new_session(2)
+    o2.prefill(sess, out[:, :P + 4])
+    cache = o2.anchor_forward(sess, z10)
+    np.testing.assert_allclose(o2.denoise_logits(sess, z10, cache), l10, rtol=1e-10, atol=1e-12)
+
+
+def test_encoder_pass_is_S_A_fusion_D():
+    """The block-mode encoder pass (prefill / commit, App. C.1) runs the
+    whole network causally: S, A, the fusion of (c, A(c)) and D, each layer
+    keeping its K, V.  Rebuilt from the networks on a fresh session, layer by
+    layer, its K and V are the session's."""
+    for fusion in ("gated_mlp", "paired_attn"):
+        o = tiny_oracle(n_shared=1, fusion=fusion)
+        z = rng.integers(0, 63, size=9).astype(np.int32)
+        s1 = o.new_session(1)[0]
+        o._fresh_pass(s1, z)
+        s2 = o.new_session(1)[0]
+        pos = np.arange(9)
+        c = o.S(z, pos, s2, causal=True, keep_kv=True)
+        h = o.A(c, pos, s2, causal=True, keep_kv=True)
+        ht = o.fuse(c, o.make_cache(c, h))
+        o.D_hidden(ht, pos, s2, causal=True, keep_kv=True)
+        assert sorted(s1.kv) == sorted(s2.kv) and any(k.startswith("denoise.") for k in s1.kv)
+        for name in s1.kv:
+            np.testing.assert_allclose(s1.kv[name][0], s2.kv[name][0], rtol=1e-12, atol=1e-14)
+            np.testing.assert_allclose(s1.kv[name][1], s2.kv[name][1], rtol=1e-12, atol=1e-14)
