@@ -53,6 +53,21 @@ def test_generator_moments_and_bf16_rounding():
     assert np.array_equal(ref, b)                                  # torch's conversion is also RNE
 
 
+def test_zipf_prompts_follow_the_power_law():
+    """Prompt ids (the synthetic stand-in for real prompts): rank r = id + 1
+    with p(r) proportional to r^-1.1 over ranks 1 .. V-1; the empirical
+    frequencies of the first ranks match it and MASK never appears."""
+    m = tiny_model(vocab=1000)
+    w = wl.Workload("z", m, batch=64, prompt_len=4096, gen_len=8, steps_per_block=1, K=1, prompt_dist="zipf")
+    ids = wl.make_prompts(w, seed=9).ravel()
+    assert ids.min() >= 0 and ids.max() <= m.vocab - 2
+    r = np.arange(1, m.vocab, dtype=np.float64)
+    p = r ** -1.1 / np.sum(r ** -1.1)
+    f = np.bincount(ids, minlength=m.vocab - 1)[: m.vocab - 1] / ids.size
+    se = np.sqrt(p[:20] * (1 - p[:20]) / ids.size)
+    assert np.all(np.abs(f[:20] - p[:20]) < 5 * se), (f[:5], p[:5])
+
+
 # --------------------------------------------------------------------------- elementary ops
 def test_norms_against_torch_and_closed_form():
     x = rng.standard_normal((5, 12))
