@@ -8,8 +8,11 @@
  * denoiser D.  The anchor latent h = A(S(z)) is refreshed once every K
  * reverse steps and cached in HBM; every step encodes the current canvas
  * c = S(z), fuses it with the stale cache, h~ = Phi(c, h_cache)
- * (Eq. stale-anchor-fusion), and denoises, x = D(h~) (Alg. 1).  The sampler
- * unmasks the most confident masked positions of the active block.
+ * (Eq. stale-anchor-fusion), and denoises, x = D(h~) (Alg. 1).  The default
+ * sampler unmasks the most confident masked positions of the active block;
+ * the paper's own samplers, ReMDM remasking (App. C.2) and the entropy-bound
+ * sampler with self-conditioning (App. C.1, Alg. 2), have entry points of
+ * their own at the end of this header.
  *
  * Conventions for every call:
  *  - Pointers named "device" are CUDA device pointers; the caller owns and
@@ -225,8 +228,9 @@ TADM_API tadm_status tadm_probe_read(tadm_handle* h, int64_t* launches, double* 
 /* The records split by kind: GEMM epilogues 0 plain, 1 residual, 2 QKV +
  * RoPE, 3 GLU, 4 fusion gate/hidden, 5 fusion output, 6 output head,
  * 7..10 paired-attention fusion; 11 attention; 12 RMSNorm / LayerNorm
- * launches; 13 attention over fewer than 128 canvas rows (block steps).  Arrays of n_kinds entries.  Call before tadm_probe_read, which
- * clears the records. */
+ * launches; 13 attention over fewer than 128 canvas rows (block steps).
+ * Arrays of n_kinds entries.  Call before tadm_probe_read, which clears the
+ * records. */
 TADM_API tadm_status tadm_probe_breakdown(tadm_handle* h, int n_kinds, int64_t* launches, double* ms,
                                           double* flops);
 
