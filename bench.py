@@ -56,6 +56,12 @@ def parse():
     ap.add_argument("--sweep-batches", default="", help="batches for the 'sweep' workload (default 1,8,32,128)")
     ap.add_argument("--kernel-bench", default=None,
                     help="time one building block alone instead, e.g. gemm:16384,32768,768")
+    ap.add_argument("--configs", default="block,posttrain",
+                    help="at N = 1: workloads also timed whole (K = 1 and the workload's K) and reported under "
+                         "'configs' in the same JSON line ('' for none)")
+    ap.add_argument("--config-steps", type=int, default=2, help="timed generations per K of each extra workload")
+    ap.add_argument("--config-warmup", type=int, default=2,
+                    help="untimed generations per K of each extra workload (the second one captures the CUDA graph)")
     return ap.parse_args()
 
 
@@ -64,6 +70,30 @@ def dist_env():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     return rank, world, local
+
+
+def rank_launch_command(gpus: int, argv, port: int):
+    """torch.distributed.run command that starts `gpus` local ranks of this
+    script with the same arguments (rendezvous on 127.0.0.1)."""
+    return [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", f"--nproc-per-node={gpus}",
+            "--master-addr", "127.0.0.1", f"--master-port={port}", os.path.abspath(__file__), *argv]
+
+
+def launch_ranks_if_needed(gpus: int, argv):
+    """--gpus N > 1 outside torchrun: start the N ranks here and return their
+    exit code.  Inside torchrun, WORLD_SIZE must equal N (None: go on)."""
+    env_world = os.environ.get("WORLD_SIZE")
+    if env_world is not None:
+        if int(env_world) != gpus:
+            raise SystemExit(f"bench.py: --gpus {gpus} but WORLD_SIZE={env_world}; launch one rank per GPU")
+        return None
+    if gpus <= 1:
+        return None
+    import socket
+    with socket.socket() as sk:
+        sk.bind(("127.0.0.1", 0))
+        port = sk.getsockname()[1]
+    return subprocess.call(rank_launch_command(gpus, argv, port))
 
 
 class Ranks:
@@ -166,6 +196,7 @@ sys.path.insert(0, {ROOT!r})
 import numpy as np
 import workloads as wl
 from oracle import tadm_oracle as O
+t_start = time.perf_counter()
 w = wl.get_workload({workload!r})
 m = w.model
 host = wl.make_weights(m, seed=w.seed)
@@ -173,7 +204,7 @@ o = O.Oracle(m, host)
 prompts = wl.make_prompts(w, batch=1)
 T, K = w.steps_per_block, {K}
 budget = {budget_s}
-t_start = time.perf_counter()
+t_work = time.perf_counter()
 sess = o.new_session(1)
 R = w.block_len if w.block_len else w.total_len
 if w.block_len:
@@ -189,9 +220,10 @@ for n in range(K):
     r = o.denoise_step(sess, z, cache, n, T, w.block_len or w.gen_len)
     steps.append(time.perf_counter() - t0)
     z = r["z"]
-    if time.perf_counter() - t_start > budget and len(steps) >= 1:
+    if time.perf_counter() - t_work > budget and len(steps) >= 1:
         break
 t_step = sum(steps) / len(steps)
+# wall covers the whole sample: weights, prompts, prefill, refresh and steps
 nb = w.n_blocks
 refresh = nb * (-(-T // K))
 gen_time = refresh * t_anchor + nb * T * t_step + (t_prefill * (1 + nb) if w.block_len else 0.0)
@@ -228,7 +260,10 @@ def reference_arm(args):
               f"{w.steps_per_block * w.n_blocks}-step generation of {w.gen_len} tokens")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "higher_is_better": True,
-            "ms_per_step": 1000.0 * statistics.median([s["gen_time"] for s in times]),
+            # one step = one timed sample (its wall time, weights and set-up included); value divides the
+            # generated tokens by the generation time extrapolated from the sample's refresh and step times
+            "ms_per_step": 1000.0 * statistics.median([s["wall"] for s in times]),
+            "extrapolated_generation_ms": 1000.0 * statistics.median([s["gen_time"] for s in times]),
             "dtype": "f64", "data": "synthetic",
             "config": {"workload": w.name, "batch": 1, "K": K},
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": threads, "kind": "oracle", "sample": sample},
@@ -366,21 +401,113 @@ def gpu_arm(args):
                        "l2": "inputs larger than L2 (weights + activations per step >> 129 MB)"},
             "k_sweep_tokens_per_s": sweep, "roofline": roofline, "clocks": clk,
             "e2e": e2e, "gpu_launches": launches}
+    # the other configurations, timed whole by this same run (N = 1 only)
+    del tm, dev_w
+    torch.cuda.empty_cache()
+    if world == 1 and args.configs:
+        line["configs"] = {}
+        for name in [x for x in args.configs.split(",") if x]:
+            try:
+                line["configs"][name] = config_leg(name, args.config_steps, args.config_warmup, peaks, local)
+            except Exception as e:  # context for the headline; the line still prints
+                line["configs"][name] = {"error": str(e)[-300:]}
+            torch.cuda.empty_cache()
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         try:
             threads = os.cpu_count() or 1
             s = cpu_oracle_sample(args.workload, K, args.cpu_sample_seconds, threads)
+            s1 = cpu_oracle_sample(args.workload, K, args.cpu_sample_seconds, 1)
             line["cpu_baseline"] = {
                 "value": s["tokens"] / s["gen_time"], "unit": "tokens/s", "cores": threads, "kind": "oracle",
                 "sample": (f"batch 1: one anchor refresh ({s['t_anchor']:.2f} s) + {s['steps']} denoising steps "
                            f"({s['t_step']:.2f} s each) of the '{w.name}' workload, extrapolated to the "
-                           f"{w.steps_per_block * w.n_blocks}-step generation of {w.gen_len} tokens")}
+                           f"{w.steps_per_block * w.n_blocks}-step generation of {w.gen_len} tokens"),
+                "single_thread": {"value": s1["tokens"] / s1["gen_time"], "unit": "tokens/s", "cores": 1,
+                                  "sample": f"the same sample on one thread (refresh {s1['t_anchor']:.2f} s, "
+                                            f"{s1['steps']} steps of {s1['t_step']:.2f} s)"}}
         except Exception as e:  # the baseline is context; the GPU line still prints
             line["cpu_baseline"] = {"error": str(e)[-300:]}
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
+
+
+def config_leg(name: str, steps: int, warmup: int, peaks, local: int) -> dict:
+    """Whole generations of another workload at K = 1 and its own K: tokens/s,
+    the speedup over K = 1 and, from one probed generation at its K, the GEMMs'
+    throughput against the tensor peak and their algorithmic bytes against
+    HBM bandwidth (the weight-streaming configurations are bound by the
+    latter).  Each timed generation includes the prompt prefill and every
+    block's commit pass."""
+    import torch
+
+    import workloads as wl
+    from paper_2609_37924_gb300 import TadmModel, upload_weights
+
+    w = wl.get_workload(name)
+    m, B, bl = w.model, w.batch, w.block_len
+    t0 = time.perf_counter()
+    dev_w = upload_weights(m, wl.make_weights(m, seed=w.seed))
+    t_weights = time.perf_counter() - t0
+    tm = TadmModel(m, dev_w, max_batch=B, max_rows=max(w.prompt_len, bl) if bl else w.total_len,
+                   max_ctx=w.total_len if bl else 0)
+    p = torch.from_numpy(wl.make_prompts(w)).cuda()
+    out = torch.empty((B, w.total_len), dtype=torch.int32, device="cuda")
+    stream = torch.cuda.current_stream()
+    res, ms_gen = {}, {}
+    clocks = ClockSampler(local)
+    for Kv in sorted({1, w.K}):
+        for _ in range(warmup):
+            tm.tadm_generate(p, out, w.gen_len, w.steps_per_block, Kv, bl, stream)
+        tm.tadm_sync_status()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(steps):
+            tm.tadm_generate(p, out, w.gen_len, w.steps_per_block, Kv, bl, stream)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms_gen[Kv] = e0.elapsed_time(e1) / steps
+        res[Kv] = B * w.gen_len / (ms_gen[Kv] / 1000.0)
+    clk = clocks.stop()
+    tm.tadm_sync_status()
+    valid = bool((out != m.mask_id).all())
+    # one probed generation at the workload's K (events around every launch)
+    tm.tadm_probe_enable(1000000)
+    tm.tadm_generate(p, out, w.gen_len, w.steps_per_block, w.K, bl, stream)
+    kinds = tm.tadm_probe_breakdown()
+    tm.tadm_probe_enable(0)
+    tm.tadm_sync_status()
+    gemm = [v for k, v in kinds.items() if k not in ("attention", "norms", "attention_short_rows")]
+    g_ms = sum(v["ms"] for v in gemm)
+    g_fl = sum(v["flops"] for v in gemm)
+    g_by = sum(v["bytes"] for v in gemm)
+    tf_peak = peaks["bf16_tflops_sustained"] if peaks else 1700.0
+    bw_peak = peaks["hbm_gbs"] if peaks else 6800.0
+    tflops = g_fl / (g_ms / 1000.0) / 1e12 if g_ms > 0 else None
+    gbs = g_by / (g_ms / 1000.0) / 1e9 if g_ms > 0 else None
+    bound = "hbm" if (gbs or 0) / bw_peak > (tflops or 0) / tf_peak else "tensor"
+    leg = {"workload": name, "batch": B, "prompt_len": w.prompt_len, "gen_len": w.gen_len, "block_len": bl,
+           "steps_per_block": w.steps_per_block, "d_model": m.d_model,
+           "layers": [m.n_shared, m.n_anchor, m.n_denoise], "vocab": m.vocab,
+           "tokens_per_s": {str(k): v for k, v in res.items()},
+           "ms_per_generation": {str(k): v for k, v in ms_gen.items()},
+           "vs_K1": res[w.K] / res[1], "timed_generations": steps, "warmup": warmup,
+           "all_unmasked": valid, "weights_s": round(t_weights, 1), "clocks": clk,
+           "roofline": {"bound": bound, "kernel": "gemm_tc kernels (all GEMM launches of one generation at K="
+                                                  f"{w.K})",
+                        "tflops": tflops, "tensor_peak": tf_peak, "tensor_frac": tflops / tf_peak if tflops else None,
+                        "gbs": gbs, "hbm_peak": bw_peak, "hbm_frac": gbs / bw_peak if gbs else None,
+                        "gemm_ms_per_generation": g_ms,
+                        "gemm_share": g_ms / ms_gen[w.K] if ms_gen.get(w.K) else None,
+                        "launches": int(sum(v["launches"] for v in gemm)),
+                        "peak_source": "MEASURED_PEAKS.json (sustained bf16, HBM copy)" if peaks else "fallback"},
+           "others_ms_per_generation": {k: v["ms"] for k, v in kinds.items()
+                                        if k in ("attention", "norms", "attention_short_rows")}}
+    tm.close()
+    del tm, dev_w
+    return leg
 
 
 def kernel_bench(args):
@@ -537,6 +664,9 @@ def workload_sweep(args):
 
 def main():
     args = parse()
+    rc = launch_ranks_if_needed(args.gpus, sys.argv[1:])
+    if rc is not None:
+        sys.exit(rc)
     if args.sweep_workloads:
         import __graft_entry__
         __graft_entry__.build()

@@ -129,7 +129,10 @@ TADM_API const char* tadm_status_string(tadm_status s);
 /* Device workspace: activations, KV caches, the internal anchor cache of
  * tadm_generate and the status word.  Caller allocates >= *bytes, 256-byte
  * aligned, and binds it before any compute call.  Binding synchronises the
- * device once (it fills the RoPE table). */
+ * device once (it fills the RoPE table) and drops the CUDA graph that
+ * tadm_generate may hold, so nothing recorded on the previous workspace is
+ * replayed; the previous workspace may be freed once the work queued on it
+ * has finished. */
 TADM_API tadm_status tadm_workspace_size(const tadm_handle* h, size_t* bytes);
 TADM_API tadm_status tadm_bind_workspace(tadm_handle* h, void* dev_ptr, size_t bytes);
 
@@ -194,7 +197,11 @@ TADM_API tadm_status tadm_commit_block(tadm_handle* h, const int32_t* x_block, i
  * prompt_len]; out: device int32 [batch, prompt_len + gen_len], the final
  * canvas.  block_len = 0: one block over the whole canvas (bidirectional,
  * no KV context); else gen_len % block_len == 0 and the prompt is prefilled.
- * The anchor refreshes at n = 0, K, 2K, ... of every block. */
+ * The anchor refreshes at n = 0, K, 2K, ... of every block.  The second call
+ * with the same sizes, prompt, out and workspace is captured into a CUDA
+ * graph on an internal stream and later identical calls replay it (ordered
+ * after the caller's stream by events); TADM_GRAPH=0 in the environment
+ * keeps every call eager. */
 TADM_API tadm_status tadm_generate(tadm_handle* h, const int32_t* prompt, int batch, int prompt_len,
                           int32_t* out, int gen_len, int steps_per_block, int K, int block_len,
                           tadm_stream stream);
@@ -229,10 +236,13 @@ TADM_API tadm_status tadm_probe_read(tadm_handle* h, int64_t* launches, double* 
  * RoPE, 3 GLU, 4 fusion gate/hidden, 5 fusion output, 6 output head,
  * 7..10 paired-attention fusion; 11 attention; 12 RMSNorm / LayerNorm
  * launches; 13 attention over fewer than 128 canvas rows (block steps).
- * Arrays of n_kinds entries.  Call before tadm_probe_read, which clears the
- * records. */
+ * Arrays of n_kinds entries.  bytes (optional, may be NULL): the algorithmic
+ * bytes of the GEMM records (A and B read once, the output written once, the
+ * residual stream read and written by residual epilogues; for the output
+ * head only A and B, its logits never reach memory).  Call before
+ * tadm_probe_read, which clears the records. */
 TADM_API tadm_status tadm_probe_breakdown(tadm_handle* h, int n_kinds, int64_t* launches, double* ms,
-                                          double* flops);
+                                          double* flops, double* bytes);
 
 /* Plan of tadm_generate (host only, no GPU): the ordered phases it issues.
  * kind: 0 prefill, 1 anchor refresh, 2 denoise step, 3 commit.  For kinds 1
@@ -299,6 +309,11 @@ TADM_API tadm_status tadm_head_confidence(const void* x, const void* w, int rows
  *  - The first call on each device looks up the array's device address
  *    (cudaGetSymbolAddress, with that device current); make that first call
  *    before any stream capture.  Later calls on the device only launch.
+ *    Like every entry point of this library it assumes one device per
+ *    process whose context lives until exit: after cudaDeviceReset the
+ *    remembered address is stale and the library must not be called again.
+ *  - Argument errors are those of tadm_head_confidence, checked in the same
+ *    order (also when rows == 0).
  *  - No allocation of any kind: no cudaMalloc / cudaFree, no allocating
  *    library routine.
  *  - Every call shares the one array and leaves its partials there; nothing

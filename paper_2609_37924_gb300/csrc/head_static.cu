@@ -25,7 +25,11 @@ std::mutex g_mu;
 void* g_addr[kMaxDevices] = {};
 
 // Device address of g_head_partials on the current device, looked up once
-// per device (with that device current) and remembered.
+// per device (with that device current) and remembered.  Like the rest of
+// the library (whose GEMM launch attributes are also set once per process),
+// this assumes one device per process and a context that lives as long as
+// the process: after cudaDeviceReset the remembered address is stale, so the
+// library must not be called again in that process.
 tadm_status partials_address(void** out) {
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return TADM_ERR_CUDA;
@@ -46,6 +50,8 @@ extern "C" tadm_status tadm_head_confidence_static(const void* x, const void* w,
                                                    tadm_stream stream) {
   size_t need = 0;
   if (tadm_head_scratch_size(rows, vocab, dtype, &need) != TADM_OK) return TADM_ERR_INVALID_ARG;
+  // the argument checks of tadm_head_confidence, before the early return for rows == 0
+  if (!x || !w || !conf || !tok || d <= 0 || mask_id < 0 || mask_id >= vocab) return TADM_ERR_INVALID_ARG;
   if (need > kPartialBytes) return TADM_ERR_INVALID_ARG;  // beyond the fixed array: use tadm_head_confidence
   if (rows == 0) return TADM_OK;
   void* scratch = nullptr;

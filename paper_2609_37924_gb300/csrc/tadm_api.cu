@@ -127,7 +127,7 @@ struct tadm_handle {
 
   // GEMM timing probe
   std::vector<cudaEvent_t> probe_ev;
-  std::vector<double> probe_flops;
+  std::vector<double> probe_flops, probe_bytes;   // algorithmic FLOPs and bytes of each record
   std::vector<int> probe_kind;
   int probe_next = 0;
 
@@ -137,14 +137,15 @@ struct tadm_handle {
   cudaStream_t last_stream = nullptr;
   std::string err;
 
-  // CUDA graph of a repeated tadm_generate call (same sizes and pointers):
-  // the second such call is captured on an internal stream, later ones replay
-  // it.  The host-side results of the captured run (counters, context length)
-  // are restored on replay.
+  // CUDA graph of a repeated tadm_generate call (same sizes and pointers,
+  // workspace included): the second such call is captured on an internal
+  // stream, later ones replay it.  The host-side results of the captured run
+  // (counters, context length) are restored on replay.  Binding a workspace
+  // destroys the graph.
   cudaStream_t gstream = nullptr;
   cudaEvent_t gev_in = nullptr, gev_out = nullptr;
   cudaGraphExec_t gexec = nullptr;
-  int64_t gkey[8] = {}, gkey_seen[8] = {};
+  int64_t gkey[9] = {}, gkey_seen[9] = {};   // sizes, prompt, out and workspace pointers
   tadm_counters gcounters{};
   int gctx = 0;
 
@@ -286,11 +287,12 @@ int probe_begin(tadm_handle* h, cudaStream_t s) {
   cudaEventRecord(h->probe_ev[2 * h->probe_next], s);
   return h->probe_next++;
 }
-void probe_end(tadm_handle* h, cudaStream_t s, int idx, int kind, double flops) {
+void probe_end(tadm_handle* h, cudaStream_t s, int idx, int kind, double flops, double bytes = 0.0) {
   if (idx < 0) return;
   cudaEventRecord(h->probe_ev[2 * idx + 1], s);
   h->probe_kind[idx] = kind;
   h->probe_flops[idx] = flops;
+  h->probe_bytes[idx] = bytes;
 }
 
 tadm_status gemm(tadm_handle* h, const void* A, int64_t a_rows, int lda, const void* B, int ldb, int M, int N, int K,
@@ -319,7 +321,13 @@ tadm_status gemm(tadm_handle* h, const void* A, int64_t a_rows, int lda, const v
   if (e) return fail(h, TADM_ERR_CUDA, "GEMM (M=%d N=%d K=%d epi=%d): %s", M, N, K, epi, e);
   h->counters.kernel_launches += h->cfg.dtype ? g.launched : 1;
   const double n_acc = epi == EPI_GLU ? 2.0 * N : static_cast<double>(N);
-  probe_end(h, s, pi, epi, 2.0 * M * n_acc * K);
+  // algorithmic bytes: A and B read once, the output written once (fp32 or
+  // the activation type), the residual stream read and written by EPI_RESID
+  const double es = h->es(), out_es = (epi == EPI_RESID || out_f32 || !h->act_bf16()) ? 4.0 : es;
+  const double bytes = es * (static_cast<double>(M) * K + n_acc * K) + out_es * M * N +
+                       (epi == EPI_RESID ? 4.0 * M * N : 0.0);
+  probe_end(h, s, pi, epi, 2.0 * M * n_acc * K, epi == EPI_LMHEAD ? es * (static_cast<double>(M) * K + n_acc * K)
+                                                                  : bytes);
   return TADM_OK;
 }
 
@@ -818,21 +826,25 @@ tadm_status tadm_probe_enable(tadm_handle* h, int max_launches) {
   for (cudaEvent_t e : h->probe_ev) cudaEventDestroy(e);
   h->probe_ev.clear();
   h->probe_flops.clear();
+  h->probe_bytes.clear();
   h->probe_next = 0;
   if (max_launches == 0) return TADM_OK;
   h->probe_ev.resize(2 * static_cast<size_t>(max_launches));
   for (auto& e : h->probe_ev)
     if (cudaEventCreate(&e) != cudaSuccess) return fail(h, TADM_ERR_CUDA, "cudaEventCreate failed");
   h->probe_flops.assign(max_launches, 0.0);
+  h->probe_bytes.assign(max_launches, 0.0);
   h->probe_kind.assign(max_launches, 0);
   return TADM_OK;
 }
 
-tadm_status tadm_probe_breakdown(tadm_handle* h, int n_kinds, int64_t* launches, double* ms, double* flops) {
+tadm_status tadm_probe_breakdown(tadm_handle* h, int n_kinds, int64_t* launches, double* ms, double* flops,
+                                 double* bytes) {
   if (!h || n_kinds <= 0 || !launches || !ms || !flops) return TADM_ERR_INVALID_ARG;
   for (int k = 0; k < n_kinds; ++k) {
     launches[k] = 0;
     ms[k] = flops[k] = 0.0;
+    if (bytes) bytes[k] = 0.0;
   }
   if (h->probe_next > 0 && cudaEventSynchronize(h->probe_ev[2 * h->probe_next - 1]) != cudaSuccess)
     return fail(h, TADM_ERR_CUDA, "probe event sync failed");
@@ -845,6 +857,7 @@ tadm_status tadm_probe_breakdown(tadm_handle* h, int n_kinds, int64_t* launches,
     launches[k] += 1;
     ms[k] += t;
     flops[k] += h->probe_flops[i];
+    if (bytes) bytes[k] += h->probe_bytes[i];
   }
   return TADM_OK;
 }
@@ -883,6 +896,13 @@ tadm_status tadm_bind_workspace(tadm_handle* h, void* dev_ptr, size_t bytes) {
   if (!h || !dev_ptr) return TADM_ERR_INVALID_ARG;
   if (reinterpret_cast<uintptr_t>(dev_ptr) & 255) return fail(h, TADM_ERR_INVALID_ARG, "workspace not 256-byte aligned");
   if (bytes < h->ws_need) return fail(h, TADM_ERR_OOM, "workspace %zu < %zu bytes", bytes, h->ws_need);
+  // a graph captured on the previous workspace must never replay on the new one
+  if (h->gexec) {
+    cudaGraphExecDestroy(h->gexec);
+    h->gexec = nullptr;
+  }
+  std::memset(h->gkey, 0, sizeof(h->gkey));
+  std::memset(h->gkey_seen, 0, sizeof(h->gkey_seen));
   h->ws = static_cast<char*>(dev_ptr);
   h->ws_bytes = bytes;
   const int n_pos = h->kv_stride + h->max_rows;
@@ -989,9 +1009,10 @@ tadm_status tadm_generate(tadm_handle* h, const int32_t* prompt, int batch, int 
     const char* e = getenv("TADM_GRAPH");
     return !(e && e[0] == '0');
   }();
-  const int64_t key[8] = {batch, prompt_len, gen_len, steps_per_block, K, block_len,
+  const int64_t key[9] = {batch, prompt_len, gen_len, steps_per_block, K, block_len,
                           static_cast<int64_t>(reinterpret_cast<uintptr_t>(prompt)),
-                          static_cast<int64_t>(reinterpret_cast<uintptr_t>(out))};
+                          static_cast<int64_t>(reinterpret_cast<uintptr_t>(out)),
+                          static_cast<int64_t>(reinterpret_cast<uintptr_t>(h->ws))};
   if (!graphs_on || !h->probe_flops.empty()) return generate_loop(h, prompt, batch, prompt_len, out, gen_len,
                                                                   steps_per_block, K, block_len, stream);
   const bool seen = std::memcmp(key, h->gkey_seen, sizeof(key)) == 0;

@@ -111,7 +111,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "tadm_generate_entropy_bound": (I, [P, P, I, I, P, I, I, I, ctypes.c_double, ctypes.c_double,
                                             ctypes.c_double, I, ctypes.c_uint64, P, SZ, P]),
         "tadm_probe_breakdown": (I, [P, I, ctypes.POINTER(I64), ctypes.POINTER(ctypes.c_double),
-                                     ctypes.POINTER(ctypes.c_double)]),
+                                     ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double)]),
         "tadm_probe_read": (I, [P, ctypes.POINTER(I64), ctypes.POINTER(ctypes.c_double),
                                 ctypes.POINTER(ctypes.c_double)]),
     }
@@ -391,9 +391,10 @@ class TadmModel:
 
     def tadm_probe_breakdown(self) -> dict:
         n = len(self.EPI_NAMES)
-        L, ms, fl = (ctypes.c_int64 * n)(), (ctypes.c_double * n)(), (ctypes.c_double * n)()
-        _check(self.lib.tadm_probe_breakdown(self.h, n, L, ms, fl), self.h)
-        return {self.EPI_NAMES[k]: {"launches": L[k], "ms": ms[k], "tflops": fl[k] / (ms[k] / 1e3) / 1e12}
+        L, ms, fl, by = (ctypes.c_int64 * n)(), (ctypes.c_double * n)(), (ctypes.c_double * n)(), (ctypes.c_double * n)()
+        _check(self.lib.tadm_probe_breakdown(self.h, n, L, ms, fl, by), self.h)
+        return {self.EPI_NAMES[k]: {"launches": L[k], "ms": ms[k], "flops": fl[k], "bytes": by[k],
+                                    "tflops": fl[k] / (ms[k] / 1e3) / 1e12}
                 for k in range(n) if L[k] > 0}
 
     def tadm_probe_read(self):

@@ -247,6 +247,49 @@ def test_generate_graph_replay_matches_eager(T, block_len):
     assert np.all(runs[0] != m.mask_id) and np.array_equal(runs[0][:, :P], p.cpu().numpy())
 
 
+@pytest.mark.parametrize("block_len", [0, 16])
+def test_graph_dropped_when_workspace_rebound(T, block_len):
+    """A generation captured as a CUDA graph is never replayed on a workspace
+    that has since been replaced: after two calls (eager, capture) and a
+    replay, the caller binds a fresh workspace and frees the old one; the next
+    identical call must run on the new workspace and give the same tokens
+    (block mode keeps its KV context in the workspace, so a stale replay would
+    read freed memory)."""
+    import ctypes
+    m = wl.ModelConfig(**SMALL_BF16)
+    P, G = 16, 48
+    w = wl.Workload("t", m, batch=2, prompt_len=P, gen_len=G, steps_per_block=8 if block_len else 12, K=2,
+                    block_len=block_len)
+    B = 2
+    tm, _ = setup(T, m, B, max(P, block_len) if block_len else P + G, max_ctx=P + G if block_len else 0)
+    p = torch.from_numpy(wl.make_prompts(w, batch=B, seed=4)).cuda()
+    out = torch.empty((B, P + G), dtype=torch.int32, device="cuda")
+    runs = []
+    for _ in range(3):
+        out.fill_(-7)
+        tm.tadm_generate(p, out, G, w.steps_per_block, 2, block_len)
+        tm.tadm_sync_status()
+        runs.append(out.cpu().numpy())
+    n = ctypes.c_size_t()
+    T._check(tm.lib.tadm_workspace_size(tm.h, ctypes.byref(n)), tm.h)
+    fresh = torch.full((n.value,), 0x5A, dtype=torch.uint8, device="cuda")
+    T._check(tm.lib.tadm_bind_workspace(tm.h, fresh.data_ptr(), n.value), tm.h)
+    old = tm.workspace
+    tm.workspace = fresh
+    old.fill_(0xFF)   # the old workspace is garbage from here on, then released
+    torch.cuda.synchronize()
+    del old
+    torch.cuda.empty_cache()
+    for _ in range(3):   # eager on the new workspace, then capture, then replay
+        out.fill_(-7)
+        tm.tadm_generate(p, out, G, w.steps_per_block, 2, block_len)
+        tm.tadm_sync_status()
+        runs.append(out.cpu().numpy())
+    for r in runs[1:]:
+        assert np.array_equal(r, runs[0])
+    assert np.all(runs[0] != m.mask_id)
+
+
 def test_carry_over_and_zero_masking_on_gpu(T):
     m = wl.ModelConfig(**SMALL_BF16)
     w = wl.Workload("t", m, batch=2, prompt_len=16, gen_len=48, steps_per_block=6, K=2)

@@ -85,3 +85,41 @@ def test_reference_arm_runs_on_rank_zero_only():
                         "--warmup", "0"], cwd=ROOT, env=env, capture_output=True, text=True, timeout=120)
     assert r.returncode == 0, r.stderr[-2000:]
     assert r.stdout.strip() == ""
+
+
+def test_bench_spawns_its_own_ranks():
+    """`bench.py --gpus 2` outside torchrun starts two local ranks itself
+    (torch.distributed.run, rendezvous on 127.0.0.1).  Run end to end on CPU
+    through the reference arm: rank 0 prints the one JSON line, rank 1 exits
+    0 without work."""
+    env = {k: v for k, v in os.environ.items() if k not in ("RANK", "LOCAL_RANK", "WORLD_SIZE", "MASTER_ADDR",
+                                                             "MASTER_PORT")}
+    env["CUDA_VISIBLE_DEVICES"] = ""
+    r = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--gpus", "2", "--steps", "1",
+                        "--warmup", "0", "--workload", "tiny", "--cpu-sample-seconds", "1"], cwd=ROOT, env=env,
+                       capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [x for x in r.stdout.splitlines() if x.startswith("{")]
+    assert len(lines) == 1, r.stdout
+    line = json.loads(lines[0])
+    assert line["impl"] == "reference" and line["n_gpus"] == 2 and line["value"] > 0
+    assert line["ms_per_step"] > 0 and line["extrapolated_generation_ms"] > 0
+
+
+def test_bench_refuses_a_mismatched_world_size():
+    """Under torchrun, --gpus must equal WORLD_SIZE; otherwise bench.py fails
+    loudly before any work."""
+    env = dict(os.environ, RANK="0", LOCAL_RANK="0", WORLD_SIZE="3", CUDA_VISIBLE_DEVICES="")
+    r = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--gpus", "2", "--steps", "1",
+                        "--warmup", "0"], cwd=ROOT, env=env, capture_output=True, text=True, timeout=120)
+    assert r.returncode != 0
+    assert "WORLD_SIZE" in r.stderr
+
+
+def test_rank_launch_command():
+    import bench
+    cmd = bench.rank_launch_command(4, ["--gpus", "4", "--steps", "3"], 29555)
+    assert cmd[1:3] == ["-m", "torch.distributed.run"]
+    assert "--nproc-per-node=4" in cmd and "--master-port=29555" in cmd
+    assert cmd[cmd.index("--master-addr") + 1] == "127.0.0.1"
+    assert cmd[-4:] == ["--gpus", "4", "--steps", "3"] and cmd[-5].endswith("bench.py")
