@@ -30,7 +30,15 @@ What it computes (paper section / equation it follows):
   bidirectionally): App. C.1, "Architecture Details".
 * Backbone layer: pre-norm transformer (RMSNorm, RoPE, multi-head attention
   with grouped KV heads, SwiGLU / GeGLU FFN), the layer type the workloads
-  name; the paper treats it as a black box.
+  name; the paper treats it as a black box.  The Post-train backbone is
+  Gemma-3 based (App. C.1 "Architecture Details", which gives no layer
+  details); its Gemma-3 layer details are optional here: local layers with a
+  sliding attention window and global layers with their own RoPE base in a
+  fixed pattern, QK-norm, and sandwich (pre + post) norms around both
+  sub-blocks.  These follow the public Gemma-3 architecture, not the paper,
+  and parity for them is pinned by the special cases listed in the tests
+  (window >= length reduces to full attention, window 1 to the token's own
+  value, scale invariance of normalised projections).
 
 Readings where the paper is silent:
 * sampler P: confidence top-k within the active block; conf = max softmax
@@ -128,12 +136,13 @@ def rope(x: np.ndarray, pos: np.ndarray, theta: float) -> np.ndarray:
 
 
 def attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, q_pos: np.ndarray, k_pos: np.ndarray,
-              causal: bool) -> np.ndarray:
+              causal: bool, window: int = 0) -> np.ndarray:
     """softmax(q k^T / sqrt(hd)) v with grouped KV heads.
 
     q: [Hq, Lq, hd]; k, v: [Hkv, Lk, hd]; query head h reads KV head
-    h // (Hq / Hkv).  causal: key allowed iff k_pos <= q_pos.
-    Returns [Hq, Lq, hd].
+    h // (Hq / Hkv).  causal: key allowed iff k_pos <= q_pos.  window > 0
+    (a local layer of the Gemma-3 backbone): key allowed only if
+    q_pos - k_pos < window as well.  Returns [Hq, Lq, hd].
     """
     Hq, Lq, hd = q.shape
     Hkv = k.shape[0]
@@ -144,6 +153,8 @@ def attention(q: np.ndarray, k: np.ndarray, v: np.ndarray, q_pos: np.ndarray, k_
         s = q[h] @ kh.T / math.sqrt(hd)
         if causal:
             s = np.where(k_pos[None, :] <= q_pos[:, None], s, NEG_INF)
+        if window > 0:
+            s = np.where(q_pos[:, None] - k_pos[None, :] < window, s, NEG_INF)
         s = s - np.max(s, axis=-1, keepdims=True)
         p = np.exp(s)
         p = p / np.sum(p, axis=-1, keepdims=True)
@@ -343,10 +354,38 @@ class Oracle:
         return w
 
     # -- backbone layer (pre-norm) ------------------------------------------
+    def layer_index(self, name: str) -> int:
+        """Position of layer "<net>.<i>." in the whole backbone: the L_S
+        shared layers, then the L_A anchor layers, then the L_D denoiser
+        layers."""
+        net, i = name.split(".")[:2]
+        first = {"shared": 0, "anchor": self.m.n_shared, "denoise": self.m.n_shared + self.m.n_anchor}[net]
+        return first + int(i)
+
+    def layer_kind(self, name: str):
+        """(window, RoPE base) of a layer under the Gemma-3 pattern: layer i
+        is global iff global_every > 0 and (i + 1) % global_every == 0, or
+        global_every == 0.  Local layers see keys less than sliding_window
+        positions back (0: all) with base rope_theta; global layers see every
+        key, with base rope_theta_global (rope_theta when that is 0)."""
+        m = self.m
+        g = getattr(m, "global_every", 0)
+        is_global = g == 0 or (self.layer_index(name) + 1) % g == 0
+        if is_global:
+            tg = getattr(m, "rope_theta_global", 0.0)
+            return 0, (tg if tg > 0 else m.rope_theta)
+        return getattr(m, "sliding_window", 0), m.rope_theta
+
     def layer(self, name: str, x: np.ndarray, pos: np.ndarray, seq: Optional[_Seq], causal: bool,
               keep_kv: bool) -> np.ndarray:
         """x <- x + Wo Attn(RoPE(Q), RoPE(K), V) from RMSNorm(x); then
         x <- x + Wdown (act(Wg n) * (Wu n)) with n = RMSNorm(x).
+
+        Gemma-3 details when the model enables them: QK-norm (RMSNorm over
+        head_dim of each Q and K head, gains q_norm / k_norm, before RoPE);
+        sandwich norms (x <- x + RMSNorm(Wo o) with gain post_attn_norm, and
+        x <- x + RMSNorm(Wdown a) with gain post_ffn_norm); the window and
+        RoPE base of the layer's kind (``layer_kind``).
 
         Keys are the context cached in ``seq`` (committed positions) followed
         by the rows of x.  With ``keep_kv`` the rows' K, V are appended to the
@@ -355,13 +394,17 @@ class Oracle:
         m = self.m
         hd, Hq, Hkv, F = m.head_dim, m.n_heads, m.n_kv_heads, m.ffn
         L = x.shape[0]
+        window, theta = self.layer_kind(name)
         n = rms_norm(x, self.W(name + "attn_norm"), m.norm_eps)
         qkv = linear(n, self.W(name + "wqkv"))
         q = qkv[:, : Hq * hd].reshape(L, Hq, hd).transpose(1, 0, 2)
         k = qkv[:, Hq * hd: (Hq + Hkv) * hd].reshape(L, Hkv, hd).transpose(1, 0, 2)
         v = qkv[:, (Hq + Hkv) * hd:].reshape(L, Hkv, hd).transpose(1, 0, 2)
-        q = rope(q, pos, m.rope_theta)
-        k = rope(k, pos, m.rope_theta)
+        if getattr(m, "qk_norm", False):
+            q = rms_norm(q, self.W(name + "q_norm"), m.norm_eps)
+            k = rms_norm(k, self.W(name + "k_norm"), m.norm_eps)
+        q = rope(q, pos, theta)
+        k = rope(k, pos, theta)
         if seq is not None and name in seq.kv:
             kc, vc = seq.kv[name]
             k_all = np.concatenate([kc, k], axis=1)
@@ -369,13 +412,20 @@ class Oracle:
             k_pos = np.concatenate([np.arange(kc.shape[1]), pos])
         else:
             k_all, v_all, k_pos = k, v, pos
-        o = attention(q, k_all, v_all, pos, k_pos, causal)
-        x = x + linear(o.transpose(1, 0, 2).reshape(L, Hq * hd), self.W(name + "wo"))
+        o = attention(q, k_all, v_all, pos, k_pos, causal, window)
+        sandwich = getattr(m, "sandwich_norm", False)
+        a = linear(o.transpose(1, 0, 2).reshape(L, Hq * hd), self.W(name + "wo"))
+        if sandwich:
+            a = rms_norm(a, self.W(name + "post_attn_norm"), m.norm_eps)
+        x = x + a
         n = rms_norm(x, self.W(name + "ffn_norm"), m.norm_eps)
         gu = linear(n, self.W(name + "wgu"))
         g, u = gu[:, :F], gu[:, F:]
         act = silu(g) if m.glu == "swiglu" else gelu_tanh(g)
-        x = x + linear(act * u, self.W(name + "wdown"))
+        f = linear(act * u, self.W(name + "wdown"))
+        if sandwich:
+            f = rms_norm(f, self.W(name + "post_ffn_norm"), m.norm_eps)
+        x = x + f
         if keep_kv and seq is not None:
             if name in seq.kv:
                 kc, vc = seq.kv[name]

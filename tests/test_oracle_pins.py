@@ -848,3 +848,194 @@ def test_encoder_pass_is_S_A_fusion_D():
         for name in s1.kv:
             np.testing.assert_allclose(s1.kv[name][0], s2.kv[name][0], rtol=1e-12, atol=1e-14)
             np.testing.assert_allclose(s1.kv[name][1], s2.kv[name][1], rtol=1e-12, atol=1e-14)
+
+
+# --------------------------------------------------------------------------- Gemma-3 layer details
+def test_window_attention_brute_force_and_library():
+    """Sliding-window attention (the local layers): a key at position j is
+    visible to a query at position p iff p - j < W (and j <= p when causal).
+    Checked against scalar loops with that rule written out, and against
+    torch's SDPA with the same boolean mask."""
+    Hq, Hkv, Lq, Lk, hd = 2, 1, 4, 9, 4
+    q = rng.standard_normal((Hq, Lq, hd))
+    k = rng.standard_normal((Hkv, Lk, hd))
+    v = rng.standard_normal((Hkv, Lk, hd))
+    qp, kp = np.array([5, 6, 7, 8]), np.arange(Lk)
+    for causal in (False, True):
+        for W in (1, 2, 3, 6):
+            out = O.attention(q, k, v, qp, kp, causal, window=W)
+            vis = [[(not causal or kp[j] <= qp[i]) and qp[i] - kp[j] < W for j in range(Lk)] for i in range(Lq)]
+            for h in range(Hq):
+                for i in range(Lq):
+                    w = [math.exp(sum(q[h, i, t] * k[0, j, t] for t in range(hd)) / 2.0) if vis[i][j] else 0.0
+                         for j in range(Lk)]
+                    for t in range(hd):
+                        assert abs(out[h, i, t] - sum(w[j] * v[0, j, t] for j in range(Lk)) / sum(w)) < 1e-12
+            mask = torch.from_numpy(np.array(vis))
+            ref = Fn.scaled_dot_product_attention(torch.from_numpy(q), torch.from_numpy(k).repeat(Hq, 1, 1),
+                                                  torch.from_numpy(v).repeat(Hq, 1, 1), attn_mask=mask)
+            np.testing.assert_allclose(out, ref.numpy(), rtol=1e-12, atol=1e-12)
+
+
+def test_window_special_cases():
+    """A window at least as long as every query-key distance is no window; a
+    window of 1 with causal attention leaves each query only its own key, so
+    the output is that position's value."""
+    Hq, Hkv, L, hd = 4, 2, 7, 8
+    q = rng.standard_normal((Hq, L, hd))
+    k = rng.standard_normal((Hkv, L, hd))
+    v = rng.standard_normal((Hkv, L, hd))
+    pos = np.arange(L) + 11
+    for causal in (False, True):
+        np.testing.assert_allclose(O.attention(q, k, v, pos, pos, causal, window=L),
+                                   O.attention(q, k, v, pos, pos, causal), rtol=0, atol=0)
+    own = O.attention(q, k, v, pos, pos, True, window=1)
+    np.testing.assert_allclose(own, np.repeat(v, Hq // Hkv, axis=0), rtol=1e-14, atol=1e-14)
+    # a non-causal window looks ahead without bound and back by less than W
+    out = O.attention(q, k, v, pos, pos, False, window=1)
+    last = O.attention(q[:, -1:], k, v, pos[-1:], pos, False, window=1)
+    np.testing.assert_allclose(out[:, -1:], last, rtol=1e-14, atol=1e-14)
+    np.testing.assert_allclose(last[:, 0], np.repeat(v, Hq // Hkv, axis=0)[:, -1], rtol=1e-14, atol=1e-14)
+
+
+def test_gemma3_layer_pattern():
+    """Five local layers per global one over the whole backbone (S, A, D):
+    with 2 + 54 + 6 layers and global_every 6 the global layers are 5, 11,
+    ..., 59; local layers take the window and the local RoPE base, global
+    ones no window and the global base."""
+    m = wl.POSTTRAIN_G3
+    o = O.Oracle(m, {})
+    names = ([f"shared.{i}." for i in range(m.n_shared)] + [f"anchor.{i}." for i in range(m.n_anchor)] +
+             [f"denoise.{i}." for i in range(m.n_denoise)])
+    assert [o.layer_index(n) for n in names] == list(range(62))
+    kinds = [o.layer_kind(n) for n in names]
+    assert [i for i, kd in enumerate(kinds) if kd[0] == 0] == [5, 11, 17, 23, 29, 35, 41, 47, 53, 59]
+    assert {kd for kd in kinds} == {(1024, 1e4), (0, 1e6)}
+    assert O.Oracle(wl.POSTTRAIN, {}).layer_kind("anchor.3.") == (0, 1e4)     # no pattern: all global
+
+
+def _g3_oracle(eps=1e-6, **kw):
+    base = dict(qk_norm=True, sandwich_norm=True, sliding_window=3, global_every=2, rope_theta_global=5e5,
+                norm_eps=eps, n_shared=1)
+    base.update(kw)
+    return tiny_oracle(**base)
+
+
+def test_qk_norm_removes_the_scale_of_q_and_k():
+    """With QK-norm (and eps 0) scaling the Q or K rows of W_qkv by a positive
+    constant leaves the layer unchanged; without it the output moves."""
+    for qk in (True, False):
+        o = _g3_oracle(eps=0.0, qk_norm=qk)
+        m = o.m
+        x = rng.standard_normal((6, m.d_model))
+        ref = o.layer("anchor.0.", x, np.arange(6), None, False, False)
+        w = dict(o._raw)
+        wqkv = o.W("anchor.0.wqkv").copy()
+        nq = m.n_heads * m.head_dim
+        wqkv[:nq] *= 4.0            # powers of two: the float32 copy stays exact
+        wqkv[nq:nq + m.n_kv_heads * m.head_dim] *= 0.5
+        w["anchor.0.wqkv"] = wqkv.astype(np.float32)
+        got = O.Oracle(m, w).layer("anchor.0.", x, np.arange(6), None, False, False)
+        if qk:
+            np.testing.assert_allclose(got, ref, rtol=1e-11, atol=1e-11)
+        else:
+            assert not np.allclose(got, ref, rtol=1e-3)
+
+
+def test_qk_norm_comes_before_rope():
+    """RoPE keeps attention relative (a common position shift changes
+    nothing) only if the per-dimension QK-norm gains act before the rotation;
+    the gains here are far from uniform."""
+    o = _g3_oracle(affine_std=0.5, sliding_window=0)
+    x = rng.standard_normal((6, o.m.d_model))
+    for name in ("anchor.0.", "anchor.1."):        # a local and a global layer
+        a = o.layer(name, x, np.arange(6), None, False, False)
+        b = o.layer(name, x, np.arange(6) + 29, None, False, False)
+        np.testing.assert_allclose(a, b, rtol=1e-10, atol=1e-10)
+
+
+def test_sandwich_norms():
+    """Sandwich norms: zero post-norm gains silence both sub-blocks (the layer
+    is the identity), and with eps 0 scaling W_o or W_down by a positive
+    constant leaves the layer unchanged."""
+    o = _g3_oracle(eps=0.0)
+    m = o.m
+    x = rng.standard_normal((5, m.d_model))
+    w = dict(o._raw)
+    w["anchor.0.post_attn_norm"] = np.zeros(m.d_model, np.float32)
+    w["anchor.0.post_ffn_norm"] = np.zeros(m.d_model, np.float32)
+    np.testing.assert_array_equal(O.Oracle(m, w).layer("anchor.0.", x, np.arange(5), None, False, False), x)
+    ref = o.layer("anchor.0.", x, np.arange(5), None, False, False)
+    w = dict(o._raw)
+    w["anchor.0.wo"] = (o.W("anchor.0.wo") * 8.0).astype(np.float32)
+    w["anchor.0.wdown"] = (o.W("anchor.0.wdown") * 0.125).astype(np.float32)
+    np.testing.assert_allclose(O.Oracle(m, w).layer("anchor.0.", x, np.arange(5), None, False, False), ref,
+                               rtol=1e-11, atol=1e-11)
+    # only the attention branch silenced: x + RMSNorm(FFN(RMSNorm(x))) has unit-RMS increments
+    w = dict(o._raw)
+    w["anchor.0.post_attn_norm"] = np.zeros(m.d_model, np.float32)
+    got = O.Oracle(m, w).layer("anchor.0.", x, np.arange(5), None, False, False)
+    inc = (got - x) / o.W("anchor.0.post_ffn_norm")
+    np.testing.assert_allclose(np.sqrt(np.mean(inc * inc, axis=-1)), 1.0, rtol=1e-12)
+
+
+def test_global_layers_take_the_global_rope_base():
+    """A backbone whose layers are all global with base rope_theta_global
+    equals one without the pattern whose base is that value; the local
+    layers of a patterned backbone use rope_theta."""
+    a = _g3_oracle(global_every=1, sliding_window=2, rope_theta=1e4, rope_theta_global=5e5)
+    b = O.Oracle(tiny_model(**{**a.m.__dict__, "global_every": 0, "sliding_window": 0, "rope_theta": 5e5,
+                              "rope_theta_global": 0.0}), a._raw)
+    x = rng.standard_normal((6, a.m.d_model))
+    for name in ("shared.0.", "anchor.1."):
+        np.testing.assert_allclose(a.layer(name, x, np.arange(6) + 3, None, True, False),
+                                   b.layer(name, x, np.arange(6) + 3, None, True, False), rtol=0, atol=0)
+    c = _g3_oracle(global_every=2, sliding_window=6)   # anchor.0 is layer 1: global; shared.0 is layer 0: local
+    d = O.Oracle(tiny_model(**{**c.m.__dict__, "global_every": 0, "sliding_window": 0,
+                              "rope_theta_global": 0.0}), c._raw)
+    np.testing.assert_allclose(c.layer("shared.0.", x, np.arange(6), None, True, False),
+                               d.layer("shared.0.", x, np.arange(6), None, True, False), rtol=0, atol=0)
+    assert not np.allclose(c.layer("anchor.0.", x, np.arange(6), None, True, False),
+                           d.layer("anchor.0.", x, np.arange(6), None, True, False))
+
+
+def test_window_over_the_kv_context_equals_one_causal_pass():
+    """Block mode with local layers: prefill + commit through the KV cache
+    equals one causal pass over the concatenated rows, the window counting
+    positions across the committed context."""
+    o = _g3_oracle(sliding_window=3)
+    z = rng.integers(0, 63, size=11).astype(np.int32)
+    s1 = o.new_session(1)[0]
+    o._fresh_pass(s1, z[:7])
+    o._fresh_pass(s1, z[7:])
+    s2 = o.new_session(1)[0]
+    o._fresh_pass(s2, z)
+    for name in s1.kv:
+        np.testing.assert_allclose(s1.kv[name][0], s2.kv[name][0], rtol=1e-10, atol=1e-12)
+        np.testing.assert_allclose(s1.kv[name][1], s2.kv[name][1], rtol=1e-10, atol=1e-12)
+    # and the window changes the result (it is not silently ignored)
+    s3 = O.Oracle(tiny_model(**{**o.m.__dict__, "sliding_window": 0}), o._raw).new_session(1)[0]
+    O.Oracle(tiny_model(**{**o.m.__dict__, "sliding_window": 0}), o._raw)._fresh_pass(s3, z)
+    assert not np.allclose(s3.kv["anchor.1."][0], s2.kv["anchor.1."][0])
+
+
+def test_qk_norm_gains_belong_to_their_heads():
+    """Zero Q-norm gains (with non-zero K-norm gains) zero every query and
+    make attention uniform over the visible keys, exactly like zero Q rows of
+    W_qkv; zero K-norm gains do the same as zero K rows.  A swap of the two
+    gain vectors breaks both equalities."""
+    o = _g3_oracle(affine_std=0.5, sandwich_norm=False)
+    m = o.m
+    nq, nk = m.n_heads * m.head_dim, m.n_kv_heads * m.head_dim
+    x = rng.standard_normal((6, m.d_model))
+    for gain, rows in (("q_norm", slice(0, nq)), ("k_norm", slice(nq, nq + nk))):
+        a = dict(o._raw)
+        a["anchor.0." + gain] = np.zeros(m.head_dim, np.float32)
+        b = dict(o._raw)
+        wqkv = o.W("anchor.0.wqkv").copy()
+        wqkv[rows] = 0.0
+        b["anchor.0.wqkv"] = wqkv.astype(np.float32)
+        ya = O.Oracle(m, a).layer("anchor.0.", x, np.arange(6), None, False, False)
+        yb = O.Oracle(m, b).layer("anchor.0.", x, np.arange(6), None, False, False)
+        np.testing.assert_allclose(ya, yb, rtol=1e-12, atol=1e-12)
+        assert not np.allclose(ya, o.layer("anchor.0.", x, np.arange(6), None, False, False))

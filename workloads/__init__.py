@@ -144,6 +144,18 @@ class ModelConfig:
     tied_lm_head: bool = False
     norm_eps: float = 1e-6
     rope_theta: float = 10000.0
+    # Gemma-3 backbone details (off by default): local layers attend to keys
+    # less than `sliding_window` positions back (0: unbounded); layer i of the
+    # whole backbone (S, then A, then D) is global iff global_every > 0 and
+    # (i + 1) % global_every == 0, and every layer is global when
+    # global_every == 0; global layers use rope_theta_global (0: rope_theta);
+    # qk_norm: RMSNorm over head_dim of every Q and K head before RoPE;
+    # sandwich_norm: RMSNorm of each sub-block's output before the residual add
+    sliding_window: int = 0
+    global_every: int = 0
+    rope_theta_global: float = 0.0
+    qk_norm: bool = False
+    sandwich_norm: bool = False
 
     @property
     def mask_id(self) -> int:
@@ -182,6 +194,11 @@ BLOCK = ModelConfig(vocab=128000, d_model=2048, n_heads=16, n_kv_heads=8, head_d
 POSTTRAIN = ModelConfig(vocab=262144, d_model=5376, n_heads=32, n_kv_heads=16, head_dim=128, ffn=21504,
                         glu="geglu", n_shared=2, n_anchor=54, n_denoise=6, fusion="paired_attn",
                         tied_lm_head=True)
+# the same backbone with the Gemma-3 layer details: 5 local layers (1024-key
+# sliding window, RoPE base 1e4) per global layer (RoPE base 1e6), QK-norm and
+# sandwich norms
+POSTTRAIN_G3 = replace(POSTTRAIN, sliding_window=1024, global_every=6, rope_theta_global=1e6, qk_norm=True,
+                       sandwich_norm=True)
 
 WORKLOADS: Dict[str, Workload] = {
     "tiny": Workload("tiny", TINY, batch=1, prompt_len=32, gen_len=96, steps_per_block=32, K=4,
@@ -194,6 +211,8 @@ WORKLOADS: Dict[str, Workload] = {
                           steps_per_block=32, K=4, block_len=32, k_sweep=(1, 4)),
     "sweep": Workload("sweep", BLOCK, batch=32, prompt_len=512, gen_len=2048, steps_per_block=16, K=4,
                       block_len=32, k_sweep=(1, 2, 4, 8, 16)),
+    "posttrain_g3": Workload("posttrain_g3", POSTTRAIN_G3, batch=8, prompt_len=1024, gen_len=1024,
+                             steps_per_block=32, K=4, block_len=32, k_sweep=(1, 4)),
     # the post-training sampler settings of App. C.1: one 256-token canvas after the prompt, 48 reverse
     # steps, anchor refresh K in {1, 2, 3}
     "posttrain_canvas": Workload("posttrain_canvas", POSTTRAIN, batch=8, prompt_len=256, gen_len=256,
@@ -233,11 +252,19 @@ def weight_specs(m: ModelConfig) -> List[TensorSpec]:
             specs += [
                 TensorSpec(p + "attn_norm", (d,), "gain"),
                 TensorSpec(p + "wqkv", (nqkv, d), "matrix"),      # rows: Q heads, K heads, V heads
-                TensorSpec(p + "wo", (d, m.n_heads * hd), "matrix"),
+            ]
+            if m.qk_norm:
+                specs += [TensorSpec(p + "q_norm", (hd,), "gain"), TensorSpec(p + "k_norm", (hd,), "gain")]
+            specs.append(TensorSpec(p + "wo", (d, m.n_heads * hd), "matrix"))
+            if m.sandwich_norm:
+                specs.append(TensorSpec(p + "post_attn_norm", (d,), "gain"))
+            specs += [
                 TensorSpec(p + "ffn_norm", (d,), "gain"),
                 TensorSpec(p + "wgu", (2 * F, d), "matrix"),      # rows: gate (F), then up (F)
                 TensorSpec(p + "wdown", (d, F), "matrix"),
             ]
+            if m.sandwich_norm:
+                specs.append(TensorSpec(p + "post_ffn_norm", (d,), "gain"))
     if m.fusion == "gated_mlp":
         specs += [
             TensorSpec("fusion.ln_c.w", (d,), "gain"), TensorSpec("fusion.ln_c.b", (d,), "bias"),
