@@ -76,6 +76,22 @@ typedef enum {
  *  dtype:   0 = fp32 weights and activations, 1 = bf16 weights and GEMM
  *           operands (fp32 accumulation, fp32 residual stream).
  *  tied_lm_head: 1 = the output head reuses the embedding matrix.
+ *  Gemma-3 layer details of the Post-train backbone (App. C.1 names a
+ *  Gemma-3 based model and gives no layer details; these follow the public
+ *  Gemma-3 architecture; all zero = a plain pre-norm layer):
+ *  sliding_window: W > 0: a query at position p of a local layer sees only
+ *           keys at positions j with p - j < W (besides the causal rule of
+ *           prefill / commit passes); 0 = local layers see every key.
+ *  global_every: g > 0: layer i of the whole backbone (the L_S shared, then
+ *           the L_A anchor, then the L_D denoiser layers, 0-based) is global
+ *           iff (i + 1) % g == 0, otherwise local; g = 0: every layer global.
+ *           Global layers see every key.
+ *  qk_norm: 1 = RMSNorm over head_dim of every Q and K head (gains q_norm,
+ *           k_norm of the layer), before RoPE.
+ *  sandwich_norm: 1 = each sub-block's output is RMS-normalised (gains
+ *           post_attn_norm, post_ffn_norm) before the residual add.
+ *  rope_theta_global: RoPE base of global layers (0 = rope_theta); local
+ *           layers use rope_theta.
  */
 typedef struct {
   int32_t vocab, d_model, n_heads, n_kv_heads, head_dim, ffn;
@@ -86,6 +102,8 @@ typedef struct {
   int32_t dtype;
   int32_t tied_lm_head;
   float norm_eps, rope_theta;
+  int32_t sliding_window, global_every, qk_norm, sandwich_norm;
+  float rope_theta_global;
 } tadm_config;
 
 typedef struct tadm_handle tadm_handle;
@@ -98,8 +116,10 @@ typedef struct tadm_handle tadm_handle;
  *
  * Inventory: "embed" [V, d]; then for net in (shared, anchor, denoise) and
  * each layer i: "<net>.<i>.attn_norm" [d], ".wqkv" [(Hq + 2 Hkv) hd, d]
- * (rows: Q heads, K heads, V heads), ".wo" [d, Hq hd], ".ffn_norm" [d],
- * ".wgu" [2F, d] (rows: gate, then up), ".wdown" [d, F]; then the fusion
+ * (rows: Q heads, K heads, V heads), with qk_norm ".q_norm" [hd] and
+ * ".k_norm" [hd], ".wo" [d, Hq hd], with sandwich_norm ".post_attn_norm"
+ * [d], ".ffn_norm" [d], ".wgu" [2F, d] (rows: gate, then up), ".wdown"
+ * [d, F], with sandwich_norm ".post_ffn_norm" [d]; then the fusion
  * parameters; "final_norm" [d]; "lm_head" [V, d] unless tied.
  */
 /* Number of weight tensors of cfg, or -1 if cfg is invalid. */
@@ -326,13 +346,15 @@ TADM_API tadm_status tadm_head_confidence_static(const void* x, const void* w, i
 
 /* softmax(Q K^T / sqrt(hd)) V for queries at positions ctx .. ctx+rows-1 over
  * keys 0 .. ctx+rows-1 (keys < ctx always visible; the rest bidirectional,
- * or causal if `causal`).  dtype 1: bf16, 0: fp32.
+ * or causal if `causal`).  window > 0 (a local layer): a query at position p
+ * sees only keys j with p - j < window as well; 0 = no window.  dtype 1:
+ * bf16, 0: fp32.
  * q: [batch, n_heads, rows, hd]; k: [batch, n_kv_heads, kv_stride, hd];
  * v transposed: [batch, n_kv_heads, hd, kv_stride]; o: [batch*rows, n_heads*hd].
  * K and V entries at positions >= ctx + rows must hold finite values. */
 TADM_API tadm_status tadm_attention(const void* q, const void* k, const void* v, void* o, int batch,
                            int n_heads, int n_kv_heads, int head_dim, int rows, int ctx,
-                           int kv_stride, int causal, int dtype, tadm_stream stream);
+                           int kv_stride, int causal, int window, int dtype, tadm_stream stream);
 
 /* ------------------------------------------------------------ ReMDM sampler --
  * The paper's Pretraining sampler in place of the confidence top-k: the

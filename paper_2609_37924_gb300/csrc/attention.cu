@@ -4,7 +4,10 @@
 // ctx .. ctx+rows-1; keys are positions 0 .. ctx+rows-1 of the layer's K/V
 // buffers.  Keys below ctx (committed context) are always visible; the active
 // rows see each other bidirectionally, or causally for commit / prefill
-// passes.  Query head h reads KV head h / (n_heads / n_kv_heads).
+// passes.  The local layers of a Gemma-3 backbone add a sliding window: a
+// query at position p sees only keys j with p - j < window (the tcgen05 path
+// skips the key tiles below its rows' windows).  Query head h reads KV head
+// h / (n_heads / n_kv_heads).
 // Layouts: q [B, Hq, rows, hd]; k [B, Hkv, kv_stride, hd];
 // v transposed [B, Hkv, hd, kv_stride]; o [B*rows, Hq*hd].
 //
@@ -58,6 +61,7 @@ struct AttnTcCfg {
 struct AttnTcArgs {
   const bf16* q;
   int rows, ctx, kv_len, n_heads, n_kv_heads, causal;
+  int window;        // > 0: keys j < qpos - window + 1 are hidden (sliding window)
   float scale_log2;
   bf16* o;
   int n_vtiles, splits, tiles_per_split;
@@ -105,8 +109,11 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD, TKV>::MIN_BLOCKS)
   const int v_last = min(m0 + TQ, n_virt) - 1;
   const int r_max = (m0 / args.rows != v_last / args.rows) ? args.rows - 1 : v_last % args.rows;
   const int kv_end = args.causal ? min(args.kv_len, args.ctx + r_max + 1) : args.kv_len;
-  const int t0 = split * args.tiles_per_split;
-  const int n_tiles = max(0, min((kv_end + TKV - 1) / TKV, t0 + args.tiles_per_split) - t0);
+  // sliding window: no row of this CTA sees a key below the smallest row's window start
+  const int r_min = (m0 / args.rows != v_last / args.rows) ? 0 : m0 % args.rows;
+  const int kv_begin = args.window > 0 ? max(0, args.ctx + r_min - args.window + 1) : 0;
+  const int t0 = max(split * args.tiles_per_split, kv_begin / TKV);   // first tile of this CTA
+  const int n_tiles = max(0, min((kv_end + TKV - 1) / TKV, (split + 1) * args.tiles_per_split) - t0);
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 128);            // the softmax threads stage Q
@@ -234,10 +241,12 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD, TKV>::MIN_BLOCKS)
       if (!warp_wait_bounded(s_full, i & 1, abort_flag, args.status)) { ok = false; break; }
       tc_fence_after();
       const int key0 = (t0 + i) * TKV;
-      // keys visible to this row: key < kv_hi (kv_end, or the causal bound)
+      // keys visible to this row: kv_lo <= key < kv_hi (kv_end, or the causal bound; the window start)
       const int kv_hi = args.causal ? min(kv_end, qpos + 1) : kv_end;
-      const int lim = kv_hi - key0;                                   // visible keys of this tile
-      const bool masked = __any_sync(0xffffffffu, lim < TKV);         // warp-uniform path choice
+      const int kv_lo = args.window > 0 ? qpos - args.window + 1 : 0;
+      const int lim = kv_hi - key0;                                   // visible keys of this tile: [lo, lim)
+      const int lo = kv_lo - key0;
+      const bool masked = __any_sync(0xffffffffu, lim < TKV || lo > 0);   // warp-uniform path choice
       // pass 1: row max over the tile, 64 columns per TMEM round trip
       float mxa[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};   // independent chains
 #pragma unroll
@@ -250,8 +259,9 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD, TKV>::MIN_BLOCKS)
         if (masked) {
 #pragma unroll
           for (int k = 0; k < 32; ++k)
-            mxa[k & 3] = fmax3(mxa[k & 3], 64 * c + k < lim ? __uint_as_float(ra[k]) : -INFINITY,
-                               64 * c + 32 + k < lim ? __uint_as_float(rb[k]) : -INFINITY);
+            mxa[k & 3] = fmax3(mxa[k & 3],
+                               64 * c + k < lim && 64 * c + k >= lo ? __uint_as_float(ra[k]) : -INFINITY,
+                               64 * c + 32 + k < lim && 64 * c + 32 + k >= lo ? __uint_as_float(rb[k]) : -INFINITY);
         } else {
 #pragma unroll
           for (int k = 0; k < 32; ++k) mxa[k & 3] = fmax3(mxa[k & 3], __uint_as_float(ra[k]), __uint_as_float(rb[k]));
@@ -296,8 +306,8 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD, TKV>::MIN_BLOCKS)
           f2_unpack(f2_fma(f2_pack(__uint_as_float(ra[k]), __uint_as_float(ra[k + 1])), sc2, negm2), x0, x1);
           float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
           if (masked) {
-            p0 = 32 * c + k < lim ? p0 : 0.0f;
-            p1 = 32 * c + k + 1 < lim ? p1 : 0.0f;
+            p0 = 32 * c + k < lim && 32 * c + k >= lo ? p0 : 0.0f;
+            p1 = 32 * c + k + 1 < lim && 32 * c + k + 1 >= lo ? p1 : 0.0f;
           }
           ps2[(k >> 1) & 1] = f2_add(ps2[(k >> 1) & 1], f2_pack(p0, p1));
           __nv_bfloat162 t = __floats2bfloat162_rn(p0, p1);
@@ -480,7 +490,9 @@ const char* launch_tc(const AttnCall& a, cudaStream_t s) {
   // idle SMs): every split keeps >= 3 tiles and its fp32 partials fit the
   // caller's scratch
   int splits = 1;
-  if (a.part && a.part_bytes > 0) {
+  // a window that hides keys leaves each CTA only its window's tiles: no key splits then
+  const bool window_cuts = a.window > 0 && a.window < kv_len;
+  if (a.part && a.part_bytes > 0 && !window_cuts) {
     const int slots = C::MIN_BLOCKS * n_sms;
     const size_t per_split = static_cast<size_t>(a.batch) * a.n_kv_heads * n_virt * (HD + 2) * sizeof(float);
     splits = std::min(std::min(slots / base, kv_tiles / 3), 8);
@@ -491,7 +503,7 @@ const char* launch_tc(const AttnCall& a, cudaStream_t s) {
   splits = (kv_tiles + tps - 1) / tps;
   float* part_o = static_cast<float*>(a.part);
   float2* part_ml = reinterpret_cast<float2*>(part_o + static_cast<size_t>(splits) * a.batch * a.n_kv_heads * n_virt * HD);
-  AttnTcArgs args{static_cast<const bf16*>(a.q), a.rows, a.ctx, kv_len, a.n_heads, a.n_kv_heads, a.causal,
+  AttnTcArgs args{static_cast<const bf16*>(a.q), a.rows, a.ctx, kv_len, a.n_heads, a.n_kv_heads, a.causal, a.window,
                   1.4426950408889634f / sqrtf(static_cast<float>(HD)), static_cast<bf16*>(a.o),
                   n_vtiles, splits, tps, part_o, part_ml, a.status};
   dim3 grid(n_vtiles * splits, a.n_kv_heads, a.batch);
@@ -541,7 +553,7 @@ template <int HD>
 __global__ void __launch_bounds__(128) attn_bf16_kernel(const bf16* __restrict__ q, const bf16* __restrict__ k,
                                                         const bf16* __restrict__ vt, bf16* __restrict__ o,
                                                         int n_heads, int n_kv_heads, int rows, int ctx,
-                                                        int kv_stride, int causal, float scale_log2) {
+                                                        int kv_stride, int causal, int window, float scale_log2) {
   pdl_enter();
   constexpr int LD = HD + 8;   // padded smem row of Q / K (bf16)
   constexpr int LDV = AN + 8;  // padded smem row of V^T (one head dim, AN keys)
@@ -647,7 +659,7 @@ __global__ void __launch_bounds__(128) attn_bf16_kernel(const bf16* __restrict__
       for (int e = 0; e < 4; ++e) {
         const int key = n0 + j * 8 + 2 * t4 + (e & 1);
         const int qp = qpos_r[e >> 1];
-        const bool ok = key < kv_end && (!causal || key < ctx || key <= qp);
+        const bool ok = key < kv_end && (!causal || key < ctx || key <= qp) && (window <= 0 || qp - key < window);
         s[j][e] = ok ? s[j][e] * scale_log2 : -INFINITY;
         tmax[e >> 1] = fmaxf(tmax[e >> 1], s[j][e]);
       }
@@ -726,7 +738,7 @@ template <int HD>
 __global__ void __launch_bounds__(128) attn_f32_kernel(const float* __restrict__ q, const float* __restrict__ k,
                                                        const float* __restrict__ vt, float* __restrict__ o,
                                                        int n_heads, int n_kv_heads, int rows, int ctx,
-                                                       int kv_stride, int causal, float scale) {
+                                                       int kv_stride, int causal, int window, float scale) {
   pdl_enter();
   constexpr int PL = HD / 32;
   const int lane = threadIdx.x & 31;
@@ -742,8 +754,9 @@ __global__ void __launch_bounds__(128) attn_f32_kernel(const float* __restrict__
   for (int i = 0; i < PL; ++i) { qv[i] = qr[lane + 32 * i]; acc[i] = 0.0f; }
   const int qpos = ctx + row;
   const int kv_end = causal ? qpos + 1 : ctx + rows;
+  const int kv_lo = window > 0 ? max(0, qpos - window + 1) : 0;   // sliding window start
   float m = -INFINITY, l = 0.0f;
-  for (int j = 0; j < kv_end; ++j) {
+  for (int j = kv_lo; j < kv_end; ++j) {
     float d = 0.0f;
 #pragma unroll
     for (int i = 0; i < PL; ++i) d += qv[i] * kb[static_cast<size_t>(j) * HD + lane + 32 * i];
@@ -776,7 +789,8 @@ cudaError_t launch_bf16(const AttnCall& a, cudaStream_t s) {
   const float scale_log2 = 1.4426950408889634f / sqrtf(static_cast<float>(HD));
   launch_pdl(attn_bf16_kernel<HD>, grid, 128, smem, s, static_cast<const bf16*>(a.q), static_cast<const bf16*>(a.k),
                                                static_cast<const bf16*>(a.v), static_cast<bf16*>(a.o), a.n_heads,
-                                               a.n_kv_heads, a.rows, a.ctx, a.kv_stride, a.causal, scale_log2);
+                                               a.n_kv_heads, a.rows, a.ctx, a.kv_stride, a.causal, a.window,
+                                               scale_log2);
   return cudaGetLastError();
 }
 
@@ -785,7 +799,7 @@ cudaError_t launch_f32(const AttnCall& a, cudaStream_t s) {
   dim3 grid((a.rows + 3) / 4, a.n_heads, a.batch);
   launch_pdl(attn_f32_kernel<HD>, grid, 128, 0, s, static_cast<const float*>(a.q), static_cast<const float*>(a.k),
                                            static_cast<const float*>(a.v), static_cast<float*>(a.o), a.n_heads,
-                                           a.n_kv_heads, a.rows, a.ctx, a.kv_stride, a.causal,
+                                           a.n_kv_heads, a.rows, a.ctx, a.kv_stride, a.causal, a.window,
                                            1.0f / sqrtf(static_cast<float>(HD)));
   return cudaGetLastError();
 }

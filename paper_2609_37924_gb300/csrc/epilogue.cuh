@@ -12,7 +12,7 @@ namespace tadm {
 enum EpiKind : int {
   EPI_STORE = 0,     // out = acc
   EPI_RESID = 1,     // resid += acc (+ bias)
-  EPI_QKV = 2,       // split into Q / K / V heads, optional RoPE, K and V^T into the cache
+  EPI_QKV = 2,       // split into Q / K / V heads, optional QK-norm and RoPE, K and V^T into the cache
   EPI_GLU = 3,       // out = act(gate) * up (gate and up are the two halves of the tile)
   EPI_FUSION1 = 4,   // [g | hidden] = [sigmoid(acc + b) | GELU(acc + b)]
   EPI_FUSION2 = 5,   // out = h + g * (acc + b)
@@ -39,6 +39,10 @@ struct EpiParams {
   int R, ctx, kv_stride, n_heads, n_kv_heads, head_dim, rope;
   const float2* rope_tab;   // [head_dim / 2][n_pos] = (cos, sin): a warp's consecutive positions read consecutive entries
   int rope_npos;
+  // EPI_QKV with QK-norm (Gemma-3 layers): RMSNorm over head_dim of every Q / K head before RoPE,
+  // gains [head_dim] in the weights' type (bias_bf16); null: no QK-norm
+  const void *q_gain, *k_gain;
+  float qk_eps;
   // EPI_GLU
   int glu;                  // 0 SiLU, 1 tanh-GELU
   // EPI_FUSION1 / EPI_ADD
@@ -402,9 +406,26 @@ __device__ __forceinline__ void epilogue_row(const EpiParams& p, int m, int n_bl
         vt_off = (static_cast<size_t>(b) * p.n_kv_heads + head) * hd * p.kv_stride + pos;
       }
       const bool ok = row_ok && nb < p.N;
+      // QK-norm: 1 / RMS of this row's head from a first pass over its chunks
+      // (the chunks are read again below; the region is uniform across the warp)
+      const void* qk_gain = region == 0 ? p.q_gain : (region == 1 ? p.k_gain : nullptr);
+      float qk_inv = 1.0f;
+      if (qk_gain) {
+        float ss = 0.0f;
+        for (int c2 = 0; c2 < hd / 32; ++c2) {
+          src.load((hh * hd) / 32 + c2, v);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) ss = fmaf(v[i], v[i], ss);
+        }
+        qk_inv = rsqrtf(ss / static_cast<float>(hd) + p.qk_eps);
+      }
       if (hd == 32) {  // rotate-half pairs (i, i + 16) inside one chunk
         src.load(hh, v);
         if (!ok) continue;
+        if (qk_gain) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v[i] *= qk_inv * ld_param(qk_gain, p.bias_bf16, i);
+        }
         if (p.rope && region < 2) {
           const float2* tab = p.rope_tab + pos;
 #pragma unroll
@@ -428,6 +449,13 @@ __device__ __forceinline__ void epilogue_row(const EpiParams& p, int m, int n_bl
         src.load(ca, v);
         src.load(cb, w);
         if (!ok) continue;
+        if (qk_gain) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            v[i] *= qk_inv * ld_param(qk_gain, p.bias_bf16, 32 * j2 + i);
+            w[i] *= qk_inv * ld_param(qk_gain, p.bias_bf16, hd / 2 + 32 * j2 + i);
+          }
+        }
         if (p.rope && region < 2) {
           const float2* tab = p.rope_tab + static_cast<size_t>(32 * j2) * p.rope_npos + pos;
 #pragma unroll

@@ -63,6 +63,7 @@ struct AttnCall {
   int* status;   // device status word (may be null)
   void* part = nullptr;      // optional fp32 scratch for split-key partials (16-byte aligned)
   size_t part_bytes = 0;
+  int window = 0;            // > 0: a query at position p sees only keys j with p - j < window
 };
 const char* attention(const AttnCall& a, cudaStream_t s);
 
@@ -85,6 +86,10 @@ const char* ln_pair_rows(const float* c, const float* h, int M, int d, const voi
 const char* layernorm_rows(const float* x, int M, int d, const void* w, const void* b, int w_bf16, float eps,
                            float* out, cudaStream_t s);
 const char* rms_scale_rows(const float* x, int M, int d, float eps, float* s_out, cudaStream_t st);
+// sandwich norm: x += y / sqrt(mean(y^2) + eps) * g_post; with g_next, also
+// out = x / sqrt(mean(x^2) + eps) * g_next (the next sub-block's pre-norm, act type)
+const char* post_norm_add(float* x, const float* y, int M, int d, const void* g_post, const void* g_next, int w_bf16,
+                          float eps, void* out, int act_bf16, cudaStream_t s);
 const char* scale_rows(const float* x, const float* sc, int M, int d, void* out, int act_bf16, cudaStream_t s);
 const char* concat_rows(const float* const* parts, const int* widths, int n_parts, int M, void* out,
                         int act_bf16, cudaStream_t s);

@@ -228,6 +228,48 @@ __global__ void layernorm_kernel(const float* __restrict__ x, int M, int d, cons
     out[static_cast<size_t>(m) * d + j] = (xr[j] - mean) * rstd * ldw(w, w_bf16, j) + ldw(b, w_bf16, j);
 }
 
+// Sandwich norm of a Gemma-3 layer (one warp per row): x += RMSNorm(y) * g_post;
+// with g_next also out = RMSNorm(x) * g_next, the pre-norm of the next
+// sub-block, from the row just written (read back through L1/L2).
+template <class T>
+__global__ void post_norm_add_kernel(float* __restrict__ x, const float* __restrict__ y, int M, int d,
+                                     const void* __restrict__ g_post, const void* __restrict__ g_next, int w_bf16,
+                                     float eps, void* __restrict__ out) {
+  pdl_enter();
+  const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (m >= M) return;
+  float* xr = x + static_cast<size_t>(m) * d;
+  const float* yr = y + static_cast<size_t>(m) * d;
+  float ss = 0.0f;
+  for (int j = lane * 4; j < d; j += 128) {
+    const float4 v = *reinterpret_cast<const float4*>(yr + j);
+    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+  }
+  const float inv = rsqrtf(warp_sum(ss) / static_cast<float>(d) + eps);
+  float sx = 0.0f;
+  for (int j = lane * 4; j < d; j += 128) {
+    const float4 v = *reinterpret_cast<const float4*>(yr + j);
+    float4 a = *reinterpret_cast<const float4*>(xr + j);
+    a.x = fmaf(v.x * inv, ldw(g_post, w_bf16, j + 0), a.x);
+    a.y = fmaf(v.y * inv, ldw(g_post, w_bf16, j + 1), a.y);
+    a.z = fmaf(v.z * inv, ldw(g_post, w_bf16, j + 2), a.z);
+    a.w = fmaf(v.w * inv, ldw(g_post, w_bf16, j + 3), a.w);
+    *reinterpret_cast<float4*>(xr + j) = a;
+    sx += a.x * a.x + a.y * a.y + a.z * a.z + a.w * a.w;
+  }
+  if (!g_next) return;
+  const float inx = rsqrtf(warp_sum(sx) / static_cast<float>(d) + eps);
+  __syncwarp();
+  for (int j = lane * 4; j < d; j += 128) {
+    const float4 a = *reinterpret_cast<const float4*>(xr + j);
+    const size_t o = static_cast<size_t>(m) * d + j;
+    store_act<T>(out, o + 0, a.x * inx * ldw(g_next, w_bf16, j + 0));
+    store_act<T>(out, o + 1, a.y * inx * ldw(g_next, w_bf16, j + 1));
+    store_act<T>(out, o + 2, a.z * inx * ldw(g_next, w_bf16, j + 2));
+    store_act<T>(out, o + 3, a.w * inx * ldw(g_next, w_bf16, j + 3));
+  }
+}
+
 __global__ void rms_scale_kernel(const float* __restrict__ x, int M, int d, float eps, float* __restrict__ s) {
   pdl_enter();
   const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
@@ -374,6 +416,18 @@ const char* layernorm_rows(const float* x, int M, int d, const void* w, const vo
 const char* rms_scale_rows(const float* x, int M, int d, float eps, float* s_out, cudaStream_t st) {
   if (M <= 0) return nullptr;
   launch_pdl(rms_scale_kernel, rows_grid(M), WPB * 32, 0, st, x, M, d, eps, s_out);
+  return err();
+}
+
+const char* post_norm_add(float* x, const float* y, int M, int d, const void* g_post, const void* g_next, int w_bf16,
+                          float eps, void* out, int act_bf16, cudaStream_t s) {
+  if (M <= 0) return nullptr;
+  if (d % 4) return "post-norm rows need d % 4 == 0";
+  if (act_bf16)
+    launch_pdl(post_norm_add_kernel<bf16>, rows_grid(M), WPB * 32, 0, s, x, y, M, d, g_post, g_next, w_bf16, eps, out);
+  else
+    launch_pdl(post_norm_add_kernel<float>, rows_grid(M), WPB * 32, 0, s, x, y, M, d, g_post, g_next, w_bf16, eps,
+               out);
   return err();
 }
 

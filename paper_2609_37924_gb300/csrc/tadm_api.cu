@@ -22,6 +22,9 @@ namespace {
 
 struct LayerW {
   const void *attn_norm, *wqkv, *wo, *ffn_norm, *wgu, *wdown;
+  const void *q_norm, *k_norm, *post_attn, *post_ffn;   // Gemma-3 details (null when off)
+  int window;      // > 0: local layer with this sliding window
+  int global;      // 1: global layer (RoPE base rope_theta_global when set)
 };
 
 struct Inventory {
@@ -46,6 +49,10 @@ bool valid_config(const tadm_config* c, std::string* why) {
     return fail("fusion_rank must be a positive multiple of fusion_heads");
   if (c->dtype != 0 && c->dtype != 1) return fail("dtype must be 0 (fp32) or 1 (bf16)");
   if (!(c->norm_eps >= 0.0f) || !(c->rope_theta > 0.0f)) return fail("norm_eps >= 0 and rope_theta > 0");
+  if (c->sliding_window < 0 || c->global_every < 0) return fail("sliding_window and global_every must be >= 0");
+  if ((c->qk_norm != 0 && c->qk_norm != 1) || (c->sandwich_norm != 0 && c->sandwich_norm != 1))
+    return fail("qk_norm and sandwich_norm must be 0 or 1");
+  if (!(c->rope_theta_global >= 0.0f)) return fail("rope_theta_global must be >= 0");
   return true;
 }
 
@@ -65,10 +72,16 @@ Inventory inventory(const tadm_config* c) {
       std::string p = std::string(nets[t]) + "." + std::to_string(i) + ".";
       add(p + "attn_norm", d, 1);
       add(p + "wqkv", (c->n_heads + 2LL * c->n_kv_heads) * hd, d);
+      if (c->qk_norm) {
+        add(p + "q_norm", hd, 1);
+        add(p + "k_norm", hd, 1);
+      }
       add(p + "wo", d, c->n_heads * hd);
+      if (c->sandwich_norm) add(p + "post_attn_norm", d, 1);
       add(p + "ffn_norm", d, 1);
       add(p + "wgu", 2 * F, d);
       add(p + "wdown", d, F);
+      if (c->sandwich_norm) add(p + "post_ffn_norm", d, 1);
     }
   if (c->fusion == 0) {
     add("fusion.ln_c.w", d, 1);
@@ -118,7 +131,8 @@ struct tadm_handle {
   char* ws = nullptr;
   size_t ws_bytes = 0, ws_need = 0;
   struct Off {
-    size_t status, rope, c, x, h_int, norm, qbuf, kv, attn, glu, f_g, f_hid, f_pre, part, conf, tok, split, idx;
+    size_t status, rope, rope_g, post, c, x, h_int, norm, qbuf, kv, attn, glu, f_g, f_hid, f_pre, part, conf, tok,
+        split, idx;
     size_t attn_part, act, cnt;
     size_t pa_z, pa_j, pa_mq, pa_mk, pa_mv, pa_mo, pa_r, pa_rb, pa_hid, pa_phi, pa_m, pa_dz, pa_f, pa_g, pa_mb;
   } off{};
@@ -150,6 +164,12 @@ struct tadm_handle {
   int gctx = 0;
 
   int es() const { return cfg.dtype ? 2 : 4; }
+  bool has_rope_g() const {
+    if (!(cfg.rope_theta_global > 0.0f) || cfg.rope_theta_global == cfg.rope_theta) return false;
+    for (const auto& L : layers)
+      if (L.global) return true;
+    return false;
+  }
   int act_bf16() const { return cfg.dtype; }
   template <class T = char>
   T* at(size_t o) const { return reinterpret_cast<T*>(ws + o); }
@@ -235,6 +255,9 @@ void layout(tadm_handle* h) {
   auto& f = h->off;
   f.status = take(256);
   f.rope = take(static_cast<size_t>(n_pos) * (c.head_dim / 2) * 8);
+  // global layers with their own RoPE base get a second table
+  f.rope_g = h->has_rope_g() ? take(static_cast<size_t>(n_pos) * (c.head_dim / 2) * 8) : f.rope;
+  f.post = c.sandwich_norm ? take(M * d * 4) : 0;   // sub-block output ahead of its post-norm
   f.c = take(M * d * 4);
   f.x = take(M * d * 4);
   f.h_int = take(cache_bytes(c, h->max_batch, h->max_rows));
@@ -337,7 +360,11 @@ void* kv_ptr(tadm_handle* h, int li, int which) {
 }
 
 // Pre-norm backbone layer on the fp32 residual x [B*R, d], rows at positions
-// ctx .. ctx+R-1, attending to the layer's KV context 0 .. ctx-1.
+// ctx .. ctx+R-1, attending to the layer's KV context 0 .. ctx-1.  With the
+// Gemma-3 details: QK-norm inside the QKV epilogue (before RoPE), the layer's
+// window and RoPE table, and sandwich norms: the O and down projections then
+// write their output to the post buffer, and one row kernel applies the
+// post-norm and the residual add (after attention also the FFN pre-norm).
 tadm_status layer_fwd(tadm_handle* h, int li, float* x, int B, int R, int ctx, int causal, cudaStream_t s) {
   const tadm_config& c = h->cfg;
   const LayerW& L = h->layers[li];
@@ -359,33 +386,57 @@ tadm_status layer_fwd(tadm_handle* h, int li, float* x, int B, int R, int ctx, i
   ep.n_kv_heads = c.n_kv_heads;
   ep.head_dim = hd;
   ep.rope = 1;
-  ep.rope_tab = h->at<const float2>(h->off.rope);
+  ep.rope_tab = h->at<const float2>(L.global ? h->off.rope_g : h->off.rope);
   ep.rope_npos = h->kv_stride + h->max_rows;
+  ep.q_gain = L.q_norm;
+  ep.k_gain = L.k_norm;
+  ep.qk_eps = c.norm_eps;
   TRYS(gemm(h, norm, Mmax, d, L.wqkv, d, M, nqkv, d, EPI_QKV, ep, s));
   AttnCall a{ep.q, ep.k, ep.v, h->at(h->off.attn), B, c.n_heads, c.n_kv_heads, hd, R, ctx, h->kv_stride, causal,
              h->act_bf16(), h->status()};
+  a.window = L.window;
   if (c.dtype) {
     a.part = h->at(h->off.attn_part);
     a.part_bytes = kAttnPartBytes;
   }
   pi = probe_begin(h, s);
   TRY(attention(a, s));
-  // keys seen per query row: all of them, or the causal average
-  const double keys = causal ? ctx + 0.5 * (R + 1) : static_cast<double>(ctx + R);
+  // keys seen per query row: all of them, or the causal average (window: at most the window)
+  double keys = causal ? ctx + 0.5 * (R + 1) : static_cast<double>(ctx + R);
+  if (L.window > 0) keys = std::min(keys, static_cast<double>(L.window + (causal ? 0 : R)));
   probe_end(h, s, pi, R < 128 ? kProbeAttentionShort : kProbeAttention, 4.0 * M * c.n_heads * keys * hd);
   EpiParams er{};
   er.resid = x;
   er.ldr = d;
-  TRYS(gemm(h, h->at(h->off.attn), Mmax, q, L.wo, q, M, d, q, EPI_RESID, er, s));
-  pi = probe_begin(h, s);
-  TRY(rmsnorm_rows(x, M, d, L.ffn_norm, c.dtype, c.norm_eps, norm, d, h->act_bf16(), s));
-  probe_end(h, s, pi, kProbeNorm, 0.0);
+  EpiParams ey{};                       // sandwich: the sub-block output, fp32, ahead of its post-norm
+  ey.out = h->at(h->off.post);
+  ey.ldo = d;
+  float* post = h->at<float>(h->off.post);
+  if (c.sandwich_norm) {
+    TRYS(gemm(h, h->at(h->off.attn), Mmax, q, L.wo, q, M, d, q, EPI_STORE, ey, s, true));
+    // x += RMSNorm(o W_o^T) * post_attn; norm = RMSNorm(x) * ffn_norm
+    pi = probe_begin(h, s);
+    TRY(post_norm_add(x, post, M, d, L.post_attn, L.ffn_norm, c.dtype, c.norm_eps, norm, h->act_bf16(), s));
+    probe_end(h, s, pi, kProbeNorm, 0.0);
+  } else {
+    TRYS(gemm(h, h->at(h->off.attn), Mmax, q, L.wo, q, M, d, q, EPI_RESID, er, s));
+    pi = probe_begin(h, s);
+    TRY(rmsnorm_rows(x, M, d, L.ffn_norm, c.dtype, c.norm_eps, norm, d, h->act_bf16(), s));
+    probe_end(h, s, pi, kProbeNorm, 0.0);
+  }
   EpiParams eg{};
   eg.out = h->at(h->off.glu);
   eg.ldo = c.ffn;
   eg.glu = c.glu;
   TRYS(gemm(h, norm, Mmax, d, L.wgu, d, M, c.ffn, d, EPI_GLU, eg, s));
-  TRYS(gemm(h, h->at(h->off.glu), Mmax, c.ffn, L.wdown, c.ffn, M, d, c.ffn, EPI_RESID, er, s));
+  if (c.sandwich_norm) {
+    TRYS(gemm(h, h->at(h->off.glu), Mmax, c.ffn, L.wdown, c.ffn, M, d, c.ffn, EPI_STORE, ey, s, true));
+    pi = probe_begin(h, s);
+    TRY(post_norm_add(x, post, M, d, L.post_ffn, nullptr, c.dtype, c.norm_eps, nullptr, h->act_bf16(), s));
+    probe_end(h, s, pi, kProbeNorm, 0.0);
+  } else {
+    TRYS(gemm(h, h->at(h->off.glu), Mmax, c.ffn, L.wdown, c.ffn, M, d, c.ffn, EPI_RESID, er, s));
+  }
   return TADM_OK;
 }
 
@@ -783,13 +834,22 @@ tadm_status tadm_create(const tadm_config* cfg, const void* const* weights, int 
   int i = 0;
   h->embed = weights[i++];
   for (int l = 0; l < h->L_total; ++l) {
-    LayerW L;
+    LayerW L{};
     L.attn_norm = weights[i++];
     L.wqkv = weights[i++];
+    if (c.qk_norm) {
+      L.q_norm = weights[i++];
+      L.k_norm = weights[i++];
+    }
     L.wo = weights[i++];
+    if (c.sandwich_norm) L.post_attn = weights[i++];
     L.ffn_norm = weights[i++];
     L.wgu = weights[i++];
     L.wdown = weights[i++];
+    if (c.sandwich_norm) L.post_ffn = weights[i++];
+    // layer l of the whole backbone is global iff global_every == 0 or (l + 1) % global_every == 0
+    L.global = c.global_every == 0 || (l + 1) % c.global_every == 0;
+    L.window = L.global ? 0 : c.sliding_window;
     h->layers.push_back(L);
   }
   // fusion tensors (10 for fusion 0 and 1, none for fusion 2), in inventory order
@@ -908,6 +968,8 @@ tadm_status tadm_bind_workspace(tadm_handle* h, void* dev_ptr, size_t bytes) {
   const int n_pos = h->kv_stride + h->max_rows;
   cudaStream_t s = nullptr;
   TRY(rope_table(h->at<float2>(h->off.rope), n_pos, h->cfg.head_dim, h->cfg.rope_theta, s));
+  if (h->off.rope_g != h->off.rope)
+    TRY(rope_table(h->at<float2>(h->off.rope_g), n_pos, h->cfg.head_dim, h->cfg.rope_theta_global, s));
   if (cudaMemsetAsync(h->status(), 0, 256, s) != cudaSuccess) return fail(h, TADM_ERR_CUDA, "memset failed");
   // K / V positions that were never written are read with zero weight; keep them finite
   if (cudaMemsetAsync(h->at(h->off.kv), 0, h->off.attn - h->off.kv, s) != cudaSuccess)
@@ -1187,10 +1249,12 @@ tadm_status tadm_head_confidence(const void* x, const void* w, int rows, int d, 
 }
 
 tadm_status tadm_attention(const void* q, const void* k, const void* v, void* o, int batch, int n_heads, int n_kv_heads,
-                           int head_dim, int rows, int ctx, int kv_stride, int causal, int dtype, tadm_stream stream) {
-  if (!q || !k || !v || !o || batch < 0 || n_heads <= 0 || n_kv_heads <= 0 || rows < 0 || ctx < 0)
+                           int head_dim, int rows, int ctx, int kv_stride, int causal, int window, int dtype,
+                           tadm_stream stream) {
+  if (!q || !k || !v || !o || batch < 0 || n_heads <= 0 || n_kv_heads <= 0 || rows < 0 || ctx < 0 || window < 0)
     return TADM_ERR_INVALID_ARG;
   AttnCall a{q, k, v, o, batch, n_heads, n_kv_heads, head_dim, rows, ctx, kv_stride, causal, dtype, nullptr};
+  a.window = window;
   return attention(a, stream) ? TADM_ERR_CUDA : TADM_OK;
 }
 

@@ -39,7 +39,9 @@ class tadm_config(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "vocab", "d_model", "n_heads", "n_kv_heads", "head_dim", "ffn", "glu", "n_shared", "n_anchor",
         "n_denoise", "fusion", "fusion_rank", "fusion_heads", "dtype", "tied_lm_head")] + [
-        ("norm_eps", ctypes.c_float), ("rope_theta", ctypes.c_float)]
+        ("norm_eps", ctypes.c_float), ("rope_theta", ctypes.c_float)] + [
+        (n, ctypes.c_int32) for n in ("sliding_window", "global_every", "qk_norm", "sandwich_norm")] + [
+        ("rope_theta_global", ctypes.c_float)]
 
 
 class tadm_step_outputs(ctypes.Structure):
@@ -93,7 +95,7 @@ def load_library(path: str = LIB_PATH) -> ctypes.CDLL:
         "tadm_gemm": (I, [P, P, P, I, I, I, I, I, I, I, I, P]),
         "tadm_confidence": (I, [P, I, I, I, P, P, P]),
         "tadm_topk_unmask": (I, [P, I, P, P, I, I, I, I, P, P]),
-        "tadm_attention": (I, [P, P, P, P, I, I, I, I, I, I, I, I, I, P]),
+        "tadm_attention": (I, [P, P, P, P, I, I, I, I, I, I, I, I, I, I, P]),
         "tadm_head_scratch_size": (I, [I, I, I, ctypes.POINTER(SZ)]),
         "tadm_head_confidence": (I, [P, P, I, I, I, I, I, P, SZ, P, P, P]),
         "tadm_head_confidence_static": (I, [P, P, I, I, I, I, I, P, P, P]),
@@ -136,7 +138,11 @@ def make_config(model) -> tadm_config:
         head_dim=model.head_dim, ffn=model.ffn, glu=1 if model.glu == "geglu" else 0, n_shared=model.n_shared,
         n_anchor=model.n_anchor, n_denoise=model.n_denoise, fusion={"gated_mlp": 0, "paired_attn": 1, "none": 2}[model.fusion],
         fusion_rank=model.fusion_rank, fusion_heads=model.fusion_heads, dtype=1 if model.dtype == "bf16" else 0,
-        tied_lm_head=int(bool(model.tied_lm_head)), norm_eps=model.norm_eps, rope_theta=model.rope_theta)
+        tied_lm_head=int(bool(model.tied_lm_head)), norm_eps=model.norm_eps, rope_theta=model.rope_theta,
+        sliding_window=getattr(model, "sliding_window", 0), global_every=getattr(model, "global_every", 0),
+        qk_norm=int(bool(getattr(model, "qk_norm", False))),
+        sandwich_norm=int(bool(getattr(model, "sandwich_norm", False))),
+        rope_theta_global=getattr(model, "rope_theta_global", 0.0))
 
 
 # ---------------------------------------------------------------------------- C-named wrappers
@@ -222,11 +228,11 @@ def tadm_head_confidence_static(x, w, mask_id: int, conf, tok, dtype: int, strea
 
 
 def tadm_attention(q, k, v, o, n_heads: int, n_kv_heads: int, rows: int, ctx: int, causal: bool, dtype: int,
-                   stream=None):
+                   stream=None, window: int = 0):
     batch, _, _, hd = q.shape
     kv_stride = k.shape[2]
     _check(load_library().tadm_attention(_ptr(q), _ptr(k), _ptr(v), _ptr(o), batch, n_heads, n_kv_heads, hd, rows,
-                                         ctx, kv_stride, int(causal), dtype, _stream(stream)))
+                                         ctx, kv_stride, int(causal), window, dtype, _stream(stream)))
 
 
 REMDM_KINDS = {"cap": 0, "loop": 1}

@@ -105,6 +105,13 @@ def test_invalid_configs_are_rejected(lib):
     cfg = lib.make_config(base)
     cfg.fusion = 3                                  # 0, 1, 2 are the only fusion modes
     assert so.tadm_weight_count(ctypes.byref(cfg)) == -1
+    # Gemma-3 layer options: windows and patterns are non-negative, the norms are switches
+    for field, bad in (("sliding_window", -1), ("global_every", -2), ("qk_norm", 2), ("sandwich_norm", -1),
+                       ("rope_theta_global", -1.0)):
+        cfg = lib.make_config(wl.POSTTRAIN_G3)
+        assert so.tadm_weight_count(ctypes.byref(cfg)) > 0
+        setattr(cfg, field, bad)
+        assert so.tadm_weight_count(ctypes.byref(cfg)) == -1, field
     h = ctypes.c_void_p()
     cfg = lib.make_config(base)
     assert so.tadm_create(ctypes.byref(cfg), None, 0, 1, 1, 0, ctypes.byref(h)) == 1   # no weights
