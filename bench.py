@@ -56,6 +56,8 @@ def parse():
     ap.add_argument("--sweep-batches", default="", help="batches for the 'sweep' workload (default 1,8,32,128)")
     ap.add_argument("--kernel-bench", default=None,
                     help="time one building block alone instead, e.g. gemm:16384,32768,768")
+    ap.add_argument("--qkv-split", type=int, default=None, choices=[0, 1],
+                    help="override the model's qkv_split (QKV projection input as bf16 hi + lo)")
     ap.add_argument("--configs", default="block,posttrain",
                     help="at N = 1: workloads also timed whole (K = 1 and the workload's K) and reported under "
                          "'configs' in the same JSON line ('' for none)")
@@ -290,6 +292,8 @@ def gpu_arm(args):
         over["steps_per_block"] = args.T
     if args.G:
         over["gen_len"] = args.G
+    if args.qkv_split is not None:
+        over["model_qkv_split"] = bool(args.qkv_split)
     w = wl.get_workload(args.workload, **over)
     K = args.K or w.K
     m = w.model
@@ -397,6 +401,7 @@ def gpu_arm(args):
             "config": {"workload": w.name, "batch": B, "prompt_len": w.prompt_len, "gen_len": w.gen_len,
                        "steps_per_block": w.steps_per_block, "block_len": bl, "K": K, "d_model": m.d_model,
                        "layers_anchor": m.n_anchor, "layers_denoise": m.n_denoise, "vocab": m.vocab,
+                       "qkv_split": bool(m.qkv_split),
                        "parallelism": f"replicas x{world}",
                        "l2": "inputs larger than L2 (weights + activations per step >> 129 MB)"},
             "k_sweep_tokens_per_s": sweep, "roofline": roofline, "clocks": clk,

@@ -92,6 +92,14 @@ typedef enum {
  *           post_attn_norm, post_ffn_norm) before the residual add.
  *  rope_theta_global: RoPE base of global layers (0 = rope_theta); local
  *           layers use rope_theta.
+ *  qkv_split: bf16 models only: 1 = the normalised input of every QKV
+ *           projection enters the tensor cores as two bf16 terms, hi =
+ *           bf16(n) and lo = bf16(n - hi), both multiplying the same weight
+ *           tiles (the projection then costs twice the MMA work); its input
+ *           is carried to about 16 significant bits instead of 8.  The
+ *           attention logits are the most rounding-sensitive quantity of the
+ *           backbone, and this keeps the committed tokens of a
+ *           teacher-forced generation on those of the exact model.
  */
 typedef struct {
   int32_t vocab, d_model, n_heads, n_kv_heads, head_dim, ffn;
@@ -104,6 +112,7 @@ typedef struct {
   float norm_eps, rope_theta;
   int32_t sliding_window, global_every, qk_norm, sandwich_norm;
   float rope_theta_global;
+  int32_t qkv_split;
 } tadm_config;
 
 typedef struct tadm_handle tadm_handle;

@@ -70,7 +70,9 @@ struct AttnTcArgs {
   int* status;
 };
 
-template <int HD, int TKV>
+// WIN: the sliding window of local layers is in force (a separate
+// instantiation, so that the kernel without it carries no window code).
+template <int HD, int TKV, bool WIN>
 __global__ void __launch_bounds__(192, AttnTcCfg<HD, TKV>::MIN_BLOCKS)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
                    const AttnTcArgs args) {
@@ -111,7 +113,7 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD, TKV>::MIN_BLOCKS)
   const int kv_end = args.causal ? min(args.kv_len, args.ctx + r_max + 1) : args.kv_len;
   // sliding window: no row of this CTA sees a key below the smallest row's window start
   const int r_min = (m0 / args.rows != v_last / args.rows) ? 0 : m0 % args.rows;
-  const int kv_begin = args.window > 0 ? max(0, args.ctx + r_min - args.window + 1) : 0;
+  const int kv_begin = WIN ? max(0, args.ctx + r_min - args.window + 1) : 0;
   const int t0 = max(split * args.tiles_per_split, kv_begin / TKV);   // first tile of this CTA
   const int n_tiles = max(0, min((kv_end + TKV - 1) / TKV, (split + 1) * args.tiles_per_split) - t0);
 
@@ -243,10 +245,9 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD, TKV>::MIN_BLOCKS)
       const int key0 = (t0 + i) * TKV;
       // keys visible to this row: kv_lo <= key < kv_hi (kv_end, or the causal bound; the window start)
       const int kv_hi = args.causal ? min(kv_end, qpos + 1) : kv_end;
-      const int kv_lo = args.window > 0 ? qpos - args.window + 1 : 0;
       const int lim = kv_hi - key0;                                   // visible keys of this tile: [lo, lim)
-      const int lo = kv_lo - key0;
-      const bool masked = __any_sync(0xffffffffu, lim < TKV || lo > 0);   // warp-uniform path choice
+      const int lo = WIN ? qpos - args.window + 1 - key0 : 0;
+      const bool masked = __any_sync(0xffffffffu, lim < TKV || (WIN && lo > 0));   // warp-uniform path choice
       // pass 1: row max over the tile, 64 columns per TMEM round trip
       float mxa[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};   // independent chains
 #pragma unroll
@@ -459,8 +460,8 @@ bool map3d(CUtensorMap* m, const void* ptr, uint64_t d0, uint64_t d1, uint64_t d
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int HD, int TKV>
-const char* launch_tc(const AttnCall& a, cudaStream_t s) {
+template <int HD, int TKV, bool WIN>
+const char* launch_tc_win(const AttnCall& a, cudaStream_t s) {
   using C = AttnTcCfg<HD, TKV>;
   if (!encoder()) return "cuTensorMapEncodeTiled is unavailable";
   const int kv_len = a.ctx + a.rows;
@@ -473,7 +474,7 @@ const char* launch_tc(const AttnCall& a, cudaStream_t s) {
     return "attention tensor map encode failed";
   static int n_sms = 0;
   if (n_sms == 0) {
-    if (cudaFuncSetAttribute(attn_tc_kernel<HD, TKV>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM) !=
+    if (cudaFuncSetAttribute(attn_tc_kernel<HD, TKV, WIN>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM) !=
         cudaSuccess)
       return "attention smem attribute failed";
     int dev = 0;
@@ -490,9 +491,8 @@ const char* launch_tc(const AttnCall& a, cudaStream_t s) {
   // idle SMs): every split keeps >= 3 tiles and its fp32 partials fit the
   // caller's scratch
   int splits = 1;
-  // a window that hides keys leaves each CTA only its window's tiles: no key splits then
-  const bool window_cuts = a.window > 0 && a.window < kv_len;
-  if (a.part && a.part_bytes > 0 && !window_cuts) {
+  // a window leaves each CTA only its window's tiles: no key splits then
+  if (a.part && a.part_bytes > 0 && !WIN) {
     const int slots = C::MIN_BLOCKS * n_sms;
     const size_t per_split = static_cast<size_t>(a.batch) * a.n_kv_heads * n_virt * (HD + 2) * sizeof(float);
     splits = std::min(std::min(slots / base, kv_tiles / 3), 8);
@@ -507,7 +507,7 @@ const char* launch_tc(const AttnCall& a, cudaStream_t s) {
                   1.4426950408889634f / sqrtf(static_cast<float>(HD)), static_cast<bf16*>(a.o),
                   n_vtiles, splits, tps, part_o, part_ml, a.status};
   dim3 grid(n_vtiles * splits, a.n_kv_heads, a.batch);
-  launch_pdl(attn_tc_kernel<HD, TKV>, grid, 192, C::SMEM, s, mk, mv, args);
+  launch_pdl(attn_tc_kernel<HD, TKV, WIN>, grid, 192, C::SMEM, s, mk, mv, args);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cudaGetErrorString(e);
   if (splits > 1) {
@@ -519,6 +519,13 @@ const char* launch_tc(const AttnCall& a, cudaStream_t s) {
     if (e != cudaSuccess) return cudaGetErrorString(e);
   }
   return nullptr;
+}
+
+// the windowed kernel only where the window hides keys (window < ctx + rows)
+template <int HD, int TKV>
+const char* launch_tc(const AttnCall& a, cudaStream_t s) {
+  return a.window > 0 && a.window < a.ctx + a.rows ? launch_tc_win<HD, TKV, true>(a, s)
+                                                   : launch_tc_win<HD, TKV, false>(a, s);
 }
 
 // ============================================================= mma.sync path

@@ -115,6 +115,7 @@ struct TcArgs {
   int staged;              // bf16 outputs go through the per-warp boxes and TMA stores
   int b_split;             // >0: B tile = 128 rows at n*128 and 128 rows at b_split + n*128
   int n_tiles_n;
+  int kb_wrap;             // > 0: B's k-block of A's k-block kb is kb % kb_wrap (split hi + lo operand)
   int* status;
   const int* m_dev;        // optional device row count (<= M): tiles past it are skipped
   EpiParams ep;
@@ -206,12 +207,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
           if (!mbar_wait_bounded(&empty[stage], phase ^ 1, abort_flag, args.status)) { ok = false; break; }
           mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
           tma_load_2d(sA + stage * A_BYTES, &tmA, &full[stage], kb * BK, mb * BM);
+          const int kbb = args.kb_wrap > 0 ? kb % args.kb_wrap : kb;
           if (args.b_split > 0) {
-            tma_load_2d(sB + stage * B_BYTES, &tmB, &full[stage], kb * BK, nb * (BN / 2));
-            tma_load_2d(sB + stage * B_BYTES + B_BYTES / 2, &tmB, &full[stage], kb * BK,
+            tma_load_2d(sB + stage * B_BYTES, &tmB, &full[stage], kbb * BK, nb * (BN / 2));
+            tma_load_2d(sB + stage * B_BYTES + B_BYTES / 2, &tmB, &full[stage], kbb * BK,
                         args.b_split + nb * (BN / 2));
           } else {
-            tma_load_2d(sB + stage * B_BYTES, &tmB, &full[stage], kb * BK, nb * BN);
+            tma_load_2d(sB + stage * B_BYTES, &tmB, &full[stage], kbb * BK, nb * BN);
           }
           ++issued[stage];
           if (++stage == STAGES) { stage = 0; phase ^= 1; }
@@ -401,7 +403,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
           if (leader) mbar_arrive_expect_tx(&full[stage], 2 * P_STAGE_BYTES);
           const uint32_t fb = full_l0 + 8u * stage;
           tma_load_2d_pair(sA + stage * P_A_BYTES, &tmA, fb, kb * BK, mb * BM);
-          tma_load_2d_pair(sB + stage * P_B_BYTES, &tmB, fb, kb * BK, brow);
+          tma_load_2d_pair(sB + stage * P_B_BYTES, &tmB, fb, (args.kb_wrap > 0 ? kb % args.kb_wrap : kb) * BK, brow);
           if (++stage == P_STAGES) { stage = 0; phase ^= 1; }
         }
         if (!ok) break;
@@ -593,19 +595,22 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
   if (!get_encoder()) return "cuTensorMapEncodeTiled is unavailable";
   if (g.M <= 0 || g.N <= 0 || g.K <= 0) return nullptr;
   if (g.K % 8 || g.lda % 8 || g.ldb % 8) return "bf16 GEMM needs K, lda, ldb multiples of 8";
+  if (g.k_b > 0 && (g.K != 2 * g.k_b || g.k_b % BK)) return "split operand GEMM needs K = 2 k_b, k_b % 64 == 0";
+  const int k_b = g.k_b > 0 ? g.k_b : g.K;   // columns of B
   if ((reinterpret_cast<uintptr_t>(g.A) | reinterpret_cast<uintptr_t>(g.B)) & 15)
     return "bf16 GEMM operands must be 16-byte aligned";
   const bool glu = g.epi == EPI_GLU;
   CUtensorMap ta, tb;
   if (!make_map(&ta, g.A, g.A_rows > 0 ? g.A_rows : g.M, g.K, g.lda, BM)) return "tensor map (A) encode failed";
   const int64_t b_rows = glu ? 2LL * g.N : g.N;
-  if (!make_map(&tb, g.B, b_rows, g.K, g.ldb, glu ? BN / 2 : BN)) return "tensor map (B) encode failed";
+  if (!make_map(&tb, g.B, b_rows, k_b, g.ldb, glu ? BN / 2 : BN)) return "tensor map (B) encode failed";
   TcArgs a;
   a.M = g.M;
   a.K = g.K;
   a.N_acc = glu ? 2 * g.N : g.N;
   a.b_split = glu ? g.N : 0;
   a.n_tiles_n = glu ? (g.N + BN / 2 - 1) / (BN / 2) : (g.N + BN - 1) / BN;
+  a.kb_wrap = g.k_b > 0 ? g.k_b / BK : 0;
   if (glu && g.N % (BN / 2)) return "GLU GEMM needs the FFN width to be a multiple of 128";
   if (g.epi == EPI_QKV && BN % g.ep.head_dim) return "head_dim must divide 256";
   if (g.epi == EPI_PA_GATE && g.N > BN) return "gate GEMM needs N <= 256";
@@ -666,7 +671,7 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
   // than 128 rows: the same SMs as 128 x 256 tiles, less operand traffic each
   if (pair_ok && a.splits == 1 && narrow) {
     CUtensorMap tbh;
-    if (!make_map(&tbh, g.B, b_rows, g.K, g.ldb, 64)) return "tensor map (B, quarter tiles) encode failed";
+    if (!make_map(&tbh, g.B, b_rows, k_b, g.ldb, 64)) return "tensor map (B, quarter tiles) encode failed";
     TcArgs a2 = a;
     a2.n_tiles_n = (g.N + 127) / 128;
     cudaError_t e = g.epi == EPI_RESID ? launch_epi_pair<EPI_RESID, 128>(ta, tbh, tc, tc2, a2, pair_units, s)
@@ -677,7 +682,7 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
   }
   if (pair_ok && a.splits == 1) {
     CUtensorMap tbh;
-    if (!make_map(&tbh, g.B, b_rows, g.K, g.ldb, BN / 2)) return "tensor map (B, half tiles) encode failed";
+    if (!make_map(&tbh, g.B, b_rows, k_b, g.ldb, BN / 2)) return "tensor map (B, half tiles) encode failed";
     cudaError_t e;
     switch (g.epi) {
       case EPI_STORE: e = launch_epi_pair<EPI_STORE>(ta, tbh, tc, tc2, a, pair_units, s); break;

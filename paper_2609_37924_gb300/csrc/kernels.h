@@ -36,6 +36,7 @@ struct GemmCall {
   EpiParams ep;
   int* status;
   const int* m_dev = nullptr;   // optional device row count <= M (tcgen05 path): tiles past it are skipped
+  int k_b = 0;           // > 0: B has k_b columns and A's K = 2 k_b columns [hi | lo] both multiply B (split operand)
   float* split_buf;      // fp32 partials for split-K (null: no split)
   size_t split_bytes;
   int launched;          // out: kernels launched
@@ -74,8 +75,9 @@ const char* attention(const AttnCall& a, cudaStream_t s);
 const char* embed_rows(const int32_t* z, int ldz, int batch, int rows, const void* E, int e_bf16, int d,
                        int vocab, float* out, float* out2, cudaStream_t s, const float* add = nullptr,
                        int add_first = 0, const float* add_div = nullptr);
+// lo_off > 0 (bf16 activations): also the remainder bf16(y - bf16(y)) at column lo_off of each output row
 const char* rmsnorm_rows(const float* x, int M, int d, const void* gain, int w_bf16, float eps, void* out,
-                         int ldo, int act_bf16, cudaStream_t s, const int32_t* rows_idx = nullptr);
+                         int ldo, int act_bf16, cudaStream_t s, const int32_t* rows_idx = nullptr, int lo_off = 0);
 // per sequence: the rows still holding MASK (first `per_seq` of them, in order) -> idx[b * per_seq + j]
 // (global row b * rows + r); conf of every row set to -inf so that rows left out are never selected
 const char* masked_rows(const int32_t* z, int ldz, int batch, int rows, int mask_id, int per_seq, int32_t* idx,

@@ -31,6 +31,20 @@ __device__ __forceinline__ void store_act<bf16>(void* out, size_t i, float v) {
   static_cast<bf16*>(out)[i] = __float2bfloat16_rn(v);
 }
 
+// act value v at out[i]; with lo_off > 0 (bf16 only) also the rounding
+// remainder bf16(v - hi) at out[i + lo_off]: the split (hi + lo) operand of a
+// projection whose input is carried at about 16 bits
+template <class T>
+__device__ __forceinline__ void store_act2(void* out, size_t i, float v, int lo_off);
+template <>
+__device__ __forceinline__ void store_act2<float>(void* out, size_t i, float v, int) { static_cast<float*>(out)[i] = v; }
+template <>
+__device__ __forceinline__ void store_act2<bf16>(void* out, size_t i, float v, int lo_off) {
+  const bf16 hi = __float2bfloat16_rn(v);
+  static_cast<bf16*>(out)[i] = hi;
+  if (lo_off > 0) static_cast<bf16*>(out)[i + lo_off] = __float2bfloat16_rn(v - __bfloat162float(hi));
+}
+
 __device__ __forceinline__ float ldw(const void* w, int bf, int i) {
   return bf ? __bfloat162float(static_cast<const bf16*>(w)[i]) : static_cast<const float*>(w)[i];
 }
@@ -83,7 +97,7 @@ template <class T>
 __global__ void __launch_bounds__(256) rmsnorm_block_kernel(const float* __restrict__ x, int d,
                                                             const void* __restrict__ gain, int w_bf16, float eps,
                                                             void* __restrict__ out, int ldo,
-                                                            const int32_t* __restrict__ rows_idx) {
+                                                            const int32_t* __restrict__ rows_idx, int lo_off) {
   pdl_enter();
   __shared__ float red[8];
   const int m = blockIdx.x;
@@ -103,17 +117,18 @@ __global__ void __launch_bounds__(256) rmsnorm_block_kernel(const float* __restr
   for (int j = threadIdx.x * 4; j < d; j += 1024) {
     const float4 v = *reinterpret_cast<const float4*>(xr + j);
     const size_t o = static_cast<size_t>(m) * ldo + j;
-    store_act<T>(out, o + 0, v.x * inv * ldw(gain, w_bf16, j + 0));
-    store_act<T>(out, o + 1, v.y * inv * ldw(gain, w_bf16, j + 1));
-    store_act<T>(out, o + 2, v.z * inv * ldw(gain, w_bf16, j + 2));
-    store_act<T>(out, o + 3, v.w * inv * ldw(gain, w_bf16, j + 3));
+    store_act2<T>(out, o + 0, v.x * inv * ldw(gain, w_bf16, j + 0), lo_off);
+    store_act2<T>(out, o + 1, v.y * inv * ldw(gain, w_bf16, j + 1), lo_off);
+    store_act2<T>(out, o + 2, v.z * inv * ldw(gain, w_bf16, j + 2), lo_off);
+    store_act2<T>(out, o + 3, v.w * inv * ldw(gain, w_bf16, j + 3), lo_off);
   }
 }
 
 // out = x / sqrt(mean(x^2) + eps) * gain
 template <class T>
 __global__ void rmsnorm_kernel(const float* __restrict__ x, int M, int d, const void* __restrict__ gain, int w_bf16,
-                               float eps, void* __restrict__ out, int ldo, const int32_t* __restrict__ rows_idx) {
+                               float eps, void* __restrict__ out, int ldo, const int32_t* __restrict__ rows_idx,
+                               int lo_off) {
   pdl_enter();
   const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
   if (m >= M) return;
@@ -128,10 +143,10 @@ __global__ void rmsnorm_kernel(const float* __restrict__ x, int M, int d, const 
   for (int j = lane * 4; j < d; j += 128) {
     const float4 v = *reinterpret_cast<const float4*>(xr + j);
     const size_t o = static_cast<size_t>(m) * ldo + j;
-    store_act<T>(out, o + 0, v.x * inv * ldw(gain, w_bf16, j + 0));
-    store_act<T>(out, o + 1, v.y * inv * ldw(gain, w_bf16, j + 1));
-    store_act<T>(out, o + 2, v.z * inv * ldw(gain, w_bf16, j + 2));
-    store_act<T>(out, o + 3, v.w * inv * ldw(gain, w_bf16, j + 3));
+    store_act2<T>(out, o + 0, v.x * inv * ldw(gain, w_bf16, j + 0), lo_off);
+    store_act2<T>(out, o + 1, v.y * inv * ldw(gain, w_bf16, j + 1), lo_off);
+    store_act2<T>(out, o + 2, v.z * inv * ldw(gain, w_bf16, j + 2), lo_off);
+    store_act2<T>(out, o + 3, v.w * inv * ldw(gain, w_bf16, j + 3), lo_off);
   }
 }
 
@@ -143,7 +158,7 @@ template <int NCH>
 __global__ void __launch_bounds__(WPB * 32) rmsnorm_reg_kernel(const float* __restrict__ x, int M,
                                                                const bf16* __restrict__ gain, float eps,
                                                                bf16* __restrict__ out, int ldo,
-                                                               const int32_t* __restrict__ rows_idx) {
+                                                               const int32_t* __restrict__ rows_idx, int lo_off) {
   pdl_enter();
   constexpr int d = 256 * NCH;
   const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
@@ -169,14 +184,20 @@ __global__ void __launch_bounds__(WPB * 32) rmsnorm_reg_kernel(const float* __re
     const int j = (c * 32 + lane) * 8;
     const uint4 graw = *reinterpret_cast<const uint4*>(gain + j);
     const __nv_bfloat162* g2 = reinterpret_cast<const __nv_bfloat162*>(&graw);
-    uint32_t packed[4];
+    uint32_t packed[4], packed_lo[4];
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       const float2 g = __bfloat1622float2(g2[q]);
-      __nv_bfloat162 t = __floats2bfloat162_rn(v[c][2 * q] * inv * g.x, v[c][2 * q + 1] * inv * g.y);
+      const float y0 = v[c][2 * q] * inv * g.x, y1 = v[c][2 * q + 1] * inv * g.y;
+      __nv_bfloat162 t = __floats2bfloat162_rn(y0, y1);
       packed[q] = *reinterpret_cast<uint32_t*>(&t);
+      const float2 th = __bfloat1622float2(t);
+      __nv_bfloat162 tl = __floats2bfloat162_rn(y0 - th.x, y1 - th.y);   // remainder of the split operand
+      packed_lo[q] = *reinterpret_cast<uint32_t*>(&tl);
     }
     *reinterpret_cast<uint4*>(orow + j) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+    if (lo_off > 0)
+      *reinterpret_cast<uint4*>(orow + lo_off + j) = make_uint4(packed_lo[0], packed_lo[1], packed_lo[2], packed_lo[3]);
   }
 }
 
@@ -366,33 +387,35 @@ const char* embed_rows(const int32_t* z, int ldz, int batch, int rows, const voi
 }
 
 const char* rmsnorm_rows(const float* x, int M, int d, const void* gain, int w_bf16, float eps, void* out, int ldo,
-                         int act_bf16, cudaStream_t s, const int32_t* rows_idx) {
+                         int act_bf16, cudaStream_t s, const int32_t* rows_idx, int lo_off) {
   if (M <= 0) return nullptr;
+  if (!act_bf16) lo_off = 0;       // fp32 activations are not split
+  if (lo_off > 0 && (lo_off < d || lo_off + d > ldo)) return "split operand: the remainder columns must follow the row";
   if (M < 1024) {   // few rows: a block per row keeps enough SMs busy
     if (act_bf16)
-      launch_pdl(rmsnorm_block_kernel<bf16>, M, 256, 0, s, x, d, gain, w_bf16, eps, out, ldo, rows_idx);
+      launch_pdl(rmsnorm_block_kernel<bf16>, M, 256, 0, s, x, d, gain, w_bf16, eps, out, ldo, rows_idx, lo_off);
     else
-      launch_pdl(rmsnorm_block_kernel<float>, M, 256, 0, s, x, d, gain, w_bf16, eps, out, ldo, rows_idx);
+      launch_pdl(rmsnorm_block_kernel<float>, M, 256, 0, s, x, d, gain, w_bf16, eps, out, ldo, rows_idx, lo_off);
     return err();
   }
-  const bool vec = act_bf16 && w_bf16 && ldo % 8 == 0 &&
+  const bool vec = act_bf16 && w_bf16 && ldo % 8 == 0 && lo_off % 8 == 0 &&
                    ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(out) | reinterpret_cast<uintptr_t>(gain)) & 15) == 0;
   if (vec) {
     const bf16* g = static_cast<const bf16*>(gain);
     bf16* o = static_cast<bf16*>(out);
     switch (d) {
-      case 256: launch_pdl(rmsnorm_reg_kernel<1>, rows_grid(M), WPB * 32, 0, s, x, M, g, eps, o, ldo, rows_idx); return err();
-      case 512: launch_pdl(rmsnorm_reg_kernel<2>, rows_grid(M), WPB * 32, 0, s, x, M, g, eps, o, ldo, rows_idx); return err();
-      case 768: launch_pdl(rmsnorm_reg_kernel<3>, rows_grid(M), WPB * 32, 0, s, x, M, g, eps, o, ldo, rows_idx); return err();
-      case 1024: launch_pdl(rmsnorm_reg_kernel<4>, rows_grid(M), WPB * 32, 0, s, x, M, g, eps, o, ldo, rows_idx); return err();
-      case 2048: launch_pdl(rmsnorm_reg_kernel<8>, rows_grid(M), WPB * 32, 0, s, x, M, g, eps, o, ldo, rows_idx); return err();
+      case 256: launch_pdl(rmsnorm_reg_kernel<1>, rows_grid(M), WPB * 32, 0, s, x, M, g, eps, o, ldo, rows_idx, lo_off); return err();
+      case 512: launch_pdl(rmsnorm_reg_kernel<2>, rows_grid(M), WPB * 32, 0, s, x, M, g, eps, o, ldo, rows_idx, lo_off); return err();
+      case 768: launch_pdl(rmsnorm_reg_kernel<3>, rows_grid(M), WPB * 32, 0, s, x, M, g, eps, o, ldo, rows_idx, lo_off); return err();
+      case 1024: launch_pdl(rmsnorm_reg_kernel<4>, rows_grid(M), WPB * 32, 0, s, x, M, g, eps, o, ldo, rows_idx, lo_off); return err();
+      case 2048: launch_pdl(rmsnorm_reg_kernel<8>, rows_grid(M), WPB * 32, 0, s, x, M, g, eps, o, ldo, rows_idx, lo_off); return err();
       default: break;
     }
   }
   if (act_bf16)
-    launch_pdl(rmsnorm_kernel<bf16>, rows_grid(M), WPB * 32, 0, s, x, M, d, gain, w_bf16, eps, out, ldo, rows_idx);
+    launch_pdl(rmsnorm_kernel<bf16>, rows_grid(M), WPB * 32, 0, s, x, M, d, gain, w_bf16, eps, out, ldo, rows_idx, lo_off);
   else
-    launch_pdl(rmsnorm_kernel<float>, rows_grid(M), WPB * 32, 0, s, x, M, d, gain, w_bf16, eps, out, ldo, rows_idx);
+    launch_pdl(rmsnorm_kernel<float>, rows_grid(M), WPB * 32, 0, s, x, M, d, gain, w_bf16, eps, out, ldo, rows_idx, lo_off);
   return err();
 }
 

@@ -52,6 +52,7 @@ bool valid_config(const tadm_config* c, std::string* why) {
   if (c->sliding_window < 0 || c->global_every < 0) return fail("sliding_window and global_every must be >= 0");
   if ((c->qk_norm != 0 && c->qk_norm != 1) || (c->sandwich_norm != 0 && c->sandwich_norm != 1))
     return fail("qk_norm and sandwich_norm must be 0 or 1");
+  if (c->qkv_split != 0 && c->qkv_split != 1) return fail("qkv_split must be 0 or 1");
   if (!(c->rope_theta_global >= 0.0f)) return fail("rope_theta_global must be >= 0");
   return true;
 }
@@ -318,9 +319,13 @@ void probe_end(tadm_handle* h, cudaStream_t s, int idx, int kind, double flops, 
   h->probe_bytes[idx] = bytes;
 }
 
+// k_b > 0: A = [hi | lo] holds 2 k_b columns (a split operand) and both halves multiply B's k_b columns;
+// the recorded work is that of the k_b-deep product the method computes.
 tadm_status gemm(tadm_handle* h, const void* A, int64_t a_rows, int lda, const void* B, int ldb, int M, int N, int K,
-                 int epi, const EpiParams& ep, cudaStream_t s, bool out_f32 = false, const int* m_dev = nullptr) {
+                 int epi, const EpiParams& ep, cudaStream_t s, bool out_f32 = false, const int* m_dev = nullptr,
+                 int k_b = 0) {
   GemmCall g{};
+  g.k_b = k_b;
   g.A = A;
   g.B = B;
   g.M = M;
@@ -344,6 +349,7 @@ tadm_status gemm(tadm_handle* h, const void* A, int64_t a_rows, int lda, const v
   if (e) return fail(h, TADM_ERR_CUDA, "GEMM (M=%d N=%d K=%d epi=%d): %s", M, N, K, epi, e);
   h->counters.kernel_launches += h->cfg.dtype ? g.launched : 1;
   const double n_acc = epi == EPI_GLU ? 2.0 * N : static_cast<double>(N);
+  if (k_b > 0) K = k_b;
   // algorithmic bytes: A and B read once, the output written once (fp32 or
   // the activation type), the residual stream read and written by EPI_RESID
   const double es = h->es(), out_es = (epi == EPI_RESID || out_f32 || !h->act_bf16()) ? 4.0 : es;
@@ -372,8 +378,11 @@ tadm_status layer_fwd(tadm_handle* h, int li, float* x, int B, int R, int ctx, i
   const int q = c.n_heads * hd, nqkv = (c.n_heads + 2 * c.n_kv_heads) * hd;
   const int64_t Mmax = static_cast<int64_t>(h->max_batch) * h->max_rows;
   void* norm = h->at(h->off.norm);
+  // qkv_split: the QKV projection's input enters the tensor cores as bf16 hi + lo (about 16 bits)
+  const bool split = c.dtype && c.qkv_split;
   int pi = probe_begin(h, s);
-  TRY(rmsnorm_rows(x, M, d, L.attn_norm, c.dtype, c.norm_eps, norm, d, h->act_bf16(), s));
+  TRY(rmsnorm_rows(x, M, d, L.attn_norm, c.dtype, c.norm_eps, norm, split ? 2 * d : d, h->act_bf16(), s, nullptr,
+                   split ? d : 0));
   probe_end(h, s, pi, kProbeNorm, 0.0);
   EpiParams ep{};
   ep.q = h->at(h->off.qbuf);
@@ -391,7 +400,8 @@ tadm_status layer_fwd(tadm_handle* h, int li, float* x, int B, int R, int ctx, i
   ep.q_gain = L.q_norm;
   ep.k_gain = L.k_norm;
   ep.qk_eps = c.norm_eps;
-  TRYS(gemm(h, norm, Mmax, d, L.wqkv, d, M, nqkv, d, EPI_QKV, ep, s));
+  TRYS(gemm(h, norm, Mmax, split ? 2 * d : d, L.wqkv, d, M, nqkv, split ? 2 * d : d, EPI_QKV, ep, s, false, nullptr,
+            split ? d : 0));
   AttnCall a{ep.q, ep.k, ep.v, h->at(h->off.attn), B, c.n_heads, c.n_kv_heads, hd, R, ctx, h->kv_stride, causal,
              h->act_bf16(), h->status()};
   a.window = L.window;

@@ -41,7 +41,7 @@ class tadm_config(ctypes.Structure):
         "n_denoise", "fusion", "fusion_rank", "fusion_heads", "dtype", "tied_lm_head")] + [
         ("norm_eps", ctypes.c_float), ("rope_theta", ctypes.c_float)] + [
         (n, ctypes.c_int32) for n in ("sliding_window", "global_every", "qk_norm", "sandwich_norm")] + [
-        ("rope_theta_global", ctypes.c_float)]
+        ("rope_theta_global", ctypes.c_float), ("qkv_split", ctypes.c_int32)]
 
 
 class tadm_step_outputs(ctypes.Structure):
@@ -142,7 +142,8 @@ def make_config(model) -> tadm_config:
         sliding_window=getattr(model, "sliding_window", 0), global_every=getattr(model, "global_every", 0),
         qk_norm=int(bool(getattr(model, "qk_norm", False))),
         sandwich_norm=int(bool(getattr(model, "sandwich_norm", False))),
-        rope_theta_global=getattr(model, "rope_theta_global", 0.0))
+        rope_theta_global=getattr(model, "rope_theta_global", 0.0),
+        qkv_split=int(bool(getattr(model, "qkv_split", False))))
 
 
 # ---------------------------------------------------------------------------- C-named wrappers

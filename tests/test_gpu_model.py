@@ -455,7 +455,7 @@ def test_block_mode_fp32_positions_and_context_exact(T):
     tm.tadm_sync_status()
 
 
-@pytest.mark.parametrize("case", ["small_workload_dims", "test_model"])
+@pytest.mark.parametrize("case", ["small_workload_dims", "small_workload_dims_qkv_split", "test_model"])
 def test_committed_token_agreement_teacher_forced(T, case):
     """North-star token agreement on a large sample: the GPU generates step by
     step; at every step the oracle receives the same canvas (teacher forcing)
@@ -465,15 +465,19 @@ def test_committed_token_agreement_teacher_forced(T, case):
     vocab 32768) on a 256-position canvas, batch 8, 32 steps of 6 commits.
     tests/bf16_floor.py runs this very protocol with the oracle's arithmetic
     rounded to bf16 at every tensor-core operand and stores the agreement it
-    reaches (tests/golden/bf16_floor_small.json): the GPU must agree on at
-    least as many confidence-selected commits as that ideal bf16 path, less
-    six (rounding-order noise: near-ties flip either way), and on >= 99%.
+    reaches (tests/golden/bf16_floor_small.json, 1479/1488 = 99.40%): with
+    plain bf16 operands the GPU must agree on at least as many
+    confidence-selected commits as that ideal bf16 path.
+    small_workload_dims_qkv_split: the same model with the QKV projections'
+    input split into bf16 hi + lo (qkv_split), the site that carries most of
+    the flips (the floor's per-site runs); the benchmark spec's bound, >= 99.5%.
     test_model: the 4-layer d 256 vocab 4096 test model, batch 16 (>= 99%).
     Forced commits (last step of the block) are reported."""
     floor = None
-    if case == "small_workload_dims":
-        m = wl.WORKLOADS["small"].model
-        B, P, G, Tn, K, gate = 8, 64, 192, 32, 4, 0.99
+    if case.startswith("small_workload_dims"):
+        split = case.endswith("qkv_split")
+        m = wl.ModelConfig(**{**wl.WORKLOADS["small"].model.__dict__, "qkv_split": split})
+        B, P, G, Tn, K, gate = 8, 64, 192, 32, 4, (0.995 if split else 0.99)
         with open(os.path.join(os.path.dirname(__file__), "golden", "bf16_floor_small.json")) as f:
             floor = json.load(f)
         fp = floor["protocol"]
@@ -507,5 +511,33 @@ def test_committed_token_agreement_teacher_forced(T, case):
     if floor is not None:
         print(f"[agreement {case}] ideal bf16 path: {floor['selected_ok']}/{floor['selected']}")
         assert agg.committed == floor["selected"]
-        assert agg.committed_ok >= floor["selected_ok"] - 6, (agg.committed_ok, floor["selected_ok"])
+        if not split:
+            assert agg.committed_ok >= floor["selected_ok"], (agg.committed_ok, floor["selected_ok"])
     assert agg.masked_ok / agg.masked >= 0.95
+
+
+def test_qkv_split_removes_the_qkv_input_rounding(T):
+    """qkv_split carries the QKV projections' input as bf16 hi + lo.  On the
+    small workload's model the logits error against the oracle must drop by
+    about the share of that rounding site (tests/bf16_floor.py: an exact-
+    arithmetic path with bf16 operands has rel-L2 5.80e-3, and 4.64e-3 with
+    the QKV input exact, a ratio of 0.80), and both paths run the same
+    kernels otherwise."""
+    errs = {}
+    for split in (False, True):
+        m = wl.ModelConfig(**{**wl.WORKLOADS["small"].model.__dict__, "qkv_split": split})
+        w = wl.Workload("t", m, batch=2, prompt_len=64, gen_len=192, steps_per_block=32, K=4)
+        B, R = 2, 256
+        tm, o = setup(T, m, B, R, seed=7, affine_std=0.0)
+        z = wl.random_canvas(w, B, R, 0.3, seed=5, start=64)
+        cache = tm.new_cache(B, R)
+        tm.tadm_reset(B)
+        tm.tadm_anchor_forward(torch.from_numpy(z).cuda(), 32, cache)
+        g = gpu_step(tm, z, 32, 32, 192, cache)
+        sess = o.new_session(B)
+        ref = o.denoise_logits(sess, z, o.anchor_forward(sess, z))
+        errs[split] = rel_l2(g["logits"], ref)
+        tm.close()
+    print(f"[qkv_split] logits rel-L2 plain {errs[False]:.3e}, split {errs[True]:.3e}, "
+          f"ratio {errs[True] / errs[False]:.3f}")
+    assert errs[True] < 0.9 * errs[False]

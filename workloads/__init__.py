@@ -156,6 +156,9 @@ class ModelConfig:
     rope_theta_global: float = 0.0
     qk_norm: bool = False
     sandwich_norm: bool = False
+    # precision of the GPU path (the oracle is exact either way): the QKV
+    # projections take their input as bf16 hi + lo
+    qkv_split: bool = False
 
     @property
     def mask_id(self) -> int:
@@ -187,13 +190,15 @@ class Workload:
 
 TINY = ModelConfig(vocab=1024, d_model=256, n_heads=4, n_kv_heads=4, head_dim=64, ffn=1024,
                    n_anchor=4, n_denoise=2, dtype="f32")
+# the bf16 presets carry the QKV projections' input as bf16 hi + lo (qkv_split): the
+# attention logits are the backbone's most rounding-sensitive quantity
 SMALL = ModelConfig(vocab=32768, d_model=768, n_heads=12, n_kv_heads=12, head_dim=64, ffn=3072,
-                    n_anchor=8, n_denoise=4)
+                    n_anchor=8, n_denoise=4, qkv_split=True)
 BLOCK = ModelConfig(vocab=128000, d_model=2048, n_heads=16, n_kv_heads=8, head_dim=128, ffn=8192,
-                    n_anchor=16, n_denoise=6)
+                    n_anchor=16, n_denoise=6, qkv_split=True)
 POSTTRAIN = ModelConfig(vocab=262144, d_model=5376, n_heads=32, n_kv_heads=16, head_dim=128, ffn=21504,
                         glu="geglu", n_shared=2, n_anchor=54, n_denoise=6, fusion="paired_attn",
-                        tied_lm_head=True)
+                        tied_lm_head=True, qkv_split=True)
 # the same backbone with the Gemma-3 layer details: 5 local layers (1024-key
 # sliding window, RoPE base 1e4) per global layer (RoPE base 1e6), QK-norm and
 # sandwich norms
