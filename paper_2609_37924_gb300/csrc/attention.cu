@@ -23,6 +23,7 @@
 // fp32: one warp per query row on the CUDA cores.
 #include <cudaTypedefs.h>
 #include <algorithm>
+#include <cstdlib>
 #include <mutex>
 
 #include "kernels.h"
@@ -393,6 +394,307 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD, TKV>::MIN_BLOCKS)
   }
 }
 
+// ------------------------------------------------------ pipelined variant, hd 64
+// The same computation for hd 64 without key splits or a window, with the
+// tensor pipe and the softmax overlapped: 64-key tiles, S double-buffered in
+// TMEM (S0, S1, then O: 192 of the 256 columns, two CTAs per SM) and P
+// double-buffered in shared memory, four K / V stages.  The MMA thread
+// issues S(i) as soon as the softmax has released its S buffer (tile i - 2),
+// then O += P(i-1) V(i-1): while the softmax threads exponentiate tile i,
+// the tensor pipe already computes S(i+1).  Ordering facts the softmax relies
+// on (tcgen05 operations of one thread complete in issue order): P V(i-2) is
+// issued before S(i), so when S(i) is complete the P buffer of tile i and
+// the O accumulator up to tile i-2 are settled; a rescale of O at tile i
+// waits for P V(i-1) on o_full.
+struct AttnDbCfg {
+  static constexpr int HD = 64, TKV = 64, STAGES = 4;
+  static constexpr int Q_BYTES = 16384;               // 128 rows x 64 dims, one swizzle atom
+  static constexpr int K_BYTES = TKV * 128;           // 64 keys x 64 dims
+  static constexpr int V_BYTES = HD * 128;            // 64 dims x 64 keys (V^T)
+  static constexpr int P_BYTES = 16384;               // 128 rows x 64 keys
+  static constexpr int SMEM = Q_BYTES + STAGES * (K_BYTES + V_BYTES) + 2 * P_BYTES + 256;
+  static constexpr int TMEM_COLS = 256;               // S0 [0, 64), S1 [64, 128), O [128, 192)
+};
+
+__global__ void __launch_bounds__(192, 2)
+    attn_db_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                   const AttnTcArgs args) {
+  pdl_enter();
+  using C = AttnDbCfg;
+  constexpr int HD = C::HD, TKV = C::TKV, NST = C::STAGES;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = smem_raw;
+  if (smem_u32(smem_raw) & 1023) {
+    // the swizzled operand layout needs 1024-byte alignment: refuse (uniform exit, nothing started)
+    if (threadIdx.x == 0 && args.status) atomicOr(args.status, kErrLayout);
+    return;
+  }
+  uint8_t* sQ = smem;
+  uint8_t* sK = sQ + C::Q_BYTES;
+  uint8_t* sV = sK + NST * C::K_BYTES;
+  uint8_t* sP = sV + NST * C::V_BYTES;                 // two P buffers
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sP + 2 * C::P_BYTES);
+  uint64_t* q_full = bars;
+  uint64_t* kv_full = bars + 1;        // [NST]
+  uint64_t* kv_empty = bars + 5;       // [NST]
+  uint64_t* s_full = bars + 9;         // [2]
+  uint64_t* s_free = bars + 11;        // [2]
+  uint64_t* p_full = bars + 13;        // [2]
+  uint64_t* o_full = bars + 15;        // one completion per P V
+  uint64_t* drain = bars + 16;
+  uint64_t* o_done = bars + 17;        // the last P V is complete
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 18);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int m0 = blockIdx.x * TQ, hk = blockIdx.y, b = blockIdx.z;
+  const int group = args.n_heads / args.n_kv_heads, n_virt = group * args.rows;
+  const int v_last = min(m0 + TQ, n_virt) - 1;
+  const int r_max = (m0 / args.rows != v_last / args.rows) ? args.rows - 1 : v_last % args.rows;
+  const int kv_end = args.causal ? min(args.kv_len, args.ctx + r_max + 1) : args.kv_len;
+  const int n_tiles = (kv_end + TKV - 1) / TKV;
+
+  if (threadIdx.x == 0) {
+    mbar_init(q_full, 128);
+    for (int s = 0; s < NST; ++s) {
+      mbar_init(&kv_full[s], 1);
+      mbar_init(&kv_empty[s], 1);
+    }
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(&s_full[s], 1);
+      mbar_init(&s_free[s], 128);
+      mbar_init(&p_full[s], 128);
+    }
+    mbar_init(o_full, 1);
+    mbar_init(drain, 1);
+    mbar_init(o_done, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+    tma_prefetch_desc(&tmK);
+    tma_prefetch_desc(&tmV);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, C::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const uint32_t t_o = tmem + 2 * TKV;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------------------- producer
+      int issued[NST];
+      for (int s = 0; s < NST; ++s) issued[s] = 0;
+      const int z = b * args.n_kv_heads + hk;
+      for (int i = 0; i < n_tiles; ++i) {
+        const int st = i % NST;
+        if (!mbar_wait_bounded(&kv_empty[st], ((i / NST) & 1) ^ 1, abort_flag, args.status)) break;
+        mbar_arrive_expect_tx(&kv_full[st], C::K_BYTES + C::V_BYTES);
+        tma_load_3d(sK + st * C::K_BYTES, &tmK, &kv_full[st], 0, i * TKV, z);
+        tma_load_3d(sV + st * C::V_BYTES, &tmV, &kv_full[st], i * TKV, 0, z);
+        ++issued[st];
+        if (i + NST < n_tiles) {     // the stage ring holds tiles i .. i+3; L2 fetches tile i+4 meanwhile
+          tma_prefetch_3d(&tmK, 0, (i + NST) * TKV, z);
+          tma_prefetch_3d(&tmV, (i + NST) * TKV, 0, z);
+        }
+      }
+      // every copy started here has landed before the CTA may exit
+      volatile int never = 0;
+      for (int s = 0; s < NST; ++s)
+        if (issued[s] > 0) mbar_wait_bounded(&kv_full[s], (issued[s] - 1) & 1, &never, args.status);
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ------------------------------------------------------------- MMA issuer
+      constexpr uint32_t idesc_s = idesc_bf16_f32(TQ, TKV);
+      constexpr uint32_t idesc_o = idesc_bf16_f32(TQ, HD);
+      bool ok = n_tiles > 0 && mbar_wait_bounded(q_full, 0, abort_flag, args.status);
+      const uint32_t q0 = smem_u32(sQ);
+      for (int i = 0; ok && i <= n_tiles; ++i) {
+        if (i < n_tiles) {
+          // S(i) = Q K(i)^T into S buffer i & 1, once the softmax has released it (tile i - 2)
+          const int st = i % NST, sb = i & 1;
+          if (!mbar_wait_bounded(&kv_full[st], (i / NST) & 1, abort_flag, args.status)) break;
+          if (i >= 2 && !mbar_wait_bounded(&s_free[sb], ((i - 2) >> 1) & 1, abort_flag, args.status)) break;
+          tc_fence_after();
+          const uint32_t k0 = smem_u32(sK + st * C::K_BYTES);
+#pragma unroll
+          for (int kk = 0; kk < HD / 16; ++kk)
+            umma_bf16(tmem + sb * TKV, sdesc_kmajor_sw128(q0 + kk * 32), sdesc_kmajor_sw128(k0 + kk * 32), idesc_s,
+                      kk != 0);
+          umma_commit(&s_full[sb]);
+        }
+        if (i >= 1) {
+          // O += P(j) V(j) for the previous tile, once its probabilities are in shared memory
+          const int j = i - 1, pb = j & 1, st = j % NST;
+          if (!mbar_wait_bounded(&p_full[pb], (j >> 1) & 1, abort_flag, args.status)) break;
+          tc_fence_after();
+          const uint32_t p0 = smem_u32(sP + pb * C::P_BYTES), v0 = smem_u32(sV + st * C::V_BYTES);
+#pragma unroll
+          for (int kk = 0; kk < TKV / 16; ++kk)
+            umma_bf16(t_o, sdesc_kmajor_sw128(p0 + kk * 32), sdesc_kmajor_sw128(v0 + kk * 32), idesc_o,
+                      (j != 0) || (kk != 0));
+          umma_commit(o_full);
+          umma_commit(&kv_empty[st]);
+          if (j == n_tiles - 1) umma_commit(o_done);
+        }
+      }
+      umma_commit(drain);
+      volatile int never = 0;
+      mbar_wait_bounded(drain, 0, &never, args.status);
+    }
+  } else {
+    // --------------------------------------------------------------- softmax
+    // One virtual query row per thread (row = TMEM lane), the reference-max
+    // scheme of attn_tc_kernel (O rescaled only when a tile's max exceeds the
+    // reference by more than 8 in log2 units).
+    const int quad = warp & 3;
+    const int row = quad * 32 + lane;
+    const uint32_t lane_off = static_cast<uint32_t>(quad * 32) << 16;
+    const int v = m0 + row;
+    const bool v_ok = v < n_virt;
+    const int qh = hk * group + (v_ok ? v / args.rows : 0);
+    const int qr = v_ok ? v % args.rows : 0;
+    const int qpos = args.ctx + qr;
+    {
+      const uint4* src = reinterpret_cast<const uint4*>(
+          args.q + ((static_cast<size_t>(b) * args.n_heads + qh) * args.rows + qr) * HD);
+      uint8_t* dst = sQ + row * 128;
+#pragma unroll
+      for (int c = 0; c < 8; ++c) {
+        const uint4 val = v_ok ? src[c] : make_uint4(0, 0, 0, 0);
+        *reinterpret_cast<uint4*>(dst + ((c ^ (row & 7)) << 4)) = val;
+      }
+      fence_proxy_async_smem();
+      mbar_arrive(q_full);
+    }
+    float m_ref = -INFINITY, l_run = 0.0f;
+    bool ok = true;
+    const uint64_t sc2 = f2_pack(args.scale_log2, args.scale_log2);
+    const int kv_hi = args.causal ? min(kv_end, qpos + 1) : kv_end;
+    for (int i = 0; i < n_tiles; ++i) {
+      const int sb = i & 1;
+      if (!warp_wait_bounded(&s_full[sb], (i >> 1) & 1, abort_flag, args.status)) { ok = false; break; }
+      tc_fence_after();
+      const uint32_t t_s = tmem + sb * TKV + lane_off;
+      const int lim = kv_hi - i * TKV;                                // visible keys of this tile
+      const bool masked = __any_sync(0xffffffffu, lim < TKV);
+      uint32_t ra[32], rb[32];
+      tmem_ld32_nowait(t_s, ra);
+      tmem_ld32_nowait(t_s + 32, rb);
+      tmem_wait_ld(ra);
+      tmem_bind(rb);
+      // S is in registers: its TMEM buffer goes back to the MMA thread (S(i+2)) at once
+      tc_fence_before();
+      mbar_arrive(&s_free[sb]);
+      // pass 1: row max over the tile (both halves stay in registers for pass 2)
+      float mxa[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+      if (masked) {
+#pragma unroll
+        for (int k = 0; k < 32; ++k)
+          mxa[k & 3] = fmax3(mxa[k & 3], k < lim ? __uint_as_float(ra[k]) : -INFINITY,
+                             32 + k < lim ? __uint_as_float(rb[k]) : -INFINITY);
+      } else {
+#pragma unroll
+        for (int k = 0; k < 32; ++k) mxa[k & 3] = fmax3(mxa[k & 3], __uint_as_float(ra[k]), __uint_as_float(rb[k]));
+      }
+      const float m_tile = fmax3(fmaxf(mxa[0], mxa[1]), mxa[2], mxa[3]) * args.scale_log2;
+      float m_new = m_ref, factor = 1.0f;
+      if (m_ref == -INFINITY) {
+        m_new = m_tile;
+      } else if (m_tile > m_ref + 8.0f) {
+        m_new = m_tile;
+        factor = ex2_approx(m_ref - m_tile);
+      }
+      if (__any_sync(0xffffffffu, factor != 1.0f)) {
+        // O holds tiles 0 .. i-1 once P V(i-1) is complete (i >= 1 here)
+        if (!warp_wait_bounded(o_full, (i - 1) & 1, abort_flag, args.status)) { ok = false; break; }
+        tc_fence_after();
+#pragma unroll
+        for (int c = 0; c < HD / 32; ++c) {
+          uint32_t ro[32];
+          tmem_ld32_nowait(t_o + lane_off + 32 * c, ro);
+          tmem_wait_ld(ro);
+#pragma unroll
+          for (int k = 0; k < 32; ++k) ro[k] = __float_as_uint(__uint_as_float(ro[k]) * factor);
+          tmem_st32(t_o + lane_off + 32 * c, ro);
+        }
+        tmem_wait_st();
+        l_run *= factor;
+      }
+      // pass 2: P = 2^(s * scale - m_new) as bf16 into P buffer i & 1 (free: P V(i-2) is complete)
+      uint8_t* prow = sP + sb * C::P_BYTES + row * 128;
+      const uint64_t negm2 = f2_pack(-m_new, -m_new);
+      uint64_t ps2[2] = {0, 0};
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        const uint32_t* r = c ? rb : ra;
+        uint32_t pk[16];
+#pragma unroll
+        for (int k = 0; k < 32; k += 2) {
+          float x0, x1;
+          f2_unpack(f2_fma(f2_pack(__uint_as_float(r[k]), __uint_as_float(r[k + 1])), sc2, negm2), x0, x1);
+          float p0 = ex2_approx(x0), p1 = ex2_approx(x1);
+          if (masked) {
+            p0 = 32 * c + k < lim ? p0 : 0.0f;
+            p1 = 32 * c + k + 1 < lim ? p1 : 0.0f;
+          }
+          ps2[(k >> 1) & 1] = f2_add(ps2[(k >> 1) & 1], f2_pack(p0, p1));
+          __nv_bfloat162 t = __floats2bfloat162_rn(p0, p1);
+          pk[k / 2] = *reinterpret_cast<uint32_t*>(&t);
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const int chunk = c * 4 + q;
+          *reinterpret_cast<uint4*>(prow + ((chunk ^ (row & 7)) << 4)) =
+              make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+        }
+      }
+      float a0, a1, b0, b1;
+      f2_unpack(ps2[0], a0, a1);
+      f2_unpack(ps2[1], b0, b1);
+      l_run += (a0 + a1) + (b0 + b1);
+      m_ref = m_new;
+      fence_proxy_async_smem();
+      mbar_arrive(&p_full[sb]);
+    }
+    // o_done, not o_full: at this point P V(n-2) may still be running as well
+    if (ok && n_tiles > 0 && warp_wait_bounded(o_done, 0, abort_flag, args.status)) {
+      tc_fence_after();
+      const float inv = l_run > 0.0f ? 1.0f / l_run : 0.0f;
+      bf16* orow = args.o + (static_cast<size_t>(b) * args.rows + qr) * args.n_heads * HD + static_cast<size_t>(qh) * HD;
+#pragma unroll
+      for (int c = 0; c < HD / 32; ++c) {
+        uint32_t ro[32];
+        tmem_ld32_nowait(t_o + lane_off + 32 * c, ro);
+        tmem_wait_ld(ro);
+        if (v_ok) {
+#pragma unroll
+          for (int k = 0; k < 32; k += 8) {
+            __nv_bfloat162 w0 = __floats2bfloat162_rn(__uint_as_float(ro[k]) * inv, __uint_as_float(ro[k + 1]) * inv);
+            __nv_bfloat162 w1 = __floats2bfloat162_rn(__uint_as_float(ro[k + 2]) * inv, __uint_as_float(ro[k + 3]) * inv);
+            __nv_bfloat162 w2 = __floats2bfloat162_rn(__uint_as_float(ro[k + 4]) * inv, __uint_as_float(ro[k + 5]) * inv);
+            __nv_bfloat162 w3 = __floats2bfloat162_rn(__uint_as_float(ro[k + 6]) * inv, __uint_as_float(ro[k + 7]) * inv);
+            *reinterpret_cast<uint4*>(orow + 32 * c + k) =
+                make_uint4(*reinterpret_cast<uint32_t*>(&w0), *reinterpret_cast<uint32_t*>(&w1),
+                           *reinterpret_cast<uint32_t*>(&w2), *reinterpret_cast<uint32_t*>(&w3));
+          }
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
 // Merges the split partials of one virtual row per warp, in split order:
 // m* = max m_s, O = sum 2^(m_s - m*) O_s / sum 2^(m_s - m*) l_s.
 template <int HD>
@@ -519,6 +821,43 @@ const char* launch_tc_win(const AttnCall& a, cudaStream_t s) {
     if (e != cudaSuccess) return cudaGetErrorString(e);
   }
   return nullptr;
+}
+
+// The pipelined hd-64 kernel: whenever no key split is wanted (the CTAs of
+// the launch fill the SMs) and no window hides keys.  TADM_ATTN_DB=0 keeps
+// attn_tc_kernel for every shape.
+bool attn_db_enabled() {
+  static const bool on = [] {
+    const char* e = getenv("TADM_ATTN_DB");
+    return !(e && e[0] == '0');
+  }();
+  return on;
+}
+
+const char* launch_db(const AttnCall& a, cudaStream_t s) {
+  using C = AttnDbCfg;
+  if (!encoder()) return "cuTensorMapEncodeTiled is unavailable";
+  const int kv_len = a.ctx + a.rows;
+  CUtensorMap mk, mv;
+  if (!map3d(&mk, a.k, C::HD, kv_len, static_cast<uint64_t>(a.batch) * a.n_kv_heads, C::HD * 2ull,
+             static_cast<uint64_t>(a.kv_stride) * C::HD * 2, C::TKV) ||
+      !map3d(&mv, a.v, kv_len, C::HD, static_cast<uint64_t>(a.batch) * a.n_kv_heads, a.kv_stride * 2ull,
+             static_cast<uint64_t>(a.kv_stride) * C::HD * 2, C::HD))
+    return "attention tensor map encode failed";
+  static bool attr = false;
+  if (!attr) {
+    if (cudaFuncSetAttribute(attn_db_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM) != cudaSuccess)
+      return "attention smem attribute failed";
+    attr = true;
+  }
+  const int group = a.n_heads / a.n_kv_heads, n_virt = group * a.rows;
+  const int n_vtiles = (n_virt + TQ - 1) / TQ;
+  AttnTcArgs args{static_cast<const bf16*>(a.q), a.rows, a.ctx, kv_len, a.n_heads, a.n_kv_heads, a.causal, 0,
+                  1.4426950408889634f / sqrtf(static_cast<float>(C::HD)), static_cast<bf16*>(a.o),
+                  n_vtiles, 1, 0, nullptr, nullptr, a.status};
+  launch_pdl(attn_db_kernel, dim3(n_vtiles, a.n_kv_heads, a.batch), 192, C::SMEM, s, mk, mv, args);
+  const cudaError_t e = cudaGetLastError();
+  return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
 }
 
 // the windowed kernel only where the window hides keys (window < ctx + rows)
@@ -820,7 +1159,16 @@ const char* attention(const AttnCall& a, cudaStream_t s) {
     // tcgen05 whenever the V^T rows are 16-byte aligned for TMA (the library's
     // KV buffers always are); 64-key tiles for hd 128 with few query rows
     const bool tc = a.kv_stride % 8 == 0 && (reinterpret_cast<uintptr_t>(a.q) & 15) == 0;
-    if (a.head_dim == 64) return tc ? launch_tc<64, 128>(a, s) : (launch_bf16<64>(a, s) == cudaSuccess ? nullptr : "attention launch failed");
+    if (a.head_dim == 64) {
+      if (!tc) return launch_bf16<64>(a, s) == cudaSuccess ? nullptr : "attention launch failed";
+      int dev = 0, n_sms = 0;
+      cudaGetDevice(&dev);
+      cudaDeviceGetAttribute(&n_sms, cudaDevAttrMultiProcessorCount, dev);
+      const int ctas = ((a.n_heads / a.n_kv_heads) * a.rows + TQ - 1) / TQ * a.n_kv_heads * a.batch;
+      const bool window_cuts = a.window > 0 && a.window < a.ctx + a.rows;
+      if (attn_db_enabled() && !window_cuts && ctas > n_sms) return launch_db(a, s);
+      return launch_tc<64, 128>(a, s);
+    }
     if (a.head_dim == 128) {
       if (!tc) return launch_bf16<128>(a, s) == cudaSuccess ? nullptr : "attention launch failed";
       return (a.n_heads / a.n_kv_heads) * a.rows < 2 * TQ ? launch_tc<128, 64>(a, s) : launch_tc<128, 128>(a, s);

@@ -72,7 +72,10 @@ def test_gemm_f32_cuda_cores(T, M, N, K):
     (128, 4, 2, 260, 0, False, 4), (128, 2, 2, 512, 200, True, 0), (64, 2, 1, 200, 0, False, 1),
     # short rows on tcgen05: GQA group packing, heads straddling a 128-row tile, causal
     (128, 4, 2, 32, 37, False, 3), (128, 16, 8, 32, 200, True, 0), (64, 4, 2, 48, 40, True, 0),
-    (128, 2, 1, 100, 130, True, 2), (64, 8, 2, 20, 300, False, 0)])
+    (128, 2, 1, 100, 130, True, 2), (64, 8, 2, 20, 300, False, 0),
+    # hd 64 launches of more CTAs than SMs run the pipelined kernel (double-buffered S and P, 64-key
+    # tiles): bidirectional, causal with a context and a ragged last tile, GQA
+    (64, 12, 12, 1024, 0, True, 0), (64, 16, 8, 700, 100, True, 0), (64, 16, 4, 520, 44, False, 0)])
 def test_attention_bf16(T, hd, Hq, Hkv, rows, ctx, causal, pad):
     B, stride = 2, ctx + rows + pad
     q, qd = bf16_tensor((B, Hq, rows, hd), 5)
