@@ -45,6 +45,8 @@ def parse():
     ap.add_argument("--T", type=int, default=None,
                     help="override reverse steps per block (short runs for launch-list profiles)")
     ap.add_argument("--G", type=int, default=None, help="override the generation length (short profiling runs)")
+    ap.add_argument("--layers", default=None,
+                    help="override L_S,L_A,L_D (reduced-depth profiling runs of a wide model, e.g. 0,1,1)")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
     ap.add_argument("--sampler", default="topk", choices=["topk", "remdm-cap", "remdm-loop", "entropy-bound"],
                     help="with --sweep-workloads: the confidence top-k sampler, ReMDM (App. C.2 settings) or the "
@@ -61,7 +63,9 @@ def parse():
     ap.add_argument("--configs", default="block,posttrain",
                     help="at N = 1: workloads also timed whole (K = 1 and the workload's K) and reported under "
                          "'configs' in the same JSON line ('' for none)")
-    ap.add_argument("--config-steps", type=int, default=2, help="timed generations per K of each extra workload")
+    ap.add_argument("--config-steps", type=int, default=1, help="timed generations per K of each extra workload")
+    ap.add_argument("--configs-only", action="store_true",
+                    help="time only the extra workloads (one JSON line with their results)")
     ap.add_argument("--config-warmup", type=int, default=2,
                     help="untimed generations per K of each extra workload (the second one captures the CUDA graph)")
     return ap.parse_args()
@@ -294,6 +298,9 @@ def gpu_arm(args):
         over["gen_len"] = args.G
     if args.qkv_split is not None:
         over["model_qkv_split"] = bool(args.qkv_split)
+    if args.layers:
+        ls, la, ld = (int(x) for x in args.layers.split(","))
+        over.update(model_n_shared=ls, model_n_anchor=la, model_n_denoise=ld)
     w = wl.get_workload(args.workload, **over)
     K = args.K or w.K
     m = w.model
@@ -509,7 +516,11 @@ def config_leg(name: str, steps: int, warmup: int, peaks, local: int) -> dict:
                         "launches": int(sum(v["launches"] for v in gemm)),
                         "peak_source": "MEASURED_PEAKS.json (sustained bf16, HBM copy)" if peaks else "fallback"},
            "others_ms_per_generation": {k: v["ms"] for k, v in kinds.items()
-                                        if k in ("attention", "norms", "attention_short_rows")}}
+                                        if k in ("attention", "norms", "attention_short_rows")},
+           "gemm_by_epilogue": {k: {"ms": round(v["ms"], 2), "launches": v["launches"],
+                                    "tflops": round(v["tflops"], 1),
+                                    "gbs": round(v["bytes"] / (v["ms"] / 1e3) / 1e9, 1) if v["ms"] > 0 else None}
+                                for k, v in kinds.items() if k not in ("attention", "norms", "attention_short_rows")}}
     tm.close()
     del tm, dev_w
     return leg
@@ -681,6 +692,14 @@ def main():
         import __graft_entry__
         __graft_entry__.build()
         kernel_bench(args)
+        return
+    if args.configs_only:
+        import __graft_entry__
+        import torch
+        __graft_entry__.build()
+        torch.cuda.set_device(0)
+        print(json.dumps({name: config_leg(name, args.config_steps, args.config_warmup, load_peaks(), 0)
+                          for name in args.configs.split(",") if name}), flush=True)
         return
     if args.impl == "reference":
         reference_arm(args)

@@ -115,7 +115,9 @@ struct TcArgs {
   int staged;              // bf16 outputs go through the per-warp boxes and TMA stores
   int b_split;             // >0: B tile = 128 rows at n*128 and 128 rows at b_split + n*128
   int n_tiles_n;
-  int kb_wrap;             // > 0: B's k-block of A's k-block kb is kb % kb_wrap (split hi + lo operand)
+  int kb_wrap;             // > 0: split hi + lo operand of kb_wrap k-blocks per half: k-block kb reads A's
+                           // k-block (kb odd ? kb_wrap : 0) + kb / 2 and B's k-block kb / 2, so that the two
+                           // reads of a B tile follow each other (the second one hits L2)
   int* status;
   const int* m_dev;        // optional device row count (<= M): tiles past it are skipped
   EpiParams ep;
@@ -206,8 +208,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait_bounded(&empty[stage], phase ^ 1, abort_flag, args.status)) { ok = false; break; }
           mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
-          tma_load_2d(sA + stage * A_BYTES, &tmA, &full[stage], kb * BK, mb * BM);
-          const int kbb = args.kb_wrap > 0 ? kb % args.kb_wrap : kb;
+          const int kba = args.kb_wrap > 0 ? (kb & 1) * args.kb_wrap + (kb >> 1) : kb;
+          const int kbb = args.kb_wrap > 0 ? kb >> 1 : kb;
+          tma_load_2d(sA + stage * A_BYTES, &tmA, &full[stage], kba * BK, mb * BM);
           if (args.b_split > 0) {
             tma_load_2d(sB + stage * B_BYTES, &tmB, &full[stage], kbb * BK, nb * (BN / 2));
             tma_load_2d(sB + stage * B_BYTES + B_BYTES / 2, &tmB, &full[stage], kbb * BK,
@@ -402,8 +405,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
           if (!mbar_wait_bounded(&empty[stage], phase ^ 1, abort_flag, args.status)) { ok = false; break; }
           if (leader) mbar_arrive_expect_tx(&full[stage], 2 * P_STAGE_BYTES);
           const uint32_t fb = full_l0 + 8u * stage;
-          tma_load_2d_pair(sA + stage * P_A_BYTES, &tmA, fb, kb * BK, mb * BM);
-          tma_load_2d_pair(sB + stage * P_B_BYTES, &tmB, fb, (args.kb_wrap > 0 ? kb % args.kb_wrap : kb) * BK, brow);
+          const int kba = args.kb_wrap > 0 ? (kb & 1) * args.kb_wrap + (kb >> 1) : kb;
+          const int kbb = args.kb_wrap > 0 ? kb >> 1 : kb;
+          tma_load_2d_pair(sA + stage * P_A_BYTES, &tmA, fb, kba * BK, mb * BM);
+          tma_load_2d_pair(sB + stage * P_B_BYTES, &tmB, fb, kbb * BK, brow);
           if (++stage == P_STAGES) { stage = 0; phase ^= 1; }
         }
         if (!ok) break;
@@ -646,13 +651,13 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
   a.kb_per_split = kblocks;
   a.ldp = a.n_tiles_n * BN;
   // CTA-pair tiles that keep >= 40% of the SMs busy beat split-K: no fp32
-  // partials, no reduction launches.  Residual and fusion-output GEMMs (N =
-  // d) whose 256-wide pair tiles would occupy at most half the SMs use
-  // 256 x 128 pair tiles instead.
+  // partials, no reduction launches.  Residual, fusion-output and QKV GEMMs
+  // whose 256-wide pair tiles would occupy at most half the SMs (the
+  // weight-streaming block steps) use 256 x 128 pair tiles instead.
   const int m_pairs = (g.M + 2 * BM - 1) / (2 * BM);
   const bool pair_ok = g_pair_mma && g.M > BM;
-  const bool narrow = pair_ok && (g.epi == EPI_RESID || g.epi == EPI_FUSION2) &&
-                      m_pairs * a.n_tiles_n * 4 <= g_num_sms;
+  const bool narrow_kind = g.epi == EPI_RESID || g.epi == EPI_FUSION2 || (g.epi == EPI_QKV && 128 % g.ep.head_dim == 0);
+  const bool narrow = pair_ok && narrow_kind && m_pairs * a.n_tiles_n * 4 <= g_num_sms;
   const int pair_units = narrow ? m_pairs * ((g.N + 127) / 128) : m_pairs * a.n_tiles_n;
   const bool pairs_fill = pair_ok && 2 * pair_units * 5 >= g_num_sms * 2;
   if (g.split_buf && !g.m_dev && !pairs_fill && tiles * 3 < g_num_sms * 2 && kblocks >= 8) {
@@ -674,8 +679,9 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
     if (!make_map(&tbh, g.B, b_rows, k_b, g.ldb, 64)) return "tensor map (B, quarter tiles) encode failed";
     TcArgs a2 = a;
     a2.n_tiles_n = (g.N + 127) / 128;
-    cudaError_t e = g.epi == EPI_RESID ? launch_epi_pair<EPI_RESID, 128>(ta, tbh, tc, tc2, a2, pair_units, s)
-                                       : launch_epi_pair<EPI_FUSION2, 128>(ta, tbh, tc, tc2, a2, pair_units, s);
+    cudaError_t e = g.epi == EPI_RESID  ? launch_epi_pair<EPI_RESID, 128>(ta, tbh, tc, tc2, a2, pair_units, s)
+                    : g.epi == EPI_QKV  ? launch_epi_pair<EPI_QKV, 128>(ta, tbh, tc, tc2, a2, pair_units, s)
+                                        : launch_epi_pair<EPI_FUSION2, 128>(ta, tbh, tc, tc2, a2, pair_units, s);
     if (e != cudaSuccess) return cudaGetErrorString(e);
     const_cast<GemmCall&>(g).launched = 1;
     return nullptr;

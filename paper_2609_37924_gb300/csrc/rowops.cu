@@ -291,6 +291,59 @@ __global__ void post_norm_add_kernel(float* __restrict__ x, const float* __restr
   }
 }
 
+// The same with one 256-thread block per row, for few rows of a wide model
+// (a block step of the post-train backbone: 256 rows of 5376).
+template <class T>
+__global__ void __launch_bounds__(256) post_norm_add_block_kernel(float* __restrict__ x, const float* __restrict__ y,
+                                                                  int d, const void* __restrict__ g_post,
+                                                                  const void* __restrict__ g_next, int w_bf16,
+                                                                  float eps, void* __restrict__ out) {
+  pdl_enter();
+  __shared__ float red[2][8];
+  const int m = blockIdx.x, lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  float* xr = x + static_cast<size_t>(m) * d;
+  const float* yr = y + static_cast<size_t>(m) * d;
+  float ss = 0.0f;
+  for (int j = threadIdx.x * 4; j < d; j += 1024) {
+    const float4 v = *reinterpret_cast<const float4*>(yr + j);
+    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+  }
+  ss = warp_sum(ss);
+  if (lane == 0) red[0][w] = ss;
+  __syncthreads();
+  float tot = 0.0f;
+#pragma unroll
+  for (int k = 0; k < 8; ++k) tot += red[0][k];
+  const float inv = rsqrtf(tot / static_cast<float>(d) + eps);
+  float sx = 0.0f;
+  for (int j = threadIdx.x * 4; j < d; j += 1024) {
+    const float4 v = *reinterpret_cast<const float4*>(yr + j);
+    float4 a = *reinterpret_cast<const float4*>(xr + j);
+    a.x = fmaf(v.x * inv, ldw(g_post, w_bf16, j + 0), a.x);
+    a.y = fmaf(v.y * inv, ldw(g_post, w_bf16, j + 1), a.y);
+    a.z = fmaf(v.z * inv, ldw(g_post, w_bf16, j + 2), a.z);
+    a.w = fmaf(v.w * inv, ldw(g_post, w_bf16, j + 3), a.w);
+    *reinterpret_cast<float4*>(xr + j) = a;
+    sx += a.x * a.x + a.y * a.y + a.z * a.z + a.w * a.w;
+  }
+  if (!g_next) return;
+  sx = warp_sum(sx);
+  if (lane == 0) red[1][w] = sx;
+  __syncthreads();   // also orders this block's x writes before the reads below
+  float totx = 0.0f;
+#pragma unroll
+  for (int k = 0; k < 8; ++k) totx += red[1][k];
+  const float inx = rsqrtf(totx / static_cast<float>(d) + eps);
+  for (int j = threadIdx.x * 4; j < d; j += 1024) {
+    const float4 a = *reinterpret_cast<const float4*>(xr + j);
+    const size_t o = static_cast<size_t>(m) * d + j;
+    store_act<T>(out, o + 0, a.x * inx * ldw(g_next, w_bf16, j + 0));
+    store_act<T>(out, o + 1, a.y * inx * ldw(g_next, w_bf16, j + 1));
+    store_act<T>(out, o + 2, a.z * inx * ldw(g_next, w_bf16, j + 2));
+    store_act<T>(out, o + 3, a.w * inx * ldw(g_next, w_bf16, j + 3));
+  }
+}
+
 __global__ void rms_scale_kernel(const float* __restrict__ x, int M, int d, float eps, float* __restrict__ s) {
   pdl_enter();
   const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
@@ -446,6 +499,13 @@ const char* post_norm_add(float* x, const float* y, int M, int d, const void* g_
                           float eps, void* out, int act_bf16, cudaStream_t s) {
   if (M <= 0) return nullptr;
   if (d % 4) return "post-norm rows need d % 4 == 0";
+  if (M < 1024) {   // few rows: a block per row keeps enough SMs busy
+    if (act_bf16)
+      launch_pdl(post_norm_add_block_kernel<bf16>, M, 256, 0, s, x, y, d, g_post, g_next, w_bf16, eps, out);
+    else
+      launch_pdl(post_norm_add_block_kernel<float>, M, 256, 0, s, x, y, d, g_post, g_next, w_bf16, eps, out);
+    return err();
+  }
   if (act_bf16)
     launch_pdl(post_norm_add_kernel<bf16>, rows_grid(M), WPB * 32, 0, s, x, y, M, d, g_post, g_next, w_bf16, eps, out);
   else
