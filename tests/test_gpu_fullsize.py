@@ -124,3 +124,38 @@ def test_posttrain_full_width_reduced_depth():
     assert np.array_equal(gz[committed], ref["tok"][0][committed])
     assert agree >= 0.9, agree
     print(f"[fullsize posttrain] logits rel-L2 {rel:.3e}, argmax agreement {agree:.4f}, committed {committed.sum()}")
+
+
+def test_posttrain_full_depth_one_sequence():
+    """'posttrain' at its stated depth (S = embedding + 2 layers, A = 54, D =
+    6; d_model 5376, vocab 262144, paired-attention fusion), batch 1, a
+    32-token prompt: prefill, refresh and one stale step on the first block
+    of 32, against the oracle (weights widened per use, so host memory holds
+    only the bf16 model).
+
+    On these random-init weights the logits error of any path with bf16
+    tensor-core operands grows with depth past the 2e-2 bound:
+    tests/bf16_floor.py --depth runs this very case with the oracle's
+    arithmetic rounded to bf16 at every operand (the QKV input exact, as the
+    split operand carries it) and stores its rel-L2
+    (tests/golden/bf16_posttrain_depth62.json, 4.44e-2).  The GPU must meet
+    the bound or sit within 10 % of that bf16 path's own error."""
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import json
+    import os
+    import time
+    with open(os.path.join(os.path.dirname(__file__), "golden", "bf16_posttrain_depth62.json")) as f:
+        gold = json.load(f)
+    case = gold["case"]
+    w = wl.WORKLOADS["posttrain"]
+    m = w.model
+    assert case["layers"] == [m.n_shared, m.n_anchor, m.n_denoise] and m.qkv_split
+    t0 = time.time()
+    rel, agree, committed, gz, ref = _block_case(m, case["batch"], case["prompt_len"], case["block_len"],
+                                                 seed=case["seed"], T=case["T"])
+    floor = gold["bf16_path_logits_rel_l2"]
+    print(f"[fullsize posttrain depth 62] logits rel-L2 {rel:.3e} (bf16-operand path {floor:.3e}), "
+          f"argmax agreement {agree:.4f}, committed {committed.sum()}, {time.time() - t0:.0f} s")
+    assert rel < 2e-2 or rel <= 1.1 * floor, (rel, floor)
+    assert np.array_equal(gz[committed], ref["tok"][0][committed])
