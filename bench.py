@@ -138,6 +138,44 @@ def replica_prompts(w, rank: int):
     return wl.make_prompts(w, seed=w.seed + 1000 * rank)
 
 
+# DRAM traffic of the GEMM launches of a small-workload generation, from the
+# ncu capture summarised in profiles/small_workload_gemm_traffic.md (mean
+# dram__bytes_read.sum + dram__bytes_write.sum per GEMM launch); valid only
+# while the GEMM sources are the ones captured (their hash is recorded there).
+TRAFFIC_PROFILE = os.path.join(ROOT, "profiles", "small_workload_gemm_traffic.md")
+GEMM_SOURCES = ("gemm_tc.cu", "epilogue.cuh", "common.cuh", "splitk.cu")
+
+
+def gemm_source_hash() -> str:
+    import hashlib
+    h = hashlib.sha256()
+    for f in GEMM_SOURCES:
+        with open(os.path.join(ROOT, "paper_2609_37924_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def gemm_traffic():
+    """(bytes per GEMM launch, note): the captured figure while the sources
+    match, else (None, why)."""
+    try:
+        text = open(TRAFFIC_PROFILE).read()
+    except OSError:
+        return None, "no capture"
+    vals = {}
+    for line in text.splitlines():
+        if line.startswith("    ") or ":" not in line:
+            continue
+        k, _, v = line.partition(":")
+        vals[k.strip("`* -")] = v.strip(" `")
+    if vals.get("gemm_source_sha16") != gemm_source_hash():
+        return None, "GEMM sources changed since the capture"
+    try:
+        return float(vals["dram_bytes_per_gemm_launch"]), TRAFFIC_PROFILE[len(ROOT) + 1:]
+    except (KeyError, ValueError):
+        return None, "capture unreadable"
+
+
 def load_peaks():
     try:
         return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
@@ -386,9 +424,12 @@ def gpu_arm(args):
         peak, peak_src = peaks["bf16_tflops_sustained"], "measured sustained bf16 (MEASURED_PEAKS.json)"
     else:
         peak, peak_src = 1700.0, "fallback sustained bf16"
-    roofline = {"bound": "tensor", "kernel": "gemm_tc_kernel (tcgen05, all GEMM launches)",
+    traffic, traffic_src = gemm_traffic()
+    alg_bytes = sum(v["bytes"] for k, v in gemm_kinds.items() if k not in ("attention", "norms", "attention_short_rows"))
+    roofline = {"bound": "tensor", "kernel": "gemm_tc kernels (tcgen05, all GEMM launches of the step)",
                 "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                "frac": (achieved / peak) if achieved else None, "traffic": None, "peak_source": peak_src,
+                "frac": (achieved / peak) if achieved else None, "traffic": traffic, "traffic_source": traffic_src,
+                "algorithmic_bytes_per_launch": alg_bytes / n_launch if n_launch else None, "peak_source": peak_src,
                 "launches_timed": n_launch, "gemm_ms_per_step": gemm_ms,
                 "gemm_share_of_step": gemm_ms / (ms / args.steps) if ms else None,
                 "probe": "one extra generation with events around every GEMM / attention / norm launch",
