@@ -394,10 +394,11 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD, TKV>::MIN_BLOCKS)
   }
 }
 
-// ------------------------------------------------------ pipelined variant, hd 64
-// The same computation for hd 64 without key splits or a window, with the
-// tensor pipe and the softmax overlapped: 64-key tiles, S double-buffered in
-// TMEM (S0, S1, then O: 192 of the 256 columns, two CTAs per SM) and P
+// ------------------------------------------------------------ pipelined variant
+// The same computation without key splits or a window, with the tensor pipe
+// and the softmax overlapped: 64-key tiles, S double-buffered in TMEM (S0,
+// S1, then O: 2 * 64 + hd of the 256 columns; two CTAs per SM for hd 64, one
+// for hd 128, whose four stages of 32 KB fill the shared memory) and P
 // double-buffered in shared memory, four K / V stages.  The MMA thread
 // issues S(i) as soon as the softmax has released its S buffer (tile i - 2),
 // then O += P(i-1) V(i-1): while the softmax threads exponentiate tile i,
@@ -406,21 +407,25 @@ __global__ void __launch_bounds__(192, AttnTcCfg<HD, TKV>::MIN_BLOCKS)
 // issued before S(i), so when S(i) is complete the P buffer of tile i and
 // the O accumulator up to tile i-2 are settled; a rescale of O at tile i
 // waits for P V(i-1) on o_full.
+template <int HD_>
 struct AttnDbCfg {
-  static constexpr int HD = 64, TKV = 64, STAGES = 4;
-  static constexpr int Q_BYTES = 16384;               // 128 rows x 64 dims, one swizzle atom
-  static constexpr int K_BYTES = TKV * 128;           // 64 keys x 64 dims
-  static constexpr int V_BYTES = HD * 128;            // 64 dims x 64 keys (V^T)
+  static constexpr int HD = HD_, TKV = 64, STAGES = 4;
+  static constexpr int MIN_BLOCKS = HD == 64 ? 2 : 1;
+  static constexpr int Q_BYTES = HD / 64 * 16384;     // HD/64 swizzle atoms of 128 rows x 64 dims
+  static constexpr int K_BYTES = HD / 64 * TKV * 128; // HD/64 atoms of 64 keys x 64 dims
+  static constexpr int V_BYTES = HD * 128;            // HD dims x 64 keys (V^T)
   static constexpr int P_BYTES = 16384;               // 128 rows x 64 keys
   static constexpr int SMEM = Q_BYTES + STAGES * (K_BYTES + V_BYTES) + 2 * P_BYTES + 256;
-  static constexpr int TMEM_COLS = 256;               // S0 [0, 64), S1 [64, 128), O [128, 192)
+  static constexpr int TMEM_COLS = 256;               // S0 [0, 64), S1 [64, 128), O [128, 128 + HD)
+  static_assert(2 * TKV + HD <= TMEM_COLS, "TMEM columns");
 };
 
-__global__ void __launch_bounds__(192, 2)
+template <int HD_>
+__global__ void __launch_bounds__(192, AttnDbCfg<HD_>::MIN_BLOCKS)
     attn_db_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
                    const AttnTcArgs args) {
   pdl_enter();
-  using C = AttnDbCfg;
+  using C = AttnDbCfg<HD_>;
   constexpr int HD = C::HD, TKV = C::TKV, NST = C::STAGES;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = smem_raw;
@@ -493,11 +498,12 @@ __global__ void __launch_bounds__(192, 2)
         const int st = i % NST;
         if (!mbar_wait_bounded(&kv_empty[st], ((i / NST) & 1) ^ 1, abort_flag, args.status)) break;
         mbar_arrive_expect_tx(&kv_full[st], C::K_BYTES + C::V_BYTES);
-        tma_load_3d(sK + st * C::K_BYTES, &tmK, &kv_full[st], 0, i * TKV, z);
+        for (int s = 0; s < HD / 64; ++s)
+          tma_load_3d(sK + st * C::K_BYTES + s * (TKV * 128), &tmK, &kv_full[st], 64 * s, i * TKV, z);
         tma_load_3d(sV + st * C::V_BYTES, &tmV, &kv_full[st], i * TKV, 0, z);
         ++issued[st];
         if (i + NST < n_tiles) {     // the stage ring holds tiles i .. i+3; L2 fetches tile i+4 meanwhile
-          tma_prefetch_3d(&tmK, 0, (i + NST) * TKV, z);
+          for (int s = 0; s < HD / 64; ++s) tma_prefetch_3d(&tmK, 64 * s, (i + NST) * TKV, z);
           tma_prefetch_3d(&tmV, (i + NST) * TKV, 0, z);
         }
       }
@@ -523,8 +529,8 @@ __global__ void __launch_bounds__(192, 2)
           const uint32_t k0 = smem_u32(sK + st * C::K_BYTES);
 #pragma unroll
           for (int kk = 0; kk < HD / 16; ++kk)
-            umma_bf16(tmem + sb * TKV, sdesc_kmajor_sw128(q0 + kk * 32), sdesc_kmajor_sw128(k0 + kk * 32), idesc_s,
-                      kk != 0);
+            umma_bf16(tmem + sb * TKV, sdesc_kmajor_sw128(q0 + (kk >> 2) * 16384 + (kk & 3) * 32),
+                      sdesc_kmajor_sw128(k0 + (kk >> 2) * (TKV * 128) + (kk & 3) * 32), idesc_s, kk != 0);
           umma_commit(&s_full[sb]);
         }
         if (i >= 1) {
@@ -562,11 +568,14 @@ __global__ void __launch_bounds__(192, 2)
     {
       const uint4* src = reinterpret_cast<const uint4*>(
           args.q + ((static_cast<size_t>(b) * args.n_heads + qh) * args.rows + qr) * HD);
-      uint8_t* dst = sQ + row * 128;
 #pragma unroll
-      for (int c = 0; c < 8; ++c) {
-        const uint4 val = v_ok ? src[c] : make_uint4(0, 0, 0, 0);
-        *reinterpret_cast<uint4*>(dst + ((c ^ (row & 7)) << 4)) = val;
+      for (int s = 0; s < HD / 64; ++s) {
+        uint8_t* dst = sQ + s * 16384 + row * 128;
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          const uint4 val = v_ok ? src[s * 8 + c] : make_uint4(0, 0, 0, 0);
+          *reinterpret_cast<uint4*>(dst + ((c ^ (row & 7)) << 4)) = val;
+        }
       }
       fence_proxy_async_smem();
       mbar_arrive(q_full);
@@ -834,8 +843,9 @@ bool attn_db_enabled() {
   return on;
 }
 
+template <int HD>
 const char* launch_db(const AttnCall& a, cudaStream_t s) {
-  using C = AttnDbCfg;
+  using C = AttnDbCfg<HD>;
   if (!encoder()) return "cuTensorMapEncodeTiled is unavailable";
   const int kv_len = a.ctx + a.rows;
   CUtensorMap mk, mv;
@@ -846,7 +856,7 @@ const char* launch_db(const AttnCall& a, cudaStream_t s) {
     return "attention tensor map encode failed";
   static bool attr = false;
   if (!attr) {
-    if (cudaFuncSetAttribute(attn_db_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM) != cudaSuccess)
+    if (cudaFuncSetAttribute(attn_db_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM) != cudaSuccess)
       return "attention smem attribute failed";
     attr = true;
   }
@@ -855,7 +865,7 @@ const char* launch_db(const AttnCall& a, cudaStream_t s) {
   AttnTcArgs args{static_cast<const bf16*>(a.q), a.rows, a.ctx, kv_len, a.n_heads, a.n_kv_heads, a.causal, 0,
                   1.4426950408889634f / sqrtf(static_cast<float>(C::HD)), static_cast<bf16*>(a.o),
                   n_vtiles, 1, 0, nullptr, nullptr, a.status};
-  launch_pdl(attn_db_kernel, dim3(n_vtiles, a.n_kv_heads, a.batch), 192, C::SMEM, s, mk, mv, args);
+  launch_pdl(attn_db_kernel<HD>, dim3(n_vtiles, a.n_kv_heads, a.batch), 192, C::SMEM, s, mk, mv, args);
   const cudaError_t e = cudaGetLastError();
   return e == cudaSuccess ? nullptr : cudaGetErrorString(e);
 }
@@ -1166,11 +1176,19 @@ const char* attention(const AttnCall& a, cudaStream_t s) {
       cudaDeviceGetAttribute(&n_sms, cudaDevAttrMultiProcessorCount, dev);
       const int ctas = ((a.n_heads / a.n_kv_heads) * a.rows + TQ - 1) / TQ * a.n_kv_heads * a.batch;
       const bool window_cuts = a.window > 0 && a.window < a.ctx + a.rows;
-      if (attn_db_enabled() && !window_cuts && ctas > n_sms) return launch_db(a, s);
+      if (attn_db_enabled() && !window_cuts && ctas > n_sms) return launch_db<64>(a, s);
       return launch_tc<64, 128>(a, s);
     }
     if (a.head_dim == 128) {
       if (!tc) return launch_bf16<128>(a, s) == cudaSuccess ? nullptr : "attention launch failed";
+      // one CTA per SM: the pipelined kernel when the launch fills 80-100 % of the SMs in one wave (larger
+      // launches run attn_tc_kernel two CTAs per SM, smaller ones split the keys)
+      int dev = 0, n_sms = 0;
+      cudaGetDevice(&dev);
+      cudaDeviceGetAttribute(&n_sms, cudaDevAttrMultiProcessorCount, dev);
+      const int ctas = ((a.n_heads / a.n_kv_heads) * a.rows + TQ - 1) / TQ * a.n_kv_heads * a.batch;
+      const bool window_cuts = a.window > 0 && a.window < a.ctx + a.rows;
+      if (attn_db_enabled() && !window_cuts && 5 * ctas >= 4 * n_sms && ctas <= n_sms) return launch_db<128>(a, s);
       return (a.n_heads / a.n_kv_heads) * a.rows < 2 * TQ ? launch_tc<128, 64>(a, s) : launch_tc<128, 128>(a, s);
     }
     return "bf16 attention supports head_dim 64 and 128";

@@ -199,3 +199,29 @@ def test_attention_short_rows_tcgen05_as_accurate_as_mma_sync(T, hd, Hq, Hkv, ro
     print(f"[short-row attention hd {hd}] rel-L2 tcgen05 {errs[0]:.2e}  mma.sync {errs[1]:.2e}")
     assert errs[0] < 1e-2 and errs[1] < 1e-2
     assert errs[0] <= 1.5 * errs[1], errs
+
+
+@pytest.mark.parametrize("B,Hq,Hkv,rows,ctx,causal", [
+    (16, 16, 8, 32, 777, False),     # block-diffusion steps: 32 rows x a GQA group over a long context
+    (8, 32, 16, 32, 1100, False),    # post-train widths
+    (2, 16, 8, 500, 100, True),      # a causal commit / prefill pass over a context
+    (1, 64, 64, 300, 0, False)])     # ragged rows, many heads
+def test_attention_pipelined_hd128(T, B, Hq, Hkv, rows, ctx, causal):
+    """hd 128 launches that fill 80-100 % of the SMs in one wave run the
+    pipelined kernel (one CTA per SM, double-buffered S and P, four 32 KB K /
+    V stages); the others attn_tc_kernel."""
+    hd = 128
+    L = ctx + rows
+    stride = L + (-L) % 8
+    q, qd = bf16_tensor((B, Hq, rows, hd), 25)
+    k, kd = bf16_tensor((B, Hkv, stride, hd), 26)
+    vt, vtd = bf16_tensor((B, Hkv, hd, stride), 27)
+    o = torch.empty((B * rows, Hq * hd), dtype=torch.bfloat16, device="cuda")
+    T.tadm_attention(q, k, vt, o, Hq, Hkv, rows, ctx, causal, dtype=1)
+    torch.cuda.synchronize()
+    got = o.float().cpu().numpy().astype(np.float64).reshape(B, rows, Hq, hd)
+    for b in sorted({0, B - 1}):
+        ref = O.attention(qd[b], kd[b, :, :L], vtd[b, :, :, :L].transpose(0, 2, 1), ctx + np.arange(rows),
+                          np.arange(L), causal).transpose(1, 0, 2)
+        rel = np.linalg.norm(got[b] - ref) / np.linalg.norm(ref)
+        assert rel < 1e-2, (b, rel)
