@@ -659,7 +659,10 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
   const bool narrow_kind = g.epi == EPI_RESID || g.epi == EPI_FUSION2 || (g.epi == EPI_QKV && 128 % g.ep.head_dim == 0);
   const bool narrow = pair_ok && narrow_kind && m_pairs * a.n_tiles_n * 4 <= g_num_sms;
   const int pair_units = narrow ? m_pairs * ((g.N + 127) / 128) : m_pairs * a.n_tiles_n;
-  const bool pairs_fill = pair_ok && 2 * pair_units * 5 >= g_num_sms * 2;
+  // pairs must keep >= 40% of the SMs busy to beat split-K; for the residual-add and fp32-store epilogues,
+  // whose split-K reduction is one element-wise launch, >= 60% (the weight-streaming block steps)
+  const bool elem_reduce = g.epi == EPI_RESID || (g.epi == EPI_STORE && !g.ep.out_bf16);
+  const bool pairs_fill = pair_ok && 2 * pair_units * (elem_reduce ? 10 : 5) >= g_num_sms * (elem_reduce ? 6 : 2);
   if (g.split_buf && !g.m_dev && !pairs_fill && tiles * 3 < g_num_sms * 2 && kblocks >= 8) {
     int sp = std::min(std::min(g_num_sms / tiles, kblocks / 4), 16);
     const size_t per = static_cast<size_t>(g.M) * a.ldp * sizeof(float);

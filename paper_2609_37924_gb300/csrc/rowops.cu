@@ -355,15 +355,39 @@ __global__ void rms_scale_kernel(const float* __restrict__ x, int M, int d, floa
   if (lane == 0) s[m] = sqrtf(ss / static_cast<float>(d) + eps);
 }
 
+// out = x / s[row], element-wise over four columns per thread (d % 4 == 0)
 template <class T>
 __global__ void scale_rows_kernel(const float* __restrict__ x, const float* __restrict__ sc, int M, int d,
                                   void* __restrict__ out) {
   pdl_enter();
-  const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
-  if (m >= M) return;
-  const float s = sc[m];
-  for (int j = lane; j < d; j += 32)
-    store_act<T>(out, static_cast<size_t>(m) * d + j, x[static_cast<size_t>(m) * d + j] / s);
+  const size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x;
+  if (i >= static_cast<size_t>(M) * (d / 4)) return;
+  const size_t e = i * 4;
+  const float s = sc[e / d];
+  const float4 v = *reinterpret_cast<const float4*>(x + e);
+  store_act<T>(out, e + 0, v.x / s);
+  store_act<T>(out, e + 1, v.y / s);
+  store_act<T>(out, e + 2, v.z / s);
+  store_act<T>(out, e + 3, v.w / s);
+}
+
+// s[row] = sqrt(mean(x^2) + eps), one 256-thread block per row (few rows)
+__global__ void __launch_bounds__(256) rms_scale_block_kernel(const float* __restrict__ x, int d, float eps,
+                                                              float* __restrict__ s) {
+  pdl_enter();
+  __shared__ float red[8];
+  const int m = blockIdx.x;
+  const float* xr = x + static_cast<size_t>(m) * d;
+  float ss = 0.0f;
+  for (int j = threadIdx.x; j < d; j += 256) ss += xr[j] * xr[j];
+  ss = warp_sum(ss);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float tot = 0.0f;
+    for (int w = 0; w < 8; ++w) tot += red[w];
+    s[m] = sqrtf(tot / static_cast<float>(d) + eps);
+  }
 }
 
 struct Parts {
@@ -372,17 +396,16 @@ struct Parts {
   int n;
 };
 
+// out[m] = [parts[0][m], parts[1][m], ...], one output element per thread
 template <class T>
 __global__ void concat_kernel(Parts parts, int M, int width, void* __restrict__ out) {
   pdl_enter();
-  const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
-  if (m >= M) return;
-  int col = 0;
-  for (int i = 0; i < parts.n; ++i) {
-    const float* src = parts.p[i] + static_cast<size_t>(m) * parts.w[i];
-    for (int j = lane; j < parts.w[i]; j += 32) store_act<T>(out, static_cast<size_t>(m) * width + col + j, src[j]);
-    col += parts.w[i];
-  }
+  const size_t i = blockIdx.x * static_cast<size_t>(blockDim.x) + threadIdx.x;
+  if (i >= static_cast<size_t>(M) * width) return;
+  const int m = static_cast<int>(i / width);
+  int col = static_cast<int>(i % width), k = 0;
+  while (col >= parts.w[k]) col -= parts.w[k++];
+  store_act<T>(out, i, parts.p[k][static_cast<size_t>(m) * parts.w[k] + col]);
 }
 
 __global__ void sub_kernel(const float* __restrict__ a, const float* __restrict__ b, size_t n, float* __restrict__ o) {
@@ -491,6 +514,10 @@ const char* layernorm_rows(const float* x, int M, int d, const void* w, const vo
 
 const char* rms_scale_rows(const float* x, int M, int d, float eps, float* s_out, cudaStream_t st) {
   if (M <= 0) return nullptr;
+  if (M < 1024) {   // few rows: a block per row keeps enough SMs busy
+    launch_pdl(rms_scale_block_kernel, M, 256, 0, st, x, d, eps, s_out);
+    return err();
+  }
   launch_pdl(rms_scale_kernel, rows_grid(M), WPB * 32, 0, st, x, M, d, eps, s_out);
   return err();
 }
@@ -516,10 +543,12 @@ const char* post_norm_add(float* x, const float* y, int M, int d, const void* g_
 
 const char* scale_rows(const float* x, const float* sc, int M, int d, void* out, int act_bf16, cudaStream_t s) {
   if (M <= 0) return nullptr;
+  if (d % 4) return "scale_rows needs d % 4 == 0";
+  const unsigned blocks = static_cast<unsigned>((static_cast<size_t>(M) * (d / 4) + 255) / 256);
   if (act_bf16)
-    launch_pdl(scale_rows_kernel<bf16>, rows_grid(M), WPB * 32, 0, s, x, sc, M, d, out);
+    launch_pdl(scale_rows_kernel<bf16>, blocks, 256, 0, s, x, sc, M, d, out);
   else
-    launch_pdl(scale_rows_kernel<float>, rows_grid(M), WPB * 32, 0, s, x, sc, M, d, out);
+    launch_pdl(scale_rows_kernel<float>, blocks, 256, 0, s, x, sc, M, d, out);
   return err();
 }
 
@@ -535,10 +564,11 @@ const char* concat_rows(const float* const* parts, const int* widths, int n_part
     width += widths[i];
   }
   p.n = n_parts;
+  const unsigned blocks = static_cast<unsigned>((static_cast<size_t>(M) * width + 255) / 256);
   if (act_bf16)
-    launch_pdl(concat_kernel<bf16>, rows_grid(M), WPB * 32, 0, s, p, M, width, out);
+    launch_pdl(concat_kernel<bf16>, blocks, 256, 0, s, p, M, width, out);
   else
-    launch_pdl(concat_kernel<float>, rows_grid(M), WPB * 32, 0, s, p, M, width, out);
+    launch_pdl(concat_kernel<float>, blocks, 256, 0, s, p, M, width, out);
   return err();
 }
 
