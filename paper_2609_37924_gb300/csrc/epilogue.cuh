@@ -222,10 +222,19 @@ __device__ __forceinline__ void epilogue_row(const EpiParams& p, int m, int n_bl
   // through its shared-memory box and one TMA reduce-add (resid += chunk at
   // L2), so the epilogue never waits on a load of the residual stream.  Each
   // element receives exactly one add per GEMM: the result is deterministic.
+  // The next chunk's TMEM load is issued before this chunk's box wait and
+  // reduce, so its latency overlaps them.
   if constexpr (Src::kStaged && EPI == EPI_RESID) {
     if (src.has_box() && p.resid_tma) {
+      uint32_t cur[32], nxt[32];
+      if (c_lo < c_hi) {
+        src.load_async(c_lo, cur);
+        src.wait_ld(cur);
+      }
       for (int c = c_lo; c < c_hi; ++c) {
-        src.load(c, v);
+        if (c + 1 < c_hi) src.load_async(c + 1, nxt);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(cur[i]);
         const int n0 = n_blk * ncols + 32 * c;
         if (p.bias) {
           const int lane = threadIdx.x & 31;
@@ -234,6 +243,11 @@ __device__ __forceinline__ void epilogue_row(const EpiParams& p, int m, int n_bl
           for (int i = 0; i < 32; ++i) v[i] += __shfl_sync(0xffffffffu, bl, i);
         }
         if (n0 < p.N && src.row0 < p.M) src.reduce32(n0, v);   // the map clips ragged rows / columns
+        if (c + 1 < c_hi) {
+          src.wait_ld(nxt);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) cur[i] = nxt[i];
+        }
       }
       return;
     }

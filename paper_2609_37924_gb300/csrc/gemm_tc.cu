@@ -65,6 +65,12 @@ struct TmemSrc {
     __syncwarp();  // tcgen05.ld is warp-collective: reconverge after divergent stores
     tmem_ld32(taddr + 32 * chunk, v);
   }
+  // the same load without waiting: r is usable after wait_ld(r)
+  __device__ __forceinline__ void load_async(int chunk, uint32_t (&r)[32]) {
+    __syncwarp();
+    tmem_ld32_nowait(taddr + 32 * chunk, r);
+  }
+  __device__ __forceinline__ void wait_ld(uint32_t (&r)[32]) { tmem_wait_ld(r); }
   // this lane's row of a 32 x 32 fp32 chunk into the box, then one TMA
   // reduce-add of the box into the fp32 output map at column x (resid += box)
   __device__ __forceinline__ void reduce32(int x, const float (&v)[32]) {
