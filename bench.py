@@ -3,15 +3,21 @@
 One step = one whole generation (Alg. 1 over every block) of the workload's
 batch, i.e. batch * gen_len generated tokens.  Default workload: "small"
 (batch 16, 256 Zipf prompt tokens + 768 masked, 128 reverse steps, K = 4,
-d_model 768, 8 anchor + 4 denoiser layers, vocab 32768, bf16).
+d_model 768, 8 anchor + 4 denoiser layers, vocab 32768, bf16).  At N = 1 the
+same line also carries "configs": the block-diffusion workload (batch 32,
+d_model 2048, 16 + 6 layers, blocks of 32) and the 27 B post-train workload
+(batch 8, d_model 5376, 2 + 54 + 6 layers, paired-attention fusion), each
+timed over whole generations at K = 1 and its own K, with its GEMMs'
+throughput against the tensor and HBM peaks.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload small] [--K 4]
     python bench.py --impl reference ...      # the CPU oracle on a bounded sample
 
-Under torchrun (N > 1) every rank runs an independent replica on its own
-GPU with its own prompts (sequences are independent: no collective on the
-data path); value = all ranks' tokens / max-over-ranks time.
-Prints one JSON line on rank 0.
+With --gpus N > 1 every rank runs an independent replica on its own GPU
+with its own prompts (sequences are independent: no collective on the data
+path); value = all ranks' tokens / max-over-ranks time.  Launched without
+torchrun, bench.py starts the N local ranks itself.  Prints one JSON line on
+rank 0.
 """
 from __future__ import annotations
 
