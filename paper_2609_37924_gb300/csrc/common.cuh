@@ -67,17 +67,35 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+// try_wait with a suspend-time hint: a thread whose phase is not complete is
+// parked (it issues nothing) until the phase completes or `hint_ns` passes,
+// so waiting roles leave the issue slots of their SM sub-partition to the
+// working warps instead of spinning on the barrier.
+__device__ __forceinline__ bool mbar_try_wait_suspend(uint64_t* bar, uint32_t parity, uint32_t hint_ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(hint_ns)
+      : "memory");
+  return ok != 0;
+}
+
 // Waits for the phase of `parity` to complete.  Gives up when *abort becomes
 // non-zero (another role gave up) or after `limit_ns`; on its own timeout it
 // raises *abort and the device status word.  Returns false when it gave up.
+// Each suspended try_wait lasts at most 1 ms, so an abort raised elsewhere is
+// seen within about a millisecond.
 __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, volatile int* abort,
                                                   int* status, uint64_t limit_ns = 4000000000ull) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = global_ns();
   for (uint32_t it = 1;; ++it) {
-    if (mbar_try_wait(bar, parity)) return true;
+    if (mbar_try_wait_suspend(bar, parity, 1000000u)) return true;
     if (*abort) return false;
-    if ((it & 255u) == 0 && global_ns() - t0 > limit_ns) {
+    if ((it & 15u) == 0 && global_ns() - t0 > limit_ns) {
       *abort = 1;
       if (status) atomicOr(status, kErrTimeout);
       return false;

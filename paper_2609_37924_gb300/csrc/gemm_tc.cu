@@ -11,8 +11,10 @@
 //               thread; two warps per lane quadrant, each taking half of the
 //               256 columns) and run the fused epilogue of epilogue.cuh, while
 //               the MMA warp fills the other accumulator.
-// GEMMs of more than 128 rows that need no split-K run the CTA-pair variant
-// (gemm_tc2_kernel: 256 x 256 tiles, tcgen05.mma.cta_group::2, six stages).
+// GEMMs of more than 128 rows run the CTA-pair variant (gemm_tc2_kernel:
+// 256 x 256 tiles, tcgen05.mma.cta_group::2, six stages), with split-K for
+// the weight-streaming residual / fp32-store GEMMs whose tiles cannot fill
+// the SMs; other GEMMs that need split-K run this kernel.
 // Every mbarrier wait is bounded (mbar_wait_bounded): a role that gives up
 // raises a shared abort flag and the device status word, and the CTA drains
 // its in-flight copies and MMAs, frees TMEM and exits.
@@ -391,7 +393,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
 
   const int m_run = args.m_dev ? min(args.M, *args.m_dev) : args.M;   // read after pdl_enter
   const int num_m2 = (m_run + 2 * BM - 1) / (2 * BM);
-  const int units = num_m2 * args.n_tiles_n;
+  const int units = num_m2 * args.n_tiles_n * args.splits;   // unit = (pair tile, K slice)
   const int u0 = static_cast<int>(blockIdx.x >> 1), ustep = static_cast<int>(gridDim.x >> 1);
   const int kblocks = (args.K + BK - 1) / BK;
 
@@ -402,12 +404,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       int stage = 0;
       uint32_t phase = 0;
       for (int unit = u0; unit < units && !*abort_flag; unit += ustep) {
-        const int nb = unit % args.n_tiles_n;
-        const int mb = 2 * (unit / args.n_tiles_n) + static_cast<int>(rank);   // this CTA's 128-row block
-        prefetch_epilogue_inputs<EPI>(args, mb, nb, PBN);
+        const int tile = unit / args.splits, ks = unit % args.splits;
+        const int nb = tile % args.n_tiles_n;
+        const int mb = 2 * (tile / args.n_tiles_n) + static_cast<int>(rank);   // this CTA's 128-row block
+        const int kb0 = ks * args.kb_per_split, kb1 = min(kblocks, kb0 + args.kb_per_split);
+        if (args.splits == 1) prefetch_epilogue_inputs<EPI>(args, mb, nb, PBN);
         const int brow = args.b_split > 0 ? (rank ? args.b_split : 0) + nb * (PBN / 2) : nb * PBN + rank * (PBN / 2);
         bool ok = true;
-        for (int kb = 0; kb < kblocks; ++kb) {
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait_bounded(&empty[stage], phase ^ 1, abort_flag, args.status)) { ok = false; break; }
           if (leader) mbar_arrive_expect_tx(&full[stage], 2 * P_STAGE_BYTES);
           const uint32_t fb = full_l0 + 8u * stage;
@@ -436,11 +440,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
       int acc = 0;
       uint32_t acc_phase = 0;
       for (int unit = u0; unit < units && !*abort_flag; unit += ustep) {
+        const int ks = unit % args.splits;
+        const int kb0 = ks * args.kb_per_split, kb1 = min(kblocks, kb0 + args.kb_per_split);
         if (!mbar_wait_bounded(&tempty[acc], acc_phase ^ 1, abort_flag, args.status)) break;
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + acc * PBN;
         bool ok = true;
-        for (int kb = 0; kb < kblocks; ++kb) {
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!mbar_wait_bounded(&full[stage], phase, abort_flag, args.status)) { ok = false; break; }
           tc_fence_after();
           const uint32_t a0 = smem_u32(sA + stage * P_A_BYTES);
@@ -448,7 +454,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k) {
             umma_bf16_pair(d_tmem, sdesc_kmajor_sw128(a0 + 32 * k), sdesc_kmajor_sw128(b0 + 32 * k), idesc,
-                           (kb != 0) || (k != 0));
+                           (kb != kb0) || (k != 0));
           }
           umma_commit_pair_mc(&empty[stage], 0x3);
           if (++stage == P_STAGES) { stage = 0; phase ^= 1; }
@@ -473,13 +479,25 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(NUM_THREADS, 1)
     for (int unit = u0; unit < units; unit += ustep) {
       if (!warp_wait_bounded(&tfull[acc], acc_phase, abort_flag, args.status)) break;
       tc_fence_after();
-      const int nb = unit % args.n_tiles_n;
-      const int mb = 2 * (unit / args.n_tiles_n) + static_cast<int>(rank);
+      const int tile = unit / args.splits, ks = unit % args.splits;
+      const int nb = tile % args.n_tiles_n;
+      const int mb = 2 * (tile / args.n_tiles_n) + static_cast<int>(rank);
       TmemSrc src{tmem_base + static_cast<uint32_t>(acc * PBN) + (static_cast<uint32_t>(quad * 32) << 16),
                   args.staged ? sOut + (warp - 2) * STAGE_OUT_BYTES : nullptr, {&tmC, &tmC2}, mb * BM + quad * 32};
       const int m = mb * BM + quad * 32 + lane;
-      if (part < nsplit && mb * BM < args.M)   // the odd CTA's rows may lie past M
+      if (args.splits > 1) {
+        // raw fp32 partial of this K slice: this CTA's 128 rows of the pair tile, columns in natural order
+        if (mb * BM < args.M) {
+          float v[32];
+          float* dst = args.part + ks * args.part_stride + static_cast<size_t>(m) * args.ldp + nb * PBN;
+          for (int c = part * (PBN / 64); c < (part + 1) * (PBN / 64); ++c) {
+            src.load(c, v);
+            if (m < args.M) store32(dst, 0, 32 * c, v, 32);
+          }
+        }
+      } else if (part < nsplit && mb * BM < args.M) {   // the odd CTA's rows may lie past M
         epilogue_row<EPI>(args.ep, m, nb, PBN, src, part, nsplit);
+      }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive_remote(tempty_l0 + 8u * acc);
@@ -669,6 +687,37 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
   // whose split-K reduction is one element-wise launch, >= 60% (the weight-streaming block steps)
   const bool elem_reduce = g.epi == EPI_RESID || (g.epi == EPI_STORE && !g.ep.out_bf16);
   const bool pairs_fill = pair_ok && 2 * pair_units * (elem_reduce ? 10 : 5) >= g_num_sms * (elem_reduce ? 6 : 2);
+  // The residual-add / fp32-store GEMMs whose 256 x 256 pair tiles fill under
+  // 60 % of the SMs take those tiles with split-K: each weight tile crosses
+  // L2 once (128 x 256 tiles fetch it once per 128-row block) and an SM
+  // receives 32 KB per k-block (256 x 128 pair tiles: 24 KB for half the MMA
+  // work; 128 x 256 tiles: 48 KB for the same work).
+  const bool wide_fill = 2 * m_pairs * a.n_tiles_n * 10 >= g_num_sms * 6;
+  if (pair_ok && elem_reduce && !wide_fill && g.split_buf && !g.m_dev && kblocks >= 8) {
+    const int pu = m_pairs * a.n_tiles_n;
+    int sp = std::min(std::min((g_num_sms / 2) / pu, kblocks / 4), 16);
+    const size_t per = static_cast<size_t>(g.M) * a.ldp * sizeof(float);
+    while (sp > 1 && sp * per > g.split_bytes) --sp;
+    if (sp > 1) {
+      CUtensorMap tbh;
+      if (!make_map(&tbh, g.B, b_rows, k_b, g.ldb, BN / 2)) return "tensor map (B, half tiles) encode failed";
+      TcArgs a2 = a;
+      a2.kb_per_split = (kblocks + sp - 1) / sp;
+      a2.splits = (kblocks + a2.kb_per_split - 1) / a2.kb_per_split;
+      a2.part = g.split_buf;
+      a2.part_stride = static_cast<size_t>(g.M) * a2.ldp;
+      a2.staged = 0;
+      const cudaError_t e = g.epi == EPI_RESID ? launch_epi_pair<EPI_RESID>(ta, tbh, tc, tc2, a2, pu * a2.splits, s)
+                                               : launch_epi_pair<EPI_STORE>(ta, tbh, tc, tc2, a2, pu * a2.splits, s);
+      if (e != cudaSuccess) return cudaGetErrorString(e);
+      const_cast<GemmCall&>(g).launched = 1;
+      int nr = 0;
+      const char* r = splitk_reduce(g.epi, a2.ep, a2.part, a2.part_stride, a2.ldp, a2.splits, a2.n_tiles_n, s, &nr);
+      if (r) return r;
+      const_cast<GemmCall&>(g).launched = 1 + nr;
+      return nullptr;
+    }
+  }
   if (g.split_buf && !g.m_dev && !pairs_fill && tiles * 3 < g_num_sms * 2 && kblocks >= 8) {
     int sp = std::min(std::min(g_num_sms / tiles, kblocks / 4), 16);
     const size_t per = static_cast<size_t>(g.M) * a.ldp * sizeof(float);
@@ -737,9 +786,10 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
   if (e != cudaSuccess) return cudaGetErrorString(e);
   const_cast<GemmCall&>(g).launched = 1;
   if (a.splits > 1) {
-    const char* r = splitk_reduce(g.epi, a.ep, a.part, a.part_stride, a.ldp, a.splits, a.n_tiles_n, s);
+    int nr = 0;
+    const char* r = splitk_reduce(g.epi, a.ep, a.part, a.part_stride, a.ldp, a.splits, a.n_tiles_n, s, &nr);
     if (r) return r;
-    const_cast<GemmCall&>(g).launched = 3;
+    const_cast<GemmCall&>(g).launched = 1 + nr;
   }
   return nullptr;
 }

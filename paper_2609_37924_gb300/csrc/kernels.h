@@ -48,9 +48,9 @@ size_t gemm_tc_split_bytes();
 // tcgen05 path (bf16 operands)
 const char* gemm_tc(const GemmCall& g, cudaStream_t s);
 int gemm_tc_tiles_n(int N, int epi);
-// fixed-order sum of split-K partials followed by the GEMM's epilogue
+// fixed-order sum of split-K partials followed by the GEMM's epilogue; *launches = kernels it launched
 const char* splitk_reduce(int epi, const EpiParams& ep, const float* part, size_t part_stride, int ldp, int splits,
-                          int n_tiles_n, cudaStream_t s);
+                          int n_tiles_n, cudaStream_t s, int* launches);
 // CUDA-core path (fp32 operands)
 const char* gemm_simt(const GemmCall& g, cudaStream_t s);
 int gemm_simt_tiles_n(int N, int epi);

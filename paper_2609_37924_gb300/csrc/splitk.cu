@@ -119,15 +119,17 @@ bool elem_ok(int epi, const EpiParams& ep, int ldp) {
 // Phase 2: the epilogue on slice 0.
 template <int EPI>
 cudaError_t launch(const EpiParams& ep, const float* part, size_t stride, int ldp, int splits, int n_tiles_n,
-                   cudaStream_t s) {
+                   cudaStream_t s, int* launches) {
   if constexpr (EPI == EPI_RESID || EPI == EPI_STORE) {
     if (elem_ok(EPI, ep, ldp)) {
+      *launches = 1;
       const size_t n = static_cast<size_t>(ep.M) * (ep.N / 4);
       launch_pdl(splitk_elem_kernel<EPI>, static_cast<unsigned>((n + 255) / 256), 256, 0, s, ep, part, stride, ldp,
                  splits);
       return cudaGetLastError();
     }
   }
+  *launches = 2;
   const size_t n4 = static_cast<size_t>(ep.M) * ldp / 4;
   launch_pdl(splitk_sum_kernel, static_cast<unsigned>((n4 + 255) / 256), 256, 0, s, const_cast<float*>(part), stride, n4,
                                                                             splits);
@@ -138,20 +140,20 @@ cudaError_t launch(const EpiParams& ep, const float* part, size_t stride, int ld
 }  // namespace
 
 const char* splitk_reduce(int epi, const EpiParams& ep, const float* part, size_t stride, int ldp, int splits,
-                          int n_tiles_n, cudaStream_t s) {
+                          int n_tiles_n, cudaStream_t s, int* launches) {
   cudaError_t e;
   switch (epi) {
-    case EPI_STORE: e = launch<EPI_STORE>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
-    case EPI_RESID: e = launch<EPI_RESID>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
-    case EPI_QKV: e = launch<EPI_QKV>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
-    case EPI_GLU: e = launch<EPI_GLU>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
-    case EPI_FUSION1: e = launch<EPI_FUSION1>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
-    case EPI_FUSION2: e = launch<EPI_FUSION2>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
-    case EPI_LMHEAD: e = launch<EPI_LMHEAD>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
-    case EPI_PA_UP: e = launch<EPI_PA_UP>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
-    case EPI_SILU: e = launch<EPI_SILU>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
-    case EPI_ADD: e = launch<EPI_ADD>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
-    case EPI_PA_GATE: e = launch<EPI_PA_GATE>(ep, part, stride, ldp, splits, n_tiles_n, s); break;
+    case EPI_STORE: e = launch<EPI_STORE>(ep, part, stride, ldp, splits, n_tiles_n, s, launches); break;
+    case EPI_RESID: e = launch<EPI_RESID>(ep, part, stride, ldp, splits, n_tiles_n, s, launches); break;
+    case EPI_QKV: e = launch<EPI_QKV>(ep, part, stride, ldp, splits, n_tiles_n, s, launches); break;
+    case EPI_GLU: e = launch<EPI_GLU>(ep, part, stride, ldp, splits, n_tiles_n, s, launches); break;
+    case EPI_FUSION1: e = launch<EPI_FUSION1>(ep, part, stride, ldp, splits, n_tiles_n, s, launches); break;
+    case EPI_FUSION2: e = launch<EPI_FUSION2>(ep, part, stride, ldp, splits, n_tiles_n, s, launches); break;
+    case EPI_LMHEAD: e = launch<EPI_LMHEAD>(ep, part, stride, ldp, splits, n_tiles_n, s, launches); break;
+    case EPI_PA_UP: e = launch<EPI_PA_UP>(ep, part, stride, ldp, splits, n_tiles_n, s, launches); break;
+    case EPI_SILU: e = launch<EPI_SILU>(ep, part, stride, ldp, splits, n_tiles_n, s, launches); break;
+    case EPI_ADD: e = launch<EPI_ADD>(ep, part, stride, ldp, splits, n_tiles_n, s, launches); break;
+    case EPI_PA_GATE: e = launch<EPI_PA_GATE>(ep, part, stride, ldp, splits, n_tiles_n, s, launches); break;
     default: return "unknown epilogue";
   }
   return e == cudaSuccess ? nullptr : cudaGetErrorString(e);

@@ -324,10 +324,13 @@ def test_tiny_workload_full_generation_matches_oracle(T):
         assert agree >= 0.99, (K, agree)
 
 
-def test_block_mode_with_kv_context(T):
-    m = wl.ModelConfig(vocab=2048, d_model=256, n_heads=4, n_kv_heads=2, head_dim=128, ffn=512, n_anchor=2,
+# batch 8 x 32-row blocks at d_model 512: the 256-row residual projections (and the 320-row prefill, two pair
+# tiles of which the second is ragged) run CTA-pair tiles with split-K and the element-wise ordered reduction
+@pytest.mark.parametrize("B,d,ffn", [(2, 256, 512), (8, 512, 2048)])
+def test_block_mode_with_kv_context(T, B, d, ffn):
+    m = wl.ModelConfig(vocab=2048, d_model=d, n_heads=4, n_kv_heads=2, head_dim=128, ffn=ffn, n_anchor=2,
                        n_denoise=2, dtype="bf16")
-    B, P, bl = 2, 40, 32
+    P, bl = 40, 32
     w = wl.Workload("t", m, batch=B, prompt_len=P, gen_len=64, steps_per_block=4, K=2, block_len=bl)
     tm, o = setup(T, m, B, max(P, bl), max_ctx=P + 64)
     prompts = wl.make_prompts(w, batch=B, seed=9)
