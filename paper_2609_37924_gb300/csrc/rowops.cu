@@ -5,6 +5,7 @@
 // concatenations of the paired-attention fusion (App. C.1), the RoPE table,
 // and canvas set-up.
 #include <cstdlib>
+#include <initializer_list>
 
 #include "kernels.h"
 
@@ -234,6 +235,128 @@ __global__ void ln_pair_kernel(const float* __restrict__ c, const float* __restr
     for (int j = lane; j < d; j += 32)
       store_act<T>(u, static_cast<size_t>(m) * 2 * d + part * d + j,
                    (xr[j] - mean) * rstd * ldw(w, w_bf16, j) + ldw(b, w_bf16, j));
+  }
+}
+
+// Register-resident LayerNorm of one row of d = 256 NCH columns (one warp per
+// row): the lane holds the 8 consecutive values of each 256-column chunk, so
+// the row is read once; mean, then the variance about it, from registers.
+template <int NCH>
+__device__ __forceinline__ void ln_row_reg(const float* __restrict__ xr, int lane, float eps, float (&v)[NCH][8],
+                                           float& mean, float& rstd) {
+  constexpr int d = 256 * NCH;
+  float s = 0.0f;
+#pragma unroll
+  for (int c = 0; c < NCH; ++c) {
+    const int j = (c * 32 + lane) * 8;
+    const float4 a = *reinterpret_cast<const float4*>(xr + j);
+    const float4 b = *reinterpret_cast<const float4*>(xr + j + 4);
+    v[c][0] = a.x; v[c][1] = a.y; v[c][2] = a.z; v[c][3] = a.w;
+    v[c][4] = b.x; v[c][5] = b.y; v[c][6] = b.z; v[c][7] = b.w;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) s += v[c][i];
+  }
+  mean = warp_sum(s) / static_cast<float>(d);
+  float q = 0.0f;
+#pragma unroll
+  for (int c = 0; c < NCH; ++c)
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float a = v[c][i] - mean;
+      q = fmaf(a, a, q);
+    }
+  rstd = rsqrtf(warp_sum(q) / static_cast<float>(d) + eps);
+}
+
+// 8 consecutive parameters at element j (bf16 or fp32; 16-byte aligned)
+__device__ __forceinline__ void ldw8(const void* w, int bf, int j, float (&o)[8]) {
+  if (bf) {
+    const uint4 raw = *reinterpret_cast<const uint4*>(static_cast<const bf16*>(w) + j);
+    const __nv_bfloat162* p2 = reinterpret_cast<const __nv_bfloat162*>(&raw);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float2 f = __bfloat1622float2(p2[q]);
+      o[2 * q] = f.x;
+      o[2 * q + 1] = f.y;
+    }
+  } else {
+    const float4 a = *reinterpret_cast<const float4*>(static_cast<const float*>(w) + j);
+    const float4 b = *reinterpret_cast<const float4*>(static_cast<const float*>(w) + j + 4);
+    o[0] = a.x; o[1] = a.y; o[2] = a.z; o[3] = a.w;
+    o[4] = b.x; o[5] = b.y; o[6] = b.z; o[7] = b.w;
+  }
+}
+
+// 8 consecutive activations at element i (16-byte aligned)
+template <class T>
+__device__ __forceinline__ void store8(void* out, size_t i, const float (&y)[8]);
+template <>
+__device__ __forceinline__ void store8<float>(void* out, size_t i, const float (&y)[8]) {
+  float4* p = reinterpret_cast<float4*>(static_cast<float*>(out) + i);
+  p[0] = make_float4(y[0], y[1], y[2], y[3]);
+  p[1] = make_float4(y[4], y[5], y[6], y[7]);
+}
+template <>
+__device__ __forceinline__ void store8<bf16>(void* out, size_t i, const float (&y)[8]) {
+  uint32_t pk[4];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    __nv_bfloat162 t = __floats2bfloat162_rn(y[2 * q], y[2 * q + 1]);
+    pk[q] = *reinterpret_cast<uint32_t*>(&t);
+  }
+  *reinterpret_cast<uint4*>(static_cast<bf16*>(out) + i) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+}
+
+// ln_pair_kernel for d = 256 NCH with the row in registers
+template <class T, int NCH>
+__global__ void __launch_bounds__(WPB * 32) ln_pair_reg_kernel(const float* __restrict__ c, const float* __restrict__ h,
+                                                               int M, const void* wc, const void* bc, const void* wh,
+                                                               const void* bh, int w_bf16, float eps,
+                                                               void* __restrict__ u) {
+  pdl_enter();
+  constexpr int d = 256 * NCH;
+  const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (m >= M) return;
+#pragma unroll
+  for (int part = 0; part < 2; ++part) {
+    const float* xr = (part ? h : c) + static_cast<size_t>(m) * d;
+    const void* w = part ? wh : wc;
+    const void* b = part ? bh : bc;
+    float v[NCH][8], mean, rstd;
+    ln_row_reg<NCH>(xr, lane, eps, v, mean, rstd);
+#pragma unroll
+    for (int ch = 0; ch < NCH; ++ch) {
+      const int j = (ch * 32 + lane) * 8;
+      float wv[8], bv[8], y[8];
+      ldw8(w, w_bf16, j, wv);
+      ldw8(b, w_bf16, j, bv);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) y[i] = (v[ch][i] - mean) * rstd * wv[i] + bv[i];
+      store8<T>(u, static_cast<size_t>(m) * 2 * d + part * d + j, y);
+    }
+  }
+}
+
+// layernorm_kernel for d = 256 NCH with the row in registers
+template <int NCH>
+__global__ void __launch_bounds__(WPB * 32) layernorm_reg_kernel(const float* __restrict__ x, int M, const void* w,
+                                                                 const void* b, int w_bf16, float eps,
+                                                                 float* __restrict__ out) {
+  pdl_enter();
+  constexpr int d = 256 * NCH;
+  const int m = blockIdx.x * WPB + (threadIdx.x >> 5), lane = threadIdx.x & 31;
+  if (m >= M) return;
+  float v[NCH][8], mean, rstd;
+  ln_row_reg<NCH>(x + static_cast<size_t>(m) * d, lane, eps, v, mean, rstd);
+#pragma unroll
+  for (int ch = 0; ch < NCH; ++ch) {
+    const int j = (ch * 32 + lane) * 8;
+    float wv[8], bv[8], y[8];
+    ldw8(w, w_bf16, j, wv);
+    ldw8(b, w_bf16, j, bv);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) y[i] = (v[ch][i] - mean) * rstd * wv[i] + bv[i];
+    store8<float>(out, static_cast<size_t>(m) * d + j, y);
   }
 }
 
@@ -495,9 +618,34 @@ const char* rmsnorm_rows(const float* x, int M, int d, const void* gain, int w_b
   return err();
 }
 
+// true when every pointer is 16-byte aligned (the register kernels' vector accesses)
+static bool all16(std::initializer_list<const void*> ps) {
+  for (const void* p : ps)
+    if (reinterpret_cast<uintptr_t>(p) & 15) return false;
+  return true;
+}
+
+template <class T>
+static bool ln_pair_reg(const float* c, const float* h, int M, int d, const void* wc, const void* bc, const void* wh,
+                 const void* bh, int w_bf16, float eps, void* u, cudaStream_t s) {
+  switch (d) {
+    case 256: launch_pdl(ln_pair_reg_kernel<T, 1>, rows_grid(M), WPB * 32, 0, s, c, h, M, wc, bc, wh, bh, w_bf16, eps, u); return true;
+    case 512: launch_pdl(ln_pair_reg_kernel<T, 2>, rows_grid(M), WPB * 32, 0, s, c, h, M, wc, bc, wh, bh, w_bf16, eps, u); return true;
+    case 768: launch_pdl(ln_pair_reg_kernel<T, 3>, rows_grid(M), WPB * 32, 0, s, c, h, M, wc, bc, wh, bh, w_bf16, eps, u); return true;
+    case 1024: launch_pdl(ln_pair_reg_kernel<T, 4>, rows_grid(M), WPB * 32, 0, s, c, h, M, wc, bc, wh, bh, w_bf16, eps, u); return true;
+    case 2048: launch_pdl(ln_pair_reg_kernel<T, 8>, rows_grid(M), WPB * 32, 0, s, c, h, M, wc, bc, wh, bh, w_bf16, eps, u); return true;
+    default: return false;
+  }
+}
+
 const char* ln_pair_rows(const float* c, const float* h, int M, int d, const void* wc, const void* bc, const void* wh,
                          const void* bh, int w_bf16, float eps, void* u, int act_bf16, cudaStream_t s) {
   if (M <= 0) return nullptr;
+  if (all16({c, h, wc, bc, wh, bh, u})) {
+    const bool done = act_bf16 ? ln_pair_reg<bf16>(c, h, M, d, wc, bc, wh, bh, w_bf16, eps, u, s)
+                               : ln_pair_reg<float>(c, h, M, d, wc, bc, wh, bh, w_bf16, eps, u, s);
+    if (done) return err();
+  }
   if (act_bf16)
     launch_pdl(ln_pair_kernel<bf16>, rows_grid(M), WPB * 32, 0, s, c, h, M, d, wc, bc, wh, bh, w_bf16, eps, u);
   else
@@ -508,6 +656,16 @@ const char* ln_pair_rows(const float* c, const float* h, int M, int d, const voi
 const char* layernorm_rows(const float* x, int M, int d, const void* w, const void* b, int w_bf16, float eps,
                            float* out, cudaStream_t s) {
   if (M <= 0) return nullptr;
+  if (all16({x, w, b, out})) {
+    switch (d) {
+      case 256: launch_pdl(layernorm_reg_kernel<1>, rows_grid(M), WPB * 32, 0, s, x, M, w, b, w_bf16, eps, out); return err();
+      case 512: launch_pdl(layernorm_reg_kernel<2>, rows_grid(M), WPB * 32, 0, s, x, M, w, b, w_bf16, eps, out); return err();
+      case 768: launch_pdl(layernorm_reg_kernel<3>, rows_grid(M), WPB * 32, 0, s, x, M, w, b, w_bf16, eps, out); return err();
+      case 1024: launch_pdl(layernorm_reg_kernel<4>, rows_grid(M), WPB * 32, 0, s, x, M, w, b, w_bf16, eps, out); return err();
+      case 2048: launch_pdl(layernorm_reg_kernel<8>, rows_grid(M), WPB * 32, 0, s, x, M, w, b, w_bf16, eps, out); return err();
+      default: break;
+    }
+  }
   launch_pdl(layernorm_kernel, rows_grid(M), WPB * 32, 0, s, x, M, d, w, b, w_bf16, eps, out);
   return err();
 }
