@@ -460,7 +460,7 @@ def test_block_mode_fp32_positions_and_context_exact(T):
 
 @pytest.mark.parametrize("case", ["small_workload_dims", "small_workload_dims_qkv_split", "test_model"])
 def test_committed_token_agreement_teacher_forced(T, case):
-    """North-star token agreement on a large sample: the GPU generates step by
+    """Teacher-forced token agreement on a large sample: the GPU generates step by
     step; at every step the oracle receives the same canvas (teacher forcing)
     and predicts the tokens at the positions the GPU commits.
 
@@ -473,7 +473,7 @@ def test_committed_token_agreement_teacher_forced(T, case):
     confidence-selected commits as that ideal bf16 path.
     small_workload_dims_qkv_split: the same model with the QKV projections'
     input split into bf16 hi + lo (qkv_split), the site that carries most of
-    the flips (the floor's per-site runs); the benchmark spec's bound, >= 99.5%.
+    the flips (the floor's per-site runs); the 99.5 % agreement bound.
     test_model: the 4-layer d 256 vocab 4096 test model, batch 16 (>= 99%).
     Forced commits (last step of the block) are reported."""
     floor = None
