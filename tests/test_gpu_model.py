@@ -1,6 +1,6 @@
 """Model-level parity on the GPU through the C ABI against the CPU oracle.
 
-Tolerances (the benchmark spec): per-step logits rel-L2 <= 2e-2 for bf16 models
+Tolerances: per-step logits rel-L2 <= 2e-2 for bf16 models
 (1e-4 for fp32 models); tokens committed by the sampler from the same canvas
 agree; argmax over all positions agrees on >= 95% for bf16 (random-init
 logits have top-1/top-2 gaps of ~0.2 sigma, so bf16 rounding flips a few
