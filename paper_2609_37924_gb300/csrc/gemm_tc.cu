@@ -718,6 +718,34 @@ const char* gemm_tc(const GemmCall& g, cudaStream_t s) {
       return nullptr;
     }
   }
+  // QKV GEMMs of the same regime (whose 256 x 128 pair tiles re-read the
+  // activation operand once per cluster) likewise: 256-wide pair tiles with
+  // split-K; the QKV epilogue (QK-norm, RoPE, Q / K / V writes) runs in the
+  // split-K reduction on the slice-ordered sum.
+  if (narrow && g.epi == EPI_QKV && g.split_buf && !g.m_dev && kblocks >= 16) {
+    const int pu = m_pairs * a.n_tiles_n;
+    int sp = std::min(std::min((g_num_sms / 2) / pu, kblocks / 8), 16);
+    const size_t per = static_cast<size_t>(g.M) * a.ldp * sizeof(float);
+    while (sp > 1 && sp * per > g.split_bytes) --sp;
+    if (sp > 1) {
+      CUtensorMap tbh;
+      if (!make_map(&tbh, g.B, b_rows, k_b, g.ldb, BN / 2)) return "tensor map (B, half tiles) encode failed";
+      TcArgs a2 = a;
+      a2.kb_per_split = (kblocks + sp - 1) / sp;
+      a2.splits = (kblocks + a2.kb_per_split - 1) / a2.kb_per_split;
+      a2.part = g.split_buf;
+      a2.part_stride = static_cast<size_t>(g.M) * a2.ldp;
+      a2.staged = 0;
+      const cudaError_t e = launch_epi_pair<EPI_QKV>(ta, tbh, tc, tc2, a2, pu * a2.splits, s);
+      if (e != cudaSuccess) return cudaGetErrorString(e);
+      const_cast<GemmCall&>(g).launched = 1;
+      int nr = 0;
+      const char* r = splitk_reduce(g.epi, a2.ep, a2.part, a2.part_stride, a2.ldp, a2.splits, a2.n_tiles_n, s, &nr);
+      if (r) return r;
+      const_cast<GemmCall&>(g).launched = 1 + nr;
+      return nullptr;
+    }
+  }
   if (g.split_buf && !g.m_dev && !pairs_fill && tiles * 3 < g_num_sms * 2 && kblocks >= 8) {
     int sp = std::min(std::min(g_num_sms / tiles, kblocks / 4), 16);
     const size_t per = static_cast<size_t>(g.M) * a.ldp * sizeof(float);

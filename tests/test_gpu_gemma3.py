@@ -135,6 +135,47 @@ def test_gemma3_fp32_block_mode_exact(T):
     assert float(np.mean(got == ref)) >= 0.99
 
 
+def test_gemma3_bf16_block_mode_split_k_projections(T):
+    """bf16 Gemma-3 model (QK-norm, sandwich norms, a 48-key window) in block
+    mode at batch 8 x 32-row blocks, d_model 1024: its 256-row QKV
+    projections (split operand, K = 2048) run 256-wide CTA-pair tiles with
+    split-K and the QKV epilogue in the ordered split-K reduction, and so do
+    its 320-row prefill projections (the second pair tile ragged); the
+    fp32-store sandwich projections split-K with the element-wise reduction.
+    Teacher-forced steps (both sides continue from the oracle's canvas)
+    across a commit."""
+    m = wl.ModelConfig(vocab=2048, d_model=1024, n_heads=8, n_kv_heads=4, head_dim=64, ffn=2048, n_shared=1,
+                       n_anchor=2, n_denoise=1, dtype="bf16", sliding_window=48, qkv_split=True, **G3)
+    B, P, bl, Tn = 8, 40, 32, 4
+    w = wl.Workload("t", m, batch=B, prompt_len=P, gen_len=2 * bl, steps_per_block=Tn, K=2, block_len=bl)
+    tm, o = _setup(T, m, B, max(P, bl), max_ctx=P + 2 * bl)
+    prompts = wl.make_prompts(w, batch=B, seed=9)
+    tm.tadm_reset(B)
+    tm.tadm_prefill(torch.from_numpy(prompts).cuda())
+    sess = o.new_session(B)
+    o.prefill(sess, prompts)
+    cache = tm.new_cache(B, bl)
+    worst = 0.0
+    for blk in range(2):
+        zb = np.full((B, bl), m.mask_id, np.int32)
+        for n in range(Tn):
+            if n % 2 == 0:
+                tm.tadm_anchor_forward(torch.from_numpy(zb).cuda(), Tn - n, cache)
+                cache_o = o.anchor_forward(sess, zb)
+            gz, gl, gt = _step(tm, zb, Tn - n, Tn, bl, cache)
+            ref = o.denoise_step(sess, zb, cache_o, n, Tn, bl)
+            rel = rel_l2(gl, ref["logits"])
+            worst = max(worst, rel)
+            assert rel < 2e-2, (blk, n, rel)
+            masked = zb == m.mask_id
+            assert float(np.mean(gt[masked] == ref["tok"][masked])) >= 0.95, (blk, n)
+            zb = ref["z"]
+        tm.tadm_commit_block(torch.from_numpy(zb).cuda())
+        o.commit_block(sess, zb)
+    tm.tadm_sync_status()
+    print(f"[gemma3 bf16 block mode, split-K projections] worst logits rel-L2 {worst:.3e}")
+
+
 @pytest.mark.parametrize("fusion", ["gated_mlp", "paired_attn"])
 def test_gemma3_bf16_single_block_stale_step(T, fusion):
     """bf16 model on tcgen05 (QK-norm in the QKV epilogue, sandwich norms,
